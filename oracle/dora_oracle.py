@@ -1,0 +1,322 @@
+"""Plain fp64 CPU oracle for DORA's deployment hot path.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import, call or
+link this module: only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` use it.  It shares
+no code with the CUDA path (no kernels, headers, helpers or tables).
+
+Every function computes the plain definition of one step of the pruned ViT
+block of Eq. 1 (Sec. 3.1), in float64, from bf16/fp32 inputs decoded exactly:
+
+* ``select_keep``   deterministic deletion of the k highest selector scores,
+                    CLS kept, survivor order kept (Sec. 3.2 "Sampling and
+                    deployment"; Appendix A.3).
+* ``compact``       hard deletion into a packed buffer with explicit sequence
+                    boundaries (Sec. 3.1 pruning operator; Sec. 3.5
+                    "Inference").
+* ``varlen_attention``  softmax(Q K^T * scale) V within each image only
+                    (Sec. 3.5 "Inference": boundaries prevent attention
+                    between different images).
+* ``layernorm``, ``linear``, ``gelu``  the standard pre-LN ViT block pieces
+                    (Eq. 1; backbones of Sec. 4.1).
+* ``pruned_block``  Eq. 1: attention over all N_l+1 tokens, residual, delete,
+                    LayerNorm', MLP on survivors, residual.
+* ``forward``       Eq. 1 applied block after block.
+
+Readings where the paper is silent (all listed in the design doc):
+
+* Ties: among equal scores the lower index is kept (equivalently the higher
+  index is removed first).  Scores are ordered by a total order on fp32:
+  -0 equals +0, and every NaN sorts above +inf (removed first).
+* ``keep_counts`` include CLS; a count outside [1, n] is clamped and status 5
+  is reported.
+* LayerNorm uses the biased variance; GELU is the exact erf form; the qkv row
+  layout is [3][H][head_dim]; the default softmax scale is 1/sqrt(head_dim).
+
+Parity pins: every function here is checked in ``tests/test_oracle_pins.py``
+against brute force, closed forms, invariants the paper fixes, or an
+independent library routine.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+DORA_OK = 0
+DORA_ERR_DEVICE_BAD_COUNT = 5
+
+
+# ----------------------------------------------------------------------------
+# decoding (exact)
+# ----------------------------------------------------------------------------
+
+def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Exact value of bf16 bit patterns (uint16) as float64."""
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return u.view(np.float32).astype(np.float64)
+
+
+# ----------------------------------------------------------------------------
+# O1: selection (Sec. 3.2 "Sampling and deployment"; Appendix A.3)
+# ----------------------------------------------------------------------------
+
+def score_order_key(scores: np.ndarray) -> np.ndarray:
+    """Map fp32 scores to uint32 keys whose unsigned order is the score order.
+
+    Total order used for the deterministic top-k: -0.0 and +0.0 are equal, every
+    NaN is larger than +inf.  For a non-NaN float with bits b the key is
+    ``~b`` when the sign bit is set and ``b | 0x80000000`` otherwise, which
+    makes unsigned comparison of keys agree with real comparison of values.
+    """
+    s = np.ascontiguousarray(np.asarray(scores, dtype=np.float32))
+    b = s.view(np.uint32).copy()
+    b[b == np.uint32(0x80000000)] = np.uint32(0)
+    neg = (b >> np.uint32(31)) == 1
+    key = np.where(neg, ~b, b | np.uint32(0x80000000)).astype(np.uint32)
+    key[np.isnan(s)] = np.uint32(0xFFFFFFFF)
+    return key
+
+
+def select_keep(scores: np.ndarray, cu_in: np.ndarray, keep_counts: np.ndarray):
+    """Deterministic deployment selection, one image at a time.
+
+    For image i with rows [cu_in[i], cu_in[i+1]) (n rows, local row 0 = CLS) and
+    m = keep_counts[i] tokens to keep (CLS included), the k = n - m visual tokens
+    with the highest deletion scores are removed; CLS is never a candidate.
+    Equal scores: the lower local index is kept.  Kept rows are emitted in
+    ascending order as global row indices of the input packed buffer.
+
+    Returns ``(kept_idx int32[T_out], cu_out int32[B+1], status)``.
+    """
+    cu_in = np.asarray(cu_in, dtype=np.int64)
+    keep_counts = np.asarray(keep_counts, dtype=np.int64)
+    batch = len(cu_in) - 1
+    key = score_order_key(scores)
+    status = DORA_OK
+    kept_all = []
+    cu_out = np.zeros(batch + 1, dtype=np.int64)
+    for i in range(batch):
+        lo, hi = int(cu_in[i]), int(cu_in[i + 1])
+        n = hi - lo
+        m = int(keep_counts[i])
+        m_eff = min(max(m, min(1, n)), n)
+        if m_eff != m:
+            status = DORA_ERR_DEVICE_BAD_COUNT
+        if n > 0 and m_eff > 0:
+            j = np.arange(1, n, dtype=np.int64)            # visual candidates
+            cand_key = key[lo + 1:hi].astype(np.int64)
+            order = np.lexsort((j, cand_key))               # by key, then index
+            keep_local = np.sort(np.concatenate(([0], j[order[:m_eff - 1]])))
+            kept_all.append(lo + keep_local)
+        cu_out[i + 1] = cu_out[i] + m_eff
+    kept = np.concatenate(kept_all) if kept_all else np.zeros(0, dtype=np.int64)
+    return kept.astype(np.int32), cu_out.astype(np.int32), status
+
+
+# ----------------------------------------------------------------------------
+# O2: compaction (Sec. 3.1 pruning operator; Sec. 3.5 "Inference")
+# ----------------------------------------------------------------------------
+
+def compact(x: np.ndarray, kept_idx: np.ndarray, ids_in: np.ndarray | None = None):
+    """Packed survivors: ``packed[r] = x[kept_idx[r]]`` bit for bit.
+
+    ``x`` may hold raw bf16 bits (uint16) or any dtype; rows are copied
+    unchanged.  Original token ids are carried the same way.
+    """
+    kept_idx = np.asarray(kept_idx, dtype=np.int64)
+    packed = np.asarray(x)[kept_idx].copy()
+    ids_out = None if ids_in is None else np.asarray(ids_in)[kept_idx].copy()
+    return packed, ids_out
+
+
+def cu_from_counts(counts: np.ndarray) -> np.ndarray:
+    """Sequence boundaries of a packed buffer: exclusive prefix sum, int32 [B+1]."""
+    out = np.zeros(len(counts) + 1, dtype=np.int64)
+    for i, c in enumerate(counts):
+        out[i + 1] = out[i] + int(c)
+    return out.astype(np.int32)
+
+
+# ----------------------------------------------------------------------------
+# O3: packed variable-length attention (Sec. 3.5 "Inference")
+# ----------------------------------------------------------------------------
+
+def attention_single(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float):
+    """softmax(q k^T * scale) v for one image and one head, float64.
+
+    Returns ``(O, P)`` where P is the row-stochastic attention matrix.
+    """
+    s = (q @ k.T) * scale
+    s = s - s.max(axis=1, keepdims=True)
+    e = np.exp(s)
+    p = e / e.sum(axis=1, keepdims=True)
+    return p @ v, p
+
+
+def varlen_attention(qkv: np.ndarray, cu: np.ndarray, heads: int, head_dim: int = 64,
+                     scale: float | None = None) -> np.ndarray:
+    """Multi-head self-attention restricted to each image's rows.
+
+    ``qkv`` is [T, 3*heads*head_dim] (bf16 bits or float); row layout
+    [3][heads][head_dim] = (q, k, v).  Output [T, heads*head_dim] float64.
+    Rows beyond cu[-1] are left at zero.
+    """
+    if scale is None or scale == 0.0:
+        scale = 1.0 / math.sqrt(head_dim)
+    a = bf16_to_f64(qkv) if np.asarray(qkv).dtype == np.uint16 else np.asarray(qkv, np.float64)
+    t = a.shape[0]
+    a = a.reshape(t, 3, heads, head_dim)
+    out = np.zeros((t, heads, head_dim))
+    cu = np.asarray(cu, dtype=np.int64)
+    for i in range(len(cu) - 1):
+        lo, hi = int(cu[i]), int(cu[i + 1])
+        if hi <= lo:
+            continue
+        for h in range(heads):
+            o, _ = attention_single(a[lo:hi, 0, h], a[lo:hi, 1, h], a[lo:hi, 2, h], scale)
+            out[lo:hi, h] = o
+    return out.reshape(t, heads * head_dim)
+
+
+def padded_masked_attention(qkv: np.ndarray, cu: np.ndarray, heads: int, head_dim: int = 64,
+                            scale: float | None = None) -> np.ndarray:
+    """The same attention computed the padded way: every image padded to the
+    longest, keys beyond each image's length masked with -inf.  Used only to pin
+    ``varlen_attention`` (Sec. 3.5: packing removes batch-wide padding but must
+    not change the result)."""
+    if scale is None or scale == 0.0:
+        scale = 1.0 / math.sqrt(head_dim)
+    a = bf16_to_f64(qkv) if np.asarray(qkv).dtype == np.uint16 else np.asarray(qkv, np.float64)
+    t = a.shape[0]
+    a = a.reshape(t, 3, heads, head_dim)
+    cu = np.asarray(cu, dtype=np.int64)
+    b = len(cu) - 1
+    lens = cu[1:] - cu[:-1]
+    nmax = int(lens.max()) if b else 0
+    pad = np.zeros((b, nmax, 3, heads, head_dim))
+    for i in range(b):
+        pad[i, :lens[i]] = a[cu[i]:cu[i + 1]]
+    q = pad[:, :, 0].transpose(0, 2, 1, 3)        # [B, H, n, d]
+    k = pad[:, :, 1].transpose(0, 2, 1, 3)
+    v = pad[:, :, 2].transpose(0, 2, 1, 3)
+    s = np.einsum("bhqd,bhkd->bhqk", q, k) * scale
+    keymask = np.arange(nmax)[None, :] < lens[:, None]          # [B, n]
+    s = np.where(keymask[:, None, None, :], s, -np.inf)
+    s = s - s.max(axis=-1, keepdims=True)
+    e = np.exp(s)
+    p = e / e.sum(axis=-1, keepdims=True)
+    o = np.einsum("bhqk,bhkd->bhqd", p, v).transpose(0, 2, 1, 3)  # [B, n, H, d]
+    out = np.zeros((t, heads, head_dim))
+    for i in range(b):
+        out[cu[i]:cu[i + 1]] = o[i, :lens[i]]
+    return out.reshape(t, heads * head_dim)
+
+
+# ----------------------------------------------------------------------------
+# O4: block pieces and the pruned block (Eq. 1)
+# ----------------------------------------------------------------------------
+
+def layernorm(x: np.ndarray, w: np.ndarray, b: np.ndarray, eps: float) -> np.ndarray:
+    """Row LayerNorm with biased variance and affine ``w``, ``b`` (float64)."""
+    x = np.asarray(x, dtype=np.float64)
+    mu = x.mean(axis=1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=1, keepdims=True)
+    return (x - mu) / np.sqrt(var + eps) * w + b
+
+
+def linear(x: np.ndarray, w: np.ndarray, b: np.ndarray) -> np.ndarray:
+    """nn.Linear: ``y = x W^T + b`` with ``W`` stored [out, in]."""
+    return np.asarray(x, np.float64) @ np.asarray(w, np.float64).T + b
+
+
+_ERF = np.vectorize(math.erf, otypes=[np.float64])
+
+
+def gelu(x: np.ndarray) -> np.ndarray:
+    """Exact GELU, 0.5 x (1 + erf(x / sqrt 2))."""
+    x = np.asarray(x, dtype=np.float64)
+    return 0.5 * x * (1.0 + _ERF(x / math.sqrt(2.0)))
+
+
+def decode_weights(w: dict) -> dict:
+    """bf16-bit weight dict (as produced by the synthetic generator) to float64."""
+    return {k: bf16_to_f64(v) for k, v in w.items()}
+
+
+def block_attention_half(x: np.ndarray, cu: np.ndarray, wf: dict, heads: int, eps: float,
+                         head_dim: int = 64) -> np.ndarray:
+    """First line of Eq. 1: H_attn = H + Attention(LayerNorm(H)), attention
+    including its output projection, over all tokens of each image."""
+    xn = layernorm(x, wf["ln1_w"], wf["ln1_b"], eps)
+    qkv = linear(xn, wf["w_qkv"], wf["b_qkv"])
+    o = varlen_attention(qkv, cu, heads, head_dim)
+    return x + linear(o, wf["w_proj"], wf["b_proj"])
+
+
+def block_mlp_half(h_keep: np.ndarray, wf: dict, eps: float) -> np.ndarray:
+    """Second line of Eq. 1: H_{l+1} = H_keep + MLP(LayerNorm'(H_keep))."""
+    y = linear(layernorm(h_keep, wf["ln2_w"], wf["ln2_b"], eps), wf["w_fc1"], wf["b_fc1"])
+    y = linear(gelu(y), wf["w_fc2"], wf["b_fc2"])
+    return h_keep + y
+
+
+def pruned_block(x: np.ndarray, cu_in: np.ndarray, ids_in: np.ndarray, wf: dict, heads: int,
+                 eps: float, scores: np.ndarray | None = None,
+                 keep_counts: np.ndarray | None = None, head_dim: int = 64) -> dict:
+    """One ViT block with optional hard pruning, Eq. 1.
+
+    ``x`` is float64 [T_in, D] (decode bf16 inputs first).  Deletion happens
+    after the attention residual and before LayerNorm' (Eq. 1; Appendix A.3),
+    so deleted tokens take part in this block's attention only.  Returns a dict
+    with ``x_out``, ``cu_out``, ``ids_out``, ``kept_idx`` (None without pruning),
+    ``h_attn`` and ``status``.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    h_attn = block_attention_half(x, cu_in, wf, heads, eps, head_dim)
+    status = DORA_OK
+    if scores is None:
+        kept, cu_out, h_keep, ids_out = None, np.asarray(cu_in, np.int32), h_attn, ids_in
+    else:
+        kept, cu_out, status = select_keep(scores, cu_in, keep_counts)
+        h_keep, ids_out = compact(h_attn, kept, ids_in)
+    x_out = block_mlp_half(h_keep, wf, eps)
+    return dict(x_out=x_out, cu_out=cu_out, ids_out=ids_out, kept_idx=kept,
+                h_attn=h_attn, status=status)
+
+
+# ----------------------------------------------------------------------------
+# O5: the whole pruned forward (Eq. 1 block after block)
+# ----------------------------------------------------------------------------
+
+def gather_scores(table: np.ndarray, cu: np.ndarray, ids: np.ndarray) -> np.ndarray:
+    """Row-aligned scores from a per-image table indexed by original token id.
+
+    Stand-in for the actor's selector output (Eq. 2): each surviving row gets
+    the score its image's table assigns to that token's original id.
+    """
+    cu = np.asarray(cu, dtype=np.int64)
+    out = np.zeros(int(cu[-1]), dtype=np.float32)
+    for i in range(len(cu) - 1):
+        out[cu[i]:cu[i + 1]] = table[i, ids[cu[i]:cu[i + 1]]]
+    return out
+
+
+def forward(x: np.ndarray, cu: np.ndarray, ids: np.ndarray, blocks: list, heads: int,
+            eps: float, prune: dict | None = None, head_dim: int = 64) -> dict:
+    """Eq. 1 over all blocks.  ``blocks`` is a list of float64 weight dicts;
+    ``prune`` maps block index to ``(score_table, keep_counts)``.  Returns the
+    final ``x``, ``cu``, ``ids`` and the list of per-block ``kept_idx``."""
+    prune = prune or {}
+    x = np.asarray(x, dtype=np.float64)
+    kept_hist = []
+    for l, wf in enumerate(blocks):
+        if l in prune:
+            table, keep = prune[l]
+            s = gather_scores(table, cu, ids)
+            r = pruned_block(x, cu, ids, wf, heads, eps, s, keep, head_dim)
+        else:
+            r = pruned_block(x, cu, ids, wf, heads, eps, None, None, head_dim)
+        x, cu, ids = r["x_out"], r["cu_out"], r["ids_out"]
+        kept_hist.append(r["kept_idx"])
+    return dict(x=x, cu=cu, ids=ids, kept=kept_hist)

@@ -1,0 +1,412 @@
+"""Pins for the fp64 oracle: each check comes from outside the oracle itself
+(brute force, closed forms, invariants the paper fixes, an independent library
+routine, or values the paper prints)."""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import dora_synth as S
+import oracle as O
+
+pytestmark = pytest.mark.filterwarnings("ignore::RuntimeWarning")
+
+
+# ---------------------------------------------------------------------------
+# selection (Sec. 3.2 "Sampling and deployment"; Appendix A.3)
+# ---------------------------------------------------------------------------
+
+def _removal_before(a_score, a_idx, b_score, b_idx):
+    """True when token a is removed before token b, by the rule written with
+    Python float semantics: larger score first, NaN largest of all, equal
+    scores (including -0 == +0) remove the higher index first."""
+    an, bn = math.isnan(a_score), math.isnan(b_score)
+    if an or bn:
+        if an and bn:
+            return a_idx > b_idx
+        return an
+    if a_score != b_score:
+        return a_score > b_score
+    return a_idx > b_idx
+
+
+def _brute_force_keep(scores, m):
+    """Enumerate every subset of visual tokens of size m-1 and return the unique
+    one such that every kept token would be removed after every removed one."""
+    n = len(scores)
+    vis = list(range(1, n))
+    valid = []
+    for keep in itertools.combinations(vis, m - 1):
+        ks = set(keep)
+        removed = [j for j in vis if j not in ks]
+        if all(_removal_before(scores[r], r, scores[k], k) for r in removed for k in keep):
+            valid.append([0] + list(keep))
+    assert len(valid) == 1, valid
+    return valid[0]
+
+
+def _select_one(scores, m):
+    s = np.asarray(scores, dtype=np.float32)
+    kept, cu_out, st = O.select_keep(s, np.array([0, len(s)]), np.array([m]))
+    return kept.tolist(), cu_out.tolist(), st
+
+
+def test_select_brute_force_small():
+    rng = np.random.default_rng(1)
+    palette = np.array([0.0, -0.0, 0.25, 0.5, -1.0, np.inf, -np.inf, np.nan, 1e-30],
+                       dtype=np.float32)
+    for trial in range(300):
+        n = int(rng.integers(1, 10))
+        if trial % 3 == 0:
+            s = rng.choice(palette, size=n)
+        else:
+            s = rng.random(n).astype(np.float32)
+        for m in range(1, n + 1):
+            kept, cu_out, st = _select_one(s, m)
+            assert kept == _brute_force_keep([float(v) for v in s], m)
+            assert cu_out == [0, m] and st == 0
+
+
+def test_select_golden_cases(golden_dir):
+    with open(os.path.join(golden_dir, "select_cases.txt")) as f:
+        lines = [ln.strip() for ln in f if ln.strip() and not ln.startswith("#")]
+    assert len(lines) >= 8
+    for ln in lines:
+        s_txt, m_txt, k_txt = [p.strip() for p in ln.split("|")]
+        s = [float(v) for v in s_txt.split(",")]
+        kept, _, st = _select_one(s, int(m_txt))
+        assert kept == [int(v) for v in k_txt.split(",")], ln
+        assert st == 0
+
+
+def test_select_distinct_equals_partial_sort():
+    rng = np.random.default_rng(2)
+    for _ in range(50):
+        n = int(rng.integers(2, 600))
+        s = rng.permutation(n).astype(np.float32) - n / 2   # distinct
+        m = int(rng.integers(1, n + 1))
+        kept, _, _ = _select_one(s, m)
+        vis = s[1:]
+        k = n - m
+        removed = set((np.argsort(-vis, kind="stable")[:k] + 1).tolist())
+        expect = [j for j in range(n) if j not in removed]
+        assert kept == expect
+
+
+def test_select_all_equal_keeps_prefix():
+    for n in (1, 2, 17, 197, 577):
+        for m in sorted({1, min(2, n), n // 2 or 1, n}):
+            kept, _, _ = _select_one(np.full(n, 0.5), m)
+            assert kept == list(range(m))
+
+
+def test_select_invariants_all_configs():
+    for name in ("cfg1", "cfg2", "cfg3", "cfg4", "cfg5"):
+        cfg = S.get_config(name, batch=min(S.get_config(name).batch, 32))
+        cu, ids = S.initial_layout(cfg)
+        keeps, befores = S.keep_schedule(cfg, seed=3)
+        table = S.score_table(cfg, cfg.prune_blocks[0], seed=3)
+        scores = O.gather_scores(table, cu, ids)
+        kept, cu_out, st = O.select_keep(scores, cu, keeps[0])
+        assert st == 0
+        assert np.array_equal(cu_out, O.cu_from_counts(keeps[0]))
+        for i in range(cfg.batch):
+            seg = kept[cu_out[i]:cu_out[i + 1]]
+            assert len(seg) == keeps[0][i]                 # |kept| = N_i - k_i
+            assert seg[0] == cu[i]                         # CLS retained
+            assert np.all(np.diff(seg) > 0)                # order preserved
+            assert seg[-1] < cu[i + 1]
+
+
+def test_select_clamps_bad_counts():
+    s = np.random.default_rng(4).random(10).astype(np.float32)
+    cu = np.array([0, 4, 10])
+    kept, cu_out, st = O.select_keep(s, cu, np.array([0, 11]))
+    assert st == O.DORA_ERR_DEVICE_BAD_COUNT
+    assert cu_out.tolist() == [0, 1, 7]
+    assert kept[0] == 0 and kept[1:].tolist() == list(range(4, 10))
+    # empty image: nothing kept, count 0 is fine
+    kept, cu_out, st = O.select_keep(s[:3], np.array([0, 0, 3]), np.array([0, 2]))
+    assert st == 0 and cu_out.tolist() == [0, 0, 2]
+
+
+# ---------------------------------------------------------------------------
+# compaction
+# ---------------------------------------------------------------------------
+
+def test_compact_matches_naive_copy():
+    rng = np.random.default_rng(5)
+    x = rng.integers(0, 65536, size=(50, 24), dtype=np.uint16)
+    ids = rng.integers(0, 1000, size=50).astype(np.int32)
+    kept = np.sort(rng.choice(50, size=20, replace=False)).astype(np.int32)
+    packed, ids_out = O.compact(x, kept, ids)
+    for r, src in enumerate(kept):
+        assert packed[r].tobytes() == x[src].tobytes()
+        assert ids_out[r] == ids[src]
+
+
+def test_cu_from_counts_closed_form():
+    counts = np.array([3, 0, 5, 1])
+    assert O.cu_from_counts(counts).tolist() == [0, 3, 3, 8, 9]
+    c = np.random.default_rng(6).integers(0, 300, size=200)
+    cu = O.cu_from_counts(c)
+    assert cu[-1] == c.sum() and np.all(np.diff(cu) == c)
+
+
+# ---------------------------------------------------------------------------
+# attention (Sec. 3.5 "Inference")
+# ---------------------------------------------------------------------------
+
+def _rand_qkv(t, h, rng, d=64):
+    return rng.standard_normal((t, 3 * h * d))
+
+
+def test_attention_single_token_returns_v():
+    rng = np.random.default_rng(7)
+    qkv = _rand_qkv(1, 2, rng)
+    out = O.varlen_attention(qkv, np.array([0, 1]), 2)
+    v = qkv.reshape(1, 3, 2, 64)[:, 2].reshape(1, 128)
+    assert np.allclose(out, v, atol=0, rtol=1e-15)
+
+
+def test_attention_constant_v_and_identical_keys():
+    rng = np.random.default_rng(8)
+    n, h = 13, 3
+    qkv = _rand_qkv(n, h, rng).reshape(n, 3, h, 64)
+    qkv[:, 2] = qkv[0, 2]                      # constant v
+    out = O.varlen_attention(qkv.reshape(n, -1), np.array([0, n]), h).reshape(n, h, 64)
+    assert np.max(np.abs(out - qkv[0, 2][None])) < 1e-12
+    qkv = _rand_qkv(n, h, rng).reshape(n, 3, h, 64)
+    qkv[:, 1] = qkv[0, 1]                      # identical keys -> uniform weights
+    out = O.varlen_attention(qkv.reshape(n, -1), np.array([0, n]), h).reshape(n, h, 64)
+    assert np.max(np.abs(out - qkv[:, 2].mean(axis=0)[None])) < 1e-12
+
+
+def test_attention_rows_sum_to_one():
+    rng = np.random.default_rng(9)
+    q, k, v = (rng.standard_normal((40, 64)) * 3 for _ in range(3))
+    _, p = O.attention_single(q, k, v, 0.125)
+    assert np.max(np.abs(p.sum(axis=1) - 1.0)) < 1e-12
+    assert np.all(p >= 0)
+
+
+def test_attention_matches_torch_sdpa_fp64():
+    rng = np.random.default_rng(10)
+    lens = [1, 5, 64, 129, 197]
+    cu = O.cu_from_counts(lens)
+    h = 3
+    qkv = _rand_qkv(int(cu[-1]), h, rng)
+    out = O.varlen_attention(qkv, cu, h).reshape(-1, h, 64)
+    a = torch.from_numpy(qkv.reshape(-1, 3, h, 64))
+    for i in range(len(lens)):
+        seg = a[cu[i]:cu[i + 1]]
+        q, k, v = (seg[:, j].transpose(0, 1) for j in range(3))   # [h, n, d]
+        ref = torch.nn.functional.scaled_dot_product_attention(q, k, v).transpose(0, 1)
+        assert np.max(np.abs(out[cu[i]:cu[i + 1]] - ref.numpy())) < 1e-12
+
+
+def test_varlen_equals_per_image_and_padded_mask():
+    rng = np.random.default_rng(11)
+    lens = rng.integers(1, 80, size=7)
+    cu = O.cu_from_counts(lens)
+    h = 2
+    qkv = _rand_qkv(int(cu[-1]), h, rng)
+    packed = O.varlen_attention(qkv, cu, h)
+    padded = O.padded_masked_attention(qkv, cu, h)
+    assert np.max(np.abs(packed - padded)) < 1e-12
+    for i in range(len(lens)):
+        sep = O.varlen_attention(qkv[cu[i]:cu[i + 1]], np.array([0, lens[i]]), h)
+        assert np.max(np.abs(packed[cu[i]:cu[i + 1]] - sep)) < 1e-12
+
+
+def test_unpruned_packed_equals_dense_attention():
+    """k = 0 for every image: the packed buffer is the dense batch and packed
+    attention equals dense batched attention (torch SDPA, fp64)."""
+    rng = np.random.default_rng(12)
+    b, n, h = 4, 37, 2
+    qkv = _rand_qkv(b * n, h, rng)
+    packed = O.varlen_attention(qkv, np.arange(b + 1) * n, h)
+    a = torch.from_numpy(qkv.reshape(b, n, 3, h, 64))
+    q, k, v = (a[:, :, j].permute(0, 2, 1, 3) for j in range(3))
+    dense = torch.nn.functional.scaled_dot_product_attention(q, k, v).permute(0, 2, 1, 3)
+    assert np.max(np.abs(packed - dense.reshape(b * n, h * 64).numpy())) < 1e-12
+
+
+# ---------------------------------------------------------------------------
+# LayerNorm, linear, GELU
+# ---------------------------------------------------------------------------
+
+def test_layernorm_matches_torch_and_invariants():
+    rng = np.random.default_rng(13)
+    x = rng.standard_normal((33, 96)) * 4 + 2
+    w, b = rng.standard_normal(96), rng.standard_normal(96)
+    y = O.layernorm(x, w, b, 1e-6)
+    ref = torch.nn.functional.layer_norm(torch.from_numpy(x), (96,), torch.from_numpy(w),
+                                         torch.from_numpy(b), 1e-6).numpy()
+    assert np.max(np.abs(y - ref)) < 1e-12
+    y1 = O.layernorm(x, np.ones(96), np.zeros(96), 0.0)
+    assert np.max(np.abs(y1.mean(axis=1))) < 1e-12
+    assert np.max(np.abs((y1 ** 2).mean(axis=1) - 1)) < 1e-12
+
+
+def test_linear_matches_loops():
+    rng = np.random.default_rng(14)
+    x, w, b = rng.standard_normal((3, 5)), rng.standard_normal((4, 5)), rng.standard_normal(4)
+    y = O.linear(x, w, b)
+    for r in range(3):
+        for c in range(4):
+            assert abs(y[r, c] - (sum(x[r, i] * w[c, i] for i in range(5)) + b[c])) < 1e-12
+
+
+def test_gelu_closed_forms_and_torch():
+    x = np.linspace(-8, 8, 1001)
+    ref = torch.nn.functional.gelu(torch.from_numpy(x), approximate="none").numpy()
+    assert np.max(np.abs(O.gelu(x) - ref)) < 1e-14
+    assert O.gelu(np.array([0.0]))[0] == 0.0
+    assert abs(O.gelu(np.array([10.0]))[0] - 10.0) < 1e-12
+    assert abs(O.gelu(np.array([1.0]))[0] - 0.5 * (1 + math.erf(1 / math.sqrt(2)))) < 1e-15
+
+
+# ---------------------------------------------------------------------------
+# the pruned block (Eq. 1) and the forward
+# ---------------------------------------------------------------------------
+
+def _small_cfg(**kw):
+    base = dict(batch=3, n_tokens=21, dim=128, heads=2, mlp_dim=256, depth=3,
+                prune_blocks=(1,), k_law="uniform", k_max=14)
+    base.update(kw)
+    return S.Config("tiny", **base)
+
+
+def _torch_block(x, cu, wf, heads, eps, kept=None):
+    """The same block written with torch library ops (fp64): F.layer_norm,
+    F.linear, per-image SDPA, exact GELU.  Independent of the oracle."""
+    F = torch.nn.functional
+    t = {k: torch.from_numpy(v) for k, v in wf.items()}
+    x = torch.from_numpy(x)
+    d = x.shape[1]
+    xn = F.layer_norm(x, (d,), t["ln1_w"], t["ln1_b"], eps)
+    qkv = F.linear(xn, t["w_qkv"], t["b_qkv"]).reshape(-1, 3, heads, 64)
+    o = torch.zeros(x.shape[0], heads, 64, dtype=torch.float64)
+    for i in range(len(cu) - 1):
+        seg = qkv[cu[i]:cu[i + 1]]
+        q, k, v = (seg[:, j].transpose(0, 1) for j in range(3))
+        o[cu[i]:cu[i + 1]] = F.scaled_dot_product_attention(q, k, v).transpose(0, 1)
+    h = x + F.linear(o.reshape(-1, d), t["w_proj"], t["b_proj"])
+    if kept is not None:
+        h = h[torch.from_numpy(kept.astype(np.int64))]
+    y = F.gelu(F.linear(F.layer_norm(h, (d,), t["ln2_w"], t["ln2_b"], eps), t["w_fc1"], t["b_fc1"]))
+    return (h + F.linear(y, t["w_fc2"], t["b_fc2"])).numpy()
+
+
+def _block_inputs(cfg, seed=0):
+    cu, ids = S.initial_layout(cfg)
+    x = O.bf16_to_f64(S.activations_bf16(cfg, seed))
+    wf = O.decode_weights(S.block_weights(cfg, 0, seed, random_affine=True))
+    return x, cu, ids, wf
+
+
+def test_block_matches_torch_composition():
+    cfg = _small_cfg()
+    x, cu, ids, wf = _block_inputs(cfg)
+    keeps, _ = S.keep_schedule(cfg, 0)
+    scores = O.gather_scores(S.score_table(cfg, 1, 0), cu, ids)
+    r = O.pruned_block(x, cu, ids, wf, cfg.heads, 1e-6, scores, keeps[0])
+    ref = _torch_block(x, cu, wf, cfg.heads, 1e-6, r["kept_idx"])
+    assert np.max(np.abs(r["x_out"] - ref)) < 1e-10
+    r0 = O.pruned_block(x, cu, ids, wf, cfg.heads, 1e-6)
+    assert np.max(np.abs(r0["x_out"] - _torch_block(x, cu, wf, cfg.heads, 1e-6))) < 1e-10
+
+
+def test_block_pruned_rows_equal_dense_rows():
+    """Deletion happens after the attention residual and the MLP is row-wise,
+    so the pruned block's output rows are the dense block's output rows at the
+    kept positions (Eq. 1)."""
+    cfg = _small_cfg()
+    x, cu, ids, wf = _block_inputs(cfg, seed=1)
+    keeps, _ = S.keep_schedule(cfg, 1)
+    scores = O.gather_scores(S.score_table(cfg, 1, 1), cu, ids)
+    pr = O.pruned_block(x, cu, ids, wf, cfg.heads, 1e-6, scores, keeps[0])
+    dn = O.pruned_block(x, cu, ids, wf, cfg.heads, 1e-6)
+    assert np.max(np.abs(pr["x_out"] - dn["x_out"][pr["kept_idx"]])) < 1e-12
+    assert np.array_equal(pr["ids_out"], ids[pr["kept_idx"]])
+
+
+def test_block_keep_all_equals_unpruned():
+    cfg = _small_cfg()
+    x, cu, ids, wf = _block_inputs(cfg, seed=2)
+    scores = np.random.default_rng(0).random(len(ids)).astype(np.float32)
+    full = np.full(cfg.batch, cfg.n_tokens)
+    pr = O.pruned_block(x, cu, ids, wf, cfg.heads, 1e-6, scores, full)
+    dn = O.pruned_block(x, cu, ids, wf, cfg.heads, 1e-6)
+    assert np.array_equal(pr["x_out"], dn["x_out"])
+    assert np.array_equal(pr["cu_out"], cu)
+
+
+def test_forward_k0_equals_dense_and_trajectory():
+    cfg = _small_cfg(depth=3, prune_blocks=(0, 2))
+    cu, ids = S.initial_layout(cfg)
+    x = O.bf16_to_f64(S.activations_bf16(cfg, 5))
+    blocks = [O.decode_weights(S.block_weights(cfg, l, 5)) for l in range(cfg.depth)]
+    full = np.full(cfg.batch, cfg.n_tokens)
+    tabs = {l: S.score_table(cfg, l, 5) for l in cfg.prune_blocks}
+    k0 = O.forward(x, cu, ids, blocks, cfg.heads, 1e-6, {l: (tabs[l], full) for l in tabs})
+    dense = O.forward(x, cu, ids, blocks, cfg.heads, 1e-6)
+    assert np.array_equal(k0["x"], dense["x"])
+    keeps, befores = S.keep_schedule(cfg, 5)
+    pr = O.forward(x, cu, ids, blocks, cfg.heads, 1e-6,
+                   {l: (tabs[l], keeps[j]) for j, l in enumerate(cfg.prune_blocks)})
+    assert np.array_equal(np.diff(pr["cu"]), keeps[-1])
+    for i in range(cfg.batch):
+        seg = pr["ids"][pr["cu"][i]:pr["cu"][i + 1]]
+        assert seg[0] == 0 and np.all(np.diff(seg) > 0)
+
+
+# ---------------------------------------------------------------------------
+# accounting and generator (Eq. 4, Appendix A.2, Appendix E.4, Table 1, Table 3)
+# ---------------------------------------------------------------------------
+
+def test_native_gflops_reproduce_table1(golden_dir):
+    from paper_2609_34325_gb300 import accounting as A
+    rows = [ln.split() for ln in open(os.path.join(golden_dir, "native_gflops.txt"))
+            if ln.strip() and not ln.startswith("#")]
+    assert len(rows) == 4
+    for name, gf, d, L, n0, mlp, patch, ro in rows:
+        ours = A.native_gflops(int(n0) + 1, int(d), int(mlp), int(L), int(patch),
+                               readout_mult=int(ro))
+        assert abs(ours - float(gf)) / float(gf) < 0.01, (name, ours, gf)
+
+
+def test_budget_grid_legality(golden_dir):
+    rows = [ln.split() for ln in open(os.path.join(golden_dir, "budget_grid.txt"))
+            if ln.strip() and not ln.startswith("#")]
+    for name, n0, m, gmin, gmax in rows:
+        n0, m = int(n0), int(m)
+        grid = list(range(2, n0 - 4 + 1, 2))
+        assert len(grid) == m and grid[0] == int(gmin) and grid[-1] == int(gmax)
+    for name in S.CONFIGS:
+        cfg = S.get_config(name)
+        keeps, befores = S.keep_schedule(cfg, 0)
+        for m, n in zip(keeps, befores):
+            k = n - m
+            assert np.all(k >= 0)
+            assert np.all((k == 0) | (m - 1 >= 4))       # >= 4 visual tokens survive
+
+
+def test_compression_identity_and_calibration():
+    for name in S.CONFIGS:
+        cfg = S.get_config(name)
+        keeps, befores = S.keep_schedule(cfg, 0)
+        c = S.compression_from_counts(cfg, keeps, befores)
+        dc = np.zeros(cfg.batch)
+        for l, m, n in zip(cfg.prune_blocks, keeps, befores):
+            dc += (n - m) * (cfg.depth - l) / (cfg.depth * cfg.n_vis0)
+        assert np.max(np.abs(c - dc)) < 1e-12             # C = sum of Delta C_l
+    cfg = S.get_config("cfg3")
+    for seed in range(3):
+        c = S.compression_from_counts(cfg, *S.keep_schedule(cfg, seed))
+        assert abs(c.mean() - 0.38) <= 0.01
+        assert c.min() < 0.30 and c.max() > 0.45          # per-image spread
