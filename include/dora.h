@@ -1,0 +1,255 @@
+/*
+ * dora.h -- C ABI of the GB300 (sm_103a) deployment hot path of DORA's pruned
+ * Vision Transformer forward ("DORA: Dynamic Online Reinforcement Agent for
+ * Token Pruning in Vision Transformers").
+ *
+ * What the path computes (Eq. 1, Sec. 3.1):
+ *     H_attn = H + Attention(LayerNorm(H))
+ *     H_keep = H_attn with the selected visual rows deleted (CLS and the order
+ *              of survivors kept)
+ *     H_next = H_keep + MLP(LayerNorm'(H_keep))
+ * for a batch whose images carry different token counts, packed row after row
+ * into one [T, D] bf16 buffer with int32 sequence boundaries cu[B+1]
+ * (cu[0] = 0, image i owns rows [cu[i], cu[i+1]), its row cu[i] is CLS).
+ *
+ * Conventions shared by every entry point:
+ *  - Every pointer is device memory owned by the caller, unless a comment says
+ *    "host".  The library never allocates and keeps no pointer after a call.
+ *  - bf16 tensors are passed as raw 16-bit patterns (dora_bf16), row-major and
+ *    contiguous.  Pointers handed to the tensor-memory-accelerator paths
+ *    (dora_linear, dora_varlen_attn, dora_pruned_block) must be 16-byte aligned.
+ *  - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream) and never synchronises the host, except dora_read_status.
+ *  - The return value is a host-side status.  Host-side argument checks fail
+ *    fast with DORA_ERR_INVALID_ARG / DORA_ERR_UNSUPPORTED and launch nothing.
+ *  - Problems only the device can see (a keep count outside [1, n_i], an image
+ *    longer than max_seqlen, a bounded wait that ran out) are written to an
+ *    optional device int32 `status` word: the first nonzero code wins and the
+ *    kernel carries on with clamped values.  Kernels never trap.
+ *  - Row counts that depend on earlier device work (T_out after a deletion)
+ *    stay on the device: callers pass capacities (`*_cap`, upper bounds used
+ *    for grid sizes and buffer bounds) and the kernels read the live count
+ *    from cu[batch].
+ *  - The current CUDA device must be compute capability 10.3 (GB300);
+ *    otherwise every entry point returns DORA_ERR_UNSUPPORTED.
+ */
+#ifndef DORA_H_
+#define DORA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t dora_bf16;            /* raw bfloat16 bits */
+typedef struct CUstream_st* dora_stream_t;  /* same type as cudaStream_t */
+
+enum dora_status {
+  DORA_OK = 0,
+  DORA_ERR_INVALID_ARG = 1,        /* host check: null pointer, bad size, misalignment */
+  DORA_ERR_UNSUPPORTED = 2,        /* head_dim != 64, dim % 64 != 0, device is not sm_103 */
+  DORA_ERR_CUDA = 3,               /* a CUDA runtime/driver call failed */
+  DORA_ERR_TIMEOUT = 4,            /* device: a bounded pipeline wait ran out */
+  DORA_ERR_DEVICE_BAD_COUNT = 5,   /* device: keep count outside [1, n_i]; clamped */
+  DORA_ERR_DEVICE_SEQLEN = 6,      /* device: an image is longer than max_seqlen,
+                                      or a row index/count exceeds a capacity */
+};
+
+/* Epilogues of dora_linear. */
+enum dora_epilogue {
+  DORA_EPI_BIAS = 0,          /* y = x W^T + b                 */
+  DORA_EPI_BIAS_GELU = 1,     /* y = GELU(x W^T + b), exact erf */
+  DORA_EPI_BIAS_RESIDUAL = 2  /* y = r + x W^T + b             */
+};
+
+/* Human-readable name of a status code (static string). */
+const char* dora_status_string(int code);
+
+/* ABI version, currently 1. */
+int dora_version(void);
+
+/*
+ * dora_select_keep -- deterministic top-k deletion, one image at a time
+ * (Sec. 3.2 "Sampling and deployment"; Appendix A.3: at inference the
+ * selector removes the k_l highest-scoring visual tokens; CLS is never
+ * selected).
+ *
+ * scores       fp32 [T_in], row-aligned with the packed input; higher = remove
+ *              first.  The entry of each image's CLS row is ignored.
+ * cu_in        int32 [batch+1] input boundaries.
+ * keep_counts  int32 [batch]: m_i, tokens image i keeps, CLS included
+ *              (m_i = n_i - k_i).  Valid range 1 <= m_i <= n_i (an empty image
+ *              keeps 0).  Out-of-range values are clamped into the range and
+ *              DORA_ERR_DEVICE_BAD_COUNT is written to *status.
+ * max_seqlen   upper bound of n_i (<= 8192); sizes shared memory.  An image
+ *              longer than this keeps nothing and raises DORA_ERR_DEVICE_SEQLEN.
+ * kept_idx     out int32 [capacity >= T_in]: global input row of every kept
+ *              token, image after image, ascending within an image.
+ * cu_out       out int32 [batch+1]: cu_out[i+1] - cu_out[i] = clamped m_i.
+ * status       nullable device int32.
+ * Ties: among equal scores the lower index is kept.  Order of scores: -0 ==
+ * +0, every NaN ranks above +inf.  Bit-exact and deterministic.
+ */
+int dora_select_keep(const float* scores, const int32_t* cu_in, const int32_t* keep_counts,
+                     int32_t batch, int32_t max_seqlen, int32_t* kept_idx, int32_t* cu_out,
+                     int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_compact -- hard deletion by stream compaction (Sec. 3.1 pruning
+ * operator; Sec. 3.5 "Inference": surviving sequences are compacted into a
+ * packed buffer with explicit sequence boundaries, per-image order kept).
+ *
+ * x          bf16 [t_in_cap, dim] rows to gather from.
+ * kept_idx   int32 [T_out] from dora_select_keep; every entry < t_in_cap.
+ * cu_out     int32 [batch+1] from dora_select_keep; T_out = cu_out[batch].
+ * ids_in     nullable int32 [t_in_cap]: original token id of each input row.
+ * packed     out bf16 [capacity >= t_in_cap, dim]: packed[r] = x[kept_idx[r]],
+ *            bit for bit.
+ * ids_out    nullable out int32: ids_out[r] = ids_in[kept_idx[r]].
+ * dim % 8 == 0.  An index or T_out beyond t_in_cap is skipped and raises
+ * DORA_ERR_DEVICE_SEQLEN.
+ */
+int dora_compact(const dora_bf16* x, int32_t dim, const int32_t* kept_idx, const int32_t* cu_out,
+                 int32_t batch, int32_t t_in_cap, const int32_t* ids_in, dora_bf16* packed,
+                 int32_t* ids_out, int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_compact_ln -- dora_compact fused with the LayerNorm' that follows the
+ * deletion in Eq. 1: also writes ln_out[r] = LayerNorm(packed[r]) with affine
+ * ln_w, ln_b (bf16 [dim]) and epsilon eps (biased variance, fp32 statistics).
+ * dim % 8 == 0 and dim <= 2048.
+ */
+int dora_compact_ln(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
+                    const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
+                    const int32_t* ids_in, const dora_bf16* ln_w, const dora_bf16* ln_b,
+                    float eps, dora_bf16* packed, int32_t* ids_out, dora_bf16* ln_out,
+                    int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_layernorm -- y = LayerNorm(x) row by row (the LayerNorm of Eq. 1),
+ * biased variance, fp32 statistics, affine w, b (bf16 [dim]).
+ * rows_cap   rows the buffers hold; rows_dev (nullable) points at the live row
+ *            count on the device (e.g. cu + batch); rows beyond it are skipped.
+ * dim % 8 == 0 and dim <= 2048.
+ */
+int dora_layernorm(const dora_bf16* x, int32_t rows_cap, const int32_t* rows_dev, int32_t dim,
+                   const dora_bf16* w, const dora_bf16* b, float eps, dora_bf16* y,
+                   dora_stream_t stream);
+
+/*
+ * dora_linear -- y = epilogue(x W^T + b) on tcgen05 tensor cores, the QKV,
+ * projection and MLP linears of Eq. 1 applied to the packed rows.
+ * x          bf16 [m_cap, k] (16-byte aligned, k % 64 == 0).
+ * m_dev      nullable: live row count on the device; rows >= it are neither
+ *            computed nor written.  NULL means m_cap rows.
+ * w          bf16 [n, k], nn.Linear layout (16-byte aligned, n % 32 == 0).
+ * bias       nullable bf16 [n].
+ * residual   bf16 [m_cap, n], required for DORA_EPI_BIAS_RESIDUAL; may not
+ *            alias y.
+ * y          out bf16 [m_cap, n].
+ * Accumulation is fp32; the result is rounded once to bf16.
+ */
+int dora_linear(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
+                const dora_bf16* w, int32_t n, const dora_bf16* bias, const dora_bf16* residual,
+                int32_t epilogue, dora_bf16* y, int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_varlen_attn -- packed variable-length multi-head self-attention
+ * (Sec. 3.5 "Inference": attention is confined to each image by the explicit
+ * boundaries, no probability matrix is materialised, no token-size terms).
+ * For image i and head h:  O = softmax(Q K^T * softmax_scale) V  over the
+ * n_i rows of image i only.
+ * qkv        bf16 [t_cap, 3, heads, head_dim] (row layout q | k | v).
+ * cu_seqlens int32 [batch+1]; cu_seqlens[batch] <= t_cap.
+ * max_seqlen upper bound of n_i; sizes the grid (an image longer than it is
+ *            only partly computed and raises DORA_ERR_DEVICE_SEQLEN).
+ * head_dim   must be 64.  softmax_scale 0 means 1/sqrt(head_dim).
+ * out        out bf16 [t_cap, heads*head_dim]; rows >= cu_seqlens[batch] are
+ *            not written.
+ * fp32 scores and softmax statistics; P is rounded to bf16 for the PV product.
+ */
+int dora_varlen_attn(const dora_bf16* qkv, const int32_t* cu_seqlens, int32_t batch,
+                     int32_t max_seqlen, int32_t t_cap, int32_t heads, int32_t head_dim,
+                     float softmax_scale, dora_bf16* out, int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_gather_scores -- row-aligned deletion scores from per-image tables
+ * indexed by original token id: scores[r] = table[i * table_stride + ids[r]]
+ * for every row r of image i.  This stands in for the actor's selector output
+ * (Eq. 2) in synthetic workloads; it is not part of Eq. 1.
+ * An id outside [0, table_stride) yields NaN and DORA_ERR_DEVICE_SEQLEN.
+ */
+int dora_gather_scores(const float* table, int32_t table_stride, const int32_t* ids,
+                       const int32_t* cu, int32_t batch, float* scores, int32_t* status,
+                       dora_stream_t stream);
+
+/* Weights of one block, all bf16 device pointers, linears in nn.Linear layout
+ * W[out, in]: w_qkv [3*dim, dim], w_proj [dim, dim], w_fc1 [mlp_dim, dim],
+ * w_fc2 [dim, mlp_dim].  Biases may be NULL (zero). */
+typedef struct dora_block_weights {
+  const dora_bf16* ln1_w;
+  const dora_bf16* ln1_b;
+  const dora_bf16* w_qkv;
+  const dora_bf16* b_qkv;
+  const dora_bf16* w_proj;
+  const dora_bf16* b_proj;
+  const dora_bf16* ln2_w;
+  const dora_bf16* ln2_b;
+  const dora_bf16* w_fc1;
+  const dora_bf16* b_fc1;
+  const dora_bf16* w_fc2;
+  const dora_bf16* b_fc2;
+  int32_t dim;       /* D = heads * 64 */
+  int32_t heads;
+  int32_t mlp_dim;   /* multiple of 64 */
+  float ln_eps;      /* LayerNorm epsilon, e.g. 1e-6 */
+} dora_block_weights;
+
+/* Bytes of device workspace dora_pruned_block needs for t_cap rows. */
+size_t dora_workspace_size(int32_t t_cap, int32_t batch, const dora_block_weights* w);
+
+/*
+ * dora_pruned_block -- one block of Eq. 1 on the packed batch:
+ *   LN1 -> QKV linear -> varlen attention -> projection + residual  (H_attn)
+ *   [select_keep -> compaction fused with LN2]                       (H_keep)
+ *   fc1 + GELU -> fc2 + residual                                     (H_next)
+ * x_in      bf16 [t_cap, dim], rows [0, cu_in[batch]) live.
+ * cu_in     int32 [batch+1]; ids_in int32 [t_cap] original token ids
+ *           (nullable when scores is NULL).
+ * scores    nullable fp32 [t_cap] deletion scores aligned with x_in rows.
+ *           NULL = no deletion in this block (gate off for every image): then
+ *           keep_counts, cu_out, ids_out and kept_idx are ignored and the
+ *           output boundaries are cu_in.
+ * keep_counts int32 [batch] tokens kept per image (CLS included).
+ * x_out     out bf16 [t_cap, dim]; must not alias x_in.
+ * cu_out    out int32 [batch+1]; ids_out out int32 [t_cap];
+ * kept_idx  nullable out int32 [t_cap] (workspace is used when NULL).
+ * workspace device buffer of dora_workspace_size() bytes, 256-byte aligned;
+ *           it also holds the status word read by dora_read_status.  It must
+ *           be zero-filled once after allocation (rows past the live count
+ *           are then always finite).
+ * All counts after the deletion stay on the device; the call never
+ * synchronises, so a sequence of blocks can be captured in a CUDA graph.
+ */
+int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t* ids_in,
+                      int32_t batch, int32_t max_seqlen, int32_t t_cap,
+                      const dora_block_weights* w, const float* scores,
+                      const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
+                      int32_t* ids_out, int32_t* kept_idx, void* workspace,
+                      size_t workspace_bytes, dora_stream_t stream);
+
+/* Device address of the status word inside a dora_pruned_block workspace. */
+int32_t* dora_workspace_status(void* workspace);
+
+/* Synchronises the current device and copies the status word at `status_dev`
+ * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug
+ * only: it blocks the host. */
+int dora_read_status(const int32_t* status_dev, int32_t* code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DORA_H_ */

@@ -1,0 +1,286 @@
+"""GB300 (sm_103a) deployment hot path of DORA's pruned ViT forward.
+
+A thin ctypes binding over ``libdora.so`` (C ABI in ``include/dora.h``).  The
+Python functions carry the C names and only marshal arguments: torch tensors
+supply device pointers and the current CUDA stream; every step of the path
+runs in the library's CUDA kernels.  There is no fallback: when the library
+is missing or the device is not sm_103 the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+__all__ = [
+    "DoraError", "load_library", "library_path", "EPI_BIAS", "EPI_BIAS_GELU",
+    "EPI_BIAS_RESIDUAL", "EXPORTED_SYMBOLS", "dora_status_string", "dora_version",
+    "dora_select_keep", "dora_compact", "dora_compact_ln", "dora_layernorm", "dora_linear",
+    "dora_varlen_attn", "dora_gather_scores", "BlockWeights", "dora_workspace_size",
+    "dora_pruned_block", "dora_workspace_status", "dora_read_status", "alloc_workspace",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+EPI_BIAS, EPI_BIAS_GELU, EPI_BIAS_RESIDUAL = 0, 1, 2
+STATUS_NAMES = {0: "DORA_OK", 1: "DORA_ERR_INVALID_ARG", 2: "DORA_ERR_UNSUPPORTED",
+                3: "DORA_ERR_CUDA", 4: "DORA_ERR_TIMEOUT", 5: "DORA_ERR_DEVICE_BAD_COUNT",
+                6: "DORA_ERR_DEVICE_SEQLEN"}
+
+_vp, _i32, _f32, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_float, ctypes.c_size_t
+_SIGS = {
+    "dora_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "dora_version": (ctypes.c_int, []),
+    "dora_select_keep": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]),
+    "dora_compact": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp]),
+    "dora_compact_ln": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _f32,
+                                       _vp, _vp, _vp, _vp, _vp]),
+    "dora_layernorm": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _vp, _f32, _vp, _vp]),
+    "dora_linear": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _i32, _vp, _vp, _i32, _vp, _vp,
+                                   _vp]),
+    "dora_varlen_attn": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _i32, _f32, _vp, _vp,
+                                        _vp]),
+    "dora_gather_scores": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _vp, _vp, _vp]),
+    "dora_workspace_size": (_sz, [_i32, _i32, _vp]),
+    "dora_pruned_block": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp, _vp,
+                                         _vp, _vp, _vp, _vp, _sz, _vp]),
+    "dora_workspace_status": (_vp, [_vp]),
+    "dora_read_status": (ctypes.c_int, [_vp, _vp]),
+}
+EXPORTED_SYMBOLS = tuple(_SIGS)
+
+_lib = None
+
+
+class DoraError(RuntimeError):
+    """A libdora entry point returned a nonzero host status."""
+
+
+class _BlockWeightsC(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in ("ln1_w", "ln1_b", "w_qkv", "b_qkv", "w_proj", "b_proj",
+                                   "ln2_w", "ln2_b", "w_fc1", "b_fc1", "w_fc2", "b_fc2")] + [
+        ("dim", _i32), ("heads", _i32), ("mlp_dim", _i32), ("ln_eps", _f32)]
+
+
+def library_path() -> str:
+    return os.path.join(_HERE, "libdora.so")
+
+
+def load_library():
+    """Load libdora.so (built by ``__graft_entry__.build()``); raise if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = library_path()
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is not built; run __graft_entry__.build() first")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in _SIGS.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _req(t, dtype, name, optional=False):
+    if t is None:
+        if optional:
+            return
+        raise TypeError(f"{name} is required")
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise TypeError(f"{name} must be contiguous")
+
+
+def _check(code, name):
+    if code != 0:
+        raise DoraError(f"{name}: {dora_status_string(code)} ({STATUS_NAMES.get(code, code)})")
+
+
+def dora_status_string(code: int) -> str:
+    return load_library().dora_status_string(int(code)).decode()
+
+
+def dora_version() -> int:
+    return load_library().dora_version()
+
+
+def dora_select_keep(scores, cu_in, keep_counts, max_seqlen, kept_idx, cu_out, status=None,
+                     stream=None):
+    _req(scores, torch.float32, "scores")
+    for n, t in (("cu_in", cu_in), ("keep_counts", keep_counts), ("kept_idx", kept_idx),
+                 ("cu_out", cu_out)):
+        _req(t, torch.int32, n)
+    _req(status, torch.int32, "status", optional=True)
+    batch = cu_in.numel() - 1
+    _check(load_library().dora_select_keep(_ptr(scores), _ptr(cu_in), _ptr(keep_counts), batch,
+                                           int(max_seqlen), _ptr(kept_idx), _ptr(cu_out),
+                                           _ptr(status), _stream(stream)), "dora_select_keep")
+
+
+def dora_compact(x, kept_idx, cu_out, packed, ids_in=None, ids_out=None, status=None,
+                 stream=None):
+    _req(x, torch.bfloat16, "x")
+    _req(packed, torch.bfloat16, "packed")
+    _req(kept_idx, torch.int32, "kept_idx")
+    _req(cu_out, torch.int32, "cu_out")
+    _req(ids_in, torch.int32, "ids_in", optional=True)
+    _req(ids_out, torch.int32, "ids_out", optional=True)
+    _req(status, torch.int32, "status", optional=True)
+    t_in_cap, dim = x.shape
+    if packed.shape[0] < t_in_cap or packed.shape[1] != dim:
+        raise ValueError("packed must hold at least as many rows as x")
+    _check(load_library().dora_compact(_ptr(x), dim, _ptr(kept_idx), _ptr(cu_out),
+                                       cu_out.numel() - 1, t_in_cap, _ptr(ids_in), _ptr(packed),
+                                       _ptr(ids_out), _ptr(status), _stream(stream)),
+           "dora_compact")
+
+
+def dora_compact_ln(x, kept_idx, cu_out, ln_w, ln_b, eps, packed, ln_out, ids_in=None,
+                    ids_out=None, status=None, stream=None):
+    for n, t in (("x", x), ("packed", packed), ("ln_out", ln_out), ("ln_w", ln_w),
+                 ("ln_b", ln_b)):
+        _req(t, torch.bfloat16, n)
+    _req(kept_idx, torch.int32, "kept_idx")
+    _req(cu_out, torch.int32, "cu_out")
+    _req(ids_in, torch.int32, "ids_in", optional=True)
+    _req(ids_out, torch.int32, "ids_out", optional=True)
+    _req(status, torch.int32, "status", optional=True)
+    t_in_cap, dim = x.shape
+    if packed.shape[0] < t_in_cap or ln_out.shape[0] < t_in_cap:
+        raise ValueError("packed and ln_out must hold at least as many rows as x")
+    _check(load_library().dora_compact_ln(_ptr(x), dim, _ptr(kept_idx), _ptr(cu_out),
+                                          cu_out.numel() - 1, t_in_cap, _ptr(ids_in), _ptr(ln_w),
+                                          _ptr(ln_b), float(eps), _ptr(packed), _ptr(ids_out),
+                                          _ptr(ln_out), _ptr(status), _stream(stream)),
+           "dora_compact_ln")
+
+
+def dora_layernorm(x, w, b, eps, y, rows_dev=None, stream=None):
+    for n, t in (("x", x), ("w", w), ("b", b), ("y", y)):
+        _req(t, torch.bfloat16, n)
+    _req(rows_dev, torch.int32, "rows_dev", optional=True)
+    rows, dim = x.shape
+    _check(load_library().dora_layernorm(_ptr(x), rows, _ptr(rows_dev), dim, _ptr(w), _ptr(b),
+                                         float(eps), _ptr(y), _stream(stream)), "dora_layernorm")
+
+
+def dora_linear(x, w, y, bias=None, residual=None, epilogue=EPI_BIAS, m_dev=None, status=None,
+                stream=None):
+    _req(x, torch.bfloat16, "x")
+    _req(w, torch.bfloat16, "w")
+    _req(y, torch.bfloat16, "y")
+    _req(bias, torch.bfloat16, "bias", optional=True)
+    _req(residual, torch.bfloat16, "residual", optional=True)
+    _req(m_dev, torch.int32, "m_dev", optional=True)
+    _req(status, torch.int32, "status", optional=True)
+    m_cap, k = x.shape
+    n = w.shape[0]
+    if w.shape[1] != k or tuple(y.shape) != (m_cap, n):
+        raise ValueError("shape mismatch: x [M,K], w [N,K], y [M,N]")
+    _check(load_library().dora_linear(_ptr(x), m_cap, _ptr(m_dev), k, _ptr(w), n, _ptr(bias),
+                                      _ptr(residual), int(epilogue), _ptr(y), _ptr(status),
+                                      _stream(stream)), "dora_linear")
+
+
+def dora_varlen_attn(qkv, cu_seqlens, max_seqlen, heads, out, head_dim=64, softmax_scale=0.0,
+                     status=None, stream=None):
+    _req(qkv, torch.bfloat16, "qkv")
+    _req(out, torch.bfloat16, "out")
+    _req(cu_seqlens, torch.int32, "cu_seqlens")
+    _req(status, torch.int32, "status", optional=True)
+    t_cap = qkv.shape[0]
+    _check(load_library().dora_varlen_attn(_ptr(qkv), _ptr(cu_seqlens), cu_seqlens.numel() - 1,
+                                           int(max_seqlen), t_cap, int(heads), int(head_dim),
+                                           float(softmax_scale), _ptr(out), _ptr(status),
+                                           _stream(stream)), "dora_varlen_attn")
+
+
+def dora_gather_scores(table, ids, cu, scores, status=None, stream=None):
+    _req(table, torch.float32, "table")
+    _req(scores, torch.float32, "scores")
+    _req(ids, torch.int32, "ids")
+    _req(cu, torch.int32, "cu")
+    _req(status, torch.int32, "status", optional=True)
+    _check(load_library().dora_gather_scores(_ptr(table), table.shape[-1], _ptr(ids), _ptr(cu),
+                                             cu.numel() - 1, _ptr(scores), _ptr(status),
+                                             _stream(stream)), "dora_gather_scores")
+
+
+class BlockWeights:
+    """Device weights of one block plus the C struct that points at them.
+
+    ``tensors`` maps the names of ``dora_block_weights`` to bf16 CUDA tensors
+    (linears in nn.Linear layout).  The tensors are kept alive here.
+    """
+
+    NAMES = ("ln1_w", "ln1_b", "w_qkv", "b_qkv", "w_proj", "b_proj", "ln2_w", "ln2_b", "w_fc1",
+             "b_fc1", "w_fc2", "b_fc2")
+
+    def __init__(self, tensors: dict, dim: int, heads: int, mlp_dim: int, ln_eps: float = 1e-6):
+        self.tensors = {}
+        for n in self.NAMES:
+            t = tensors.get(n)
+            _req(t, torch.bfloat16, n, optional=n.startswith("b_"))
+            self.tensors[n] = t
+        self.dim, self.heads, self.mlp_dim, self.ln_eps = dim, heads, mlp_dim, ln_eps
+        self.c = _BlockWeightsC(*[_ptr(self.tensors[n]) for n in self.NAMES], dim, heads, mlp_dim,
+                                float(ln_eps))
+
+
+def dora_workspace_size(t_cap, batch, weights: BlockWeights) -> int:
+    return int(load_library().dora_workspace_size(int(t_cap), int(batch), ctypes.byref(weights.c)))
+
+
+def alloc_workspace(t_cap, batch, weights: BlockWeights, device=None) -> torch.Tensor:
+    """Zero-filled uint8 workspace (torch allocation, 256-byte aligned)."""
+    n = dora_workspace_size(t_cap, batch, weights)
+    return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def dora_pruned_block(x_in, cu_in, weights: BlockWeights, max_seqlen, x_out, workspace,
+                      ids_in=None, scores=None, keep_counts=None, cu_out=None, ids_out=None,
+                      kept_idx=None, stream=None):
+    _req(x_in, torch.bfloat16, "x_in")
+    _req(x_out, torch.bfloat16, "x_out")
+    _req(cu_in, torch.int32, "cu_in")
+    _req(workspace, torch.uint8, "workspace")
+    for n, t in (("ids_in", ids_in), ("keep_counts", keep_counts), ("cu_out", cu_out),
+                 ("ids_out", ids_out), ("kept_idx", kept_idx)):
+        _req(t, torch.int32, n, optional=True)
+    _req(scores, torch.float32, "scores", optional=True)
+    t_cap = x_in.shape[0]
+    _check(load_library().dora_pruned_block(
+        _ptr(x_in), _ptr(cu_in), _ptr(ids_in), cu_in.numel() - 1, int(max_seqlen), t_cap,
+        ctypes.byref(weights.c), _ptr(scores), _ptr(keep_counts), _ptr(x_out), _ptr(cu_out),
+        _ptr(ids_out), _ptr(kept_idx), _ptr(workspace), workspace.numel(), _stream(stream)),
+        "dora_pruned_block")
+
+
+def dora_workspace_status(workspace) -> int:
+    """Device address of the status word inside a block workspace."""
+    return int(load_library().dora_workspace_status(_ptr(workspace)))
+
+
+def dora_read_status(status) -> int:
+    """Synchronise and read a device status word (tensor or device address)."""
+    code = ctypes.c_int32(0)
+    _check(load_library().dora_read_status(_ptr(status), ctypes.byref(code)), "dora_read_status")
+    return int(code.value)

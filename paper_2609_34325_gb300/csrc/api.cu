@@ -1,0 +1,345 @@
+// Host side of the C ABI declared in include/dora.h: argument validation,
+// device checks, tensor-map encoding and the kernel sequence of one pruned
+// block.  No entry point allocates memory or synchronises (except
+// dora_read_status).
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "dora.h"
+#include "token_ops.cuh"
+
+namespace dora {
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+int g_arch_ok[kMaxDevices];       // 0 unknown, 1 sm_103, -1 other
+int g_num_sms[kMaxDevices];
+std::mutex g_mu;
+
+int current_device_checked() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return -1;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_arch_ok[dev] == 0) {
+    int major = 0, minor = 0, sms = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    g_arch_ok[dev] = (major == 10 && minor == 3) ? 1 : -1;
+    g_num_sms[dev] = sms > 0 ? sms : 1;
+  }
+  return g_arch_ok[dev] == 1 ? dev : -2;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+}  // namespace
+
+int num_sms() {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= kMaxDevices || g_num_sms[dev] <= 0) return 148;
+  return g_num_sms[dev];
+}
+
+int encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t outer,
+                        uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer) {
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (g_encode == nullptr) {
+      void* fn = nullptr;
+      cudaDriverEntryPointQueryResult q;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                           &q) != cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || fn == nullptr)
+        return -1;
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+  }
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_pitch_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(reinterpret_cast<CUtensorMap*>(map), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? 0 : static_cast<int>(r);
+}
+
+}  // namespace dora
+
+using namespace dora;
+
+#define DORA_CHECK_ARG(cond) \
+  do {                       \
+    if (!(cond)) return DORA_ERR_INVALID_ARG; \
+  } while (0)
+
+#define DORA_CHECK_DEVICE()                             \
+  do {                                                  \
+    const int _d = current_device_checked();            \
+    if (_d == -1) return DORA_ERR_CUDA;                 \
+    if (_d < 0) return DORA_ERR_UNSUPPORTED;            \
+  } while (0)
+
+static int cuda_status(cudaError_t e) { return e == cudaSuccess ? DORA_OK : DORA_ERR_CUDA; }
+
+extern "C" {
+
+const char* dora_status_string(int code) {
+  switch (code) {
+    case DORA_OK: return "ok";
+    case DORA_ERR_INVALID_ARG: return "invalid argument";
+    case DORA_ERR_UNSUPPORTED: return "unsupported (shape or device)";
+    case DORA_ERR_CUDA: return "CUDA error";
+    case DORA_ERR_TIMEOUT: return "device wait timed out";
+    case DORA_ERR_DEVICE_BAD_COUNT: return "keep count out of range (clamped)";
+    case DORA_ERR_DEVICE_SEQLEN: return "sequence longer than max_seqlen or index past capacity";
+    default: return "unknown status";
+  }
+}
+
+int dora_version(void) { return 1; }
+
+int dora_select_keep(const float* scores, const int32_t* cu_in, const int32_t* keep_counts,
+                     int32_t batch, int32_t max_seqlen, int32_t* kept_idx, int32_t* cu_out,
+                     int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(batch >= 0 && batch <= (1 << 24));
+  DORA_CHECK_ARG(max_seqlen >= 0 && max_seqlen <= kMaxSeqlenSelect);
+  DORA_CHECK_ARG(cu_in && keep_counts && cu_out);
+  DORA_CHECK_ARG(batch == 0 || (scores && kept_idx));
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_select_keep(scores, cu_in, keep_counts, batch, max_seqlen, kept_idx,
+                                        cu_out, status, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+static int compact_common(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
+                          const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
+                          const int32_t* ids_in, const dora_bf16* ln_w, const dora_bf16* ln_b,
+                          float eps, dora_bf16* packed, int32_t* ids_out, dora_bf16* ln_out,
+                          int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(batch >= 0 && t_in_cap >= 0);
+  DORA_CHECK_ARG(dim > 0 && dim % 8 == 0 && dim <= kMaxDimRow);
+  DORA_CHECK_ARG(cu_out != nullptr);
+  DORA_CHECK_ARG(t_in_cap == 0 || (x && kept_idx && packed));
+  DORA_CHECK_ARG(aligned16(x) && aligned16(packed) && aligned16(ln_out));
+  DORA_CHECK_ARG((ids_out == nullptr) || (ids_in != nullptr));
+  if (ln_out) DORA_CHECK_ARG(ln_w && ln_b && aligned16(ln_w) && aligned16(ln_b) && eps >= 0.f);
+  DORA_CHECK_DEVICE();
+  if (t_in_cap == 0) return DORA_OK;
+  return cuda_status(launch_compact(x, dim, kept_idx, cu_out, batch, t_in_cap, ids_in, ln_w, ln_b,
+                                    eps, packed, ids_out, ln_out, status,
+                                    reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_compact(const dora_bf16* x, int32_t dim, const int32_t* kept_idx, const int32_t* cu_out,
+                 int32_t batch, int32_t t_in_cap, const int32_t* ids_in, dora_bf16* packed,
+                 int32_t* ids_out, int32_t* status, dora_stream_t stream) {
+  return compact_common(x, dim, kept_idx, cu_out, batch, t_in_cap, ids_in, nullptr, nullptr, 0.f,
+                        packed, ids_out, nullptr, status, stream);
+}
+
+int dora_compact_ln(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
+                    const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
+                    const int32_t* ids_in, const dora_bf16* ln_w, const dora_bf16* ln_b,
+                    float eps, dora_bf16* packed, int32_t* ids_out, dora_bf16* ln_out,
+                    int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(ln_out != nullptr);
+  return compact_common(x, dim, kept_idx, cu_out, batch, t_in_cap, ids_in, ln_w, ln_b, eps,
+                        packed, ids_out, ln_out, status, stream);
+}
+
+int dora_layernorm(const dora_bf16* x, int32_t rows_cap, const int32_t* rows_dev, int32_t dim,
+                   const dora_bf16* w, const dora_bf16* b, float eps, dora_bf16* y,
+                   dora_stream_t stream) {
+  DORA_CHECK_ARG(rows_cap >= 0);
+  DORA_CHECK_ARG(dim > 0 && dim % 8 == 0 && dim <= kMaxDimRow);
+  DORA_CHECK_ARG(rows_cap == 0 || (x && y));
+  DORA_CHECK_ARG(w && b && eps >= 0.f);
+  DORA_CHECK_ARG(aligned16(x) && aligned16(y) && aligned16(w) && aligned16(b));
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_layernorm(x, rows_cap, rows_dev, dim, w, b, eps, y,
+                                      reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_linear(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
+                const dora_bf16* w, int32_t n, const dora_bf16* bias, const dora_bf16* residual,
+                int32_t epilogue, dora_bf16* y, int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(m_cap >= 0 && m_cap <= (1 << 30) / 1);
+  DORA_CHECK_ARG(k > 0 && k % 64 == 0 && k <= (1 << 16));
+  DORA_CHECK_ARG(n > 0 && n % 32 == 0 && n <= (1 << 16));
+  DORA_CHECK_ARG(epilogue >= DORA_EPI_BIAS && epilogue <= DORA_EPI_BIAS_RESIDUAL);
+  DORA_CHECK_ARG(w && y && (m_cap == 0 || x));
+  DORA_CHECK_ARG(aligned16(x) && aligned16(w) && aligned16(y) && aligned16(bias) &&
+                 aligned16(residual));
+  if (epilogue == DORA_EPI_BIAS_RESIDUAL) DORA_CHECK_ARG(residual && residual != y);
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_linear(x, m_cap, m_dev, k, w, n, bias, residual, epilogue, y, status,
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_varlen_attn(const dora_bf16* qkv, const int32_t* cu_seqlens, int32_t batch,
+                     int32_t max_seqlen, int32_t t_cap, int32_t heads, int32_t head_dim,
+                     float softmax_scale, dora_bf16* out, int32_t* status, dora_stream_t stream) {
+  if (head_dim != 64) return DORA_ERR_UNSUPPORTED;
+  DORA_CHECK_ARG(batch >= 0 && batch <= 65535);
+  DORA_CHECK_ARG(heads > 0 && heads <= 65535 && heads * 64 * 3 <= (1 << 16));
+  DORA_CHECK_ARG(max_seqlen >= 0 && t_cap >= 0);
+  DORA_CHECK_ARG(softmax_scale >= 0.f && isfinite(softmax_scale));
+  DORA_CHECK_ARG(cu_seqlens && (t_cap == 0 || (qkv && out)));
+  DORA_CHECK_ARG(aligned16(qkv) && aligned16(out));
+  DORA_CHECK_DEVICE();
+  const float scale = softmax_scale == 0.f ? 0.125f : softmax_scale;
+  return cuda_status(launch_varlen_attn(qkv, cu_seqlens, batch, max_seqlen, t_cap, heads, scale,
+                                        out, status, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_gather_scores(const float* table, int32_t table_stride, const int32_t* ids,
+                       const int32_t* cu, int32_t batch, float* scores, int32_t* status,
+                       dora_stream_t stream) {
+  DORA_CHECK_ARG(batch >= 0 && table_stride > 0);
+  DORA_CHECK_ARG(cu && (batch == 0 || (table && ids && scores)));
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_gather_scores(table, table_stride, ids, cu, batch, scores, status,
+                                          reinterpret_cast<cudaStream_t>(stream)));
+}
+
+// ---------------------------------------------------------------------------
+// workspace and the pruned block
+// ---------------------------------------------------------------------------
+namespace {
+struct WsLayout {
+  size_t status, xn, qkv, o, hattn, hkeep, kept, u, total;
+};
+
+size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+WsLayout ws_layout(int32_t t_cap, const dora_block_weights* w) {
+  WsLayout L{};
+  const size_t t = static_cast<size_t>(t_cap), d = static_cast<size_t>(w->dim);
+  size_t off = 0;
+  L.status = off; off += 256;
+  L.xn = off;     off += up256(t * d * 2);
+  L.qkv = off;    off += up256(t * 3 * d * 2);
+  L.o = off;      off += up256(t * d * 2);
+  L.hattn = off;  off += up256(t * d * 2);
+  L.hkeep = off;  off += up256(t * d * 2);
+  L.kept = off;   off += up256(t * 4);
+  L.u = off;      off += up256(t * static_cast<size_t>(w->mlp_dim) * 2);
+  L.total = off;
+  return L;
+}
+
+bool weights_ok(const dora_block_weights* w) {
+  if (!w) return false;
+  if (w->dim <= 0 || w->heads <= 0 || w->dim != w->heads * 64) return false;
+  if (w->dim > kMaxDimRow || w->mlp_dim <= 0 || w->mlp_dim % 64 != 0) return false;
+  if (!(w->ln_eps >= 0.f)) return false;
+  const void* req[] = {w->ln1_w, w->ln1_b, w->w_qkv, w->w_proj, w->ln2_w, w->ln2_b, w->w_fc1,
+                       w->w_fc2};
+  for (const void* p : req)
+    if (!p || !aligned16(p)) return false;
+  const void* opt[] = {w->b_qkv, w->b_proj, w->b_fc1, w->b_fc2};
+  for (const void* p : opt)
+    if (!aligned16(p)) return false;
+  return true;
+}
+}  // namespace
+
+size_t dora_workspace_size(int32_t t_cap, int32_t batch, const dora_block_weights* w) {
+  (void)batch;
+  if (t_cap < 0 || !w || w->dim <= 0 || w->mlp_dim <= 0) return 0;
+  return ws_layout(t_cap, w).total;
+}
+
+int32_t* dora_workspace_status(void* workspace) { return static_cast<int32_t*>(workspace); }
+
+int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t* ids_in,
+                      int32_t batch, int32_t max_seqlen, int32_t t_cap,
+                      const dora_block_weights* w, const float* scores,
+                      const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
+                      int32_t* ids_out, int32_t* kept_idx, void* workspace,
+                      size_t workspace_bytes, dora_stream_t stream_) {
+  DORA_CHECK_ARG(weights_ok(w));
+  DORA_CHECK_ARG(batch >= 0 && batch <= 65535 && t_cap >= 0 && max_seqlen >= 0);
+  DORA_CHECK_ARG(max_seqlen <= kMaxSeqlenSelect);
+  DORA_CHECK_ARG(x_in && x_out && cu_in && workspace && x_in != x_out);
+  DORA_CHECK_ARG(aligned16(x_in) && aligned16(x_out));
+  DORA_CHECK_ARG((reinterpret_cast<uintptr_t>(workspace) & 255u) == 0);
+  if (scores) DORA_CHECK_ARG(keep_counts && cu_out && ids_in && ids_out);
+  const WsLayout L = ws_layout(t_cap, w);
+  DORA_CHECK_ARG(workspace_bytes >= L.total);
+  DORA_CHECK_DEVICE();
+  if (t_cap == 0 || batch == 0) return DORA_OK;
+
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  int32_t* status = reinterpret_cast<int32_t*>(ws + L.status);
+  uint16_t* xn = reinterpret_cast<uint16_t*>(ws + L.xn);
+  uint16_t* qkv = reinterpret_cast<uint16_t*>(ws + L.qkv);
+  uint16_t* o = reinterpret_cast<uint16_t*>(ws + L.o);
+  uint16_t* hattn = reinterpret_cast<uint16_t*>(ws + L.hattn);
+  uint16_t* hkeep = reinterpret_cast<uint16_t*>(ws + L.hkeep);
+  int32_t* kept = kept_idx ? kept_idx : reinterpret_cast<int32_t*>(ws + L.kept);
+  uint16_t* u = reinterpret_cast<uint16_t*>(ws + L.u);
+  const int d = w->dim;
+  const int32_t* rows_in = cu_in + batch;
+
+  // H_attn = H + Attention(LayerNorm(H))
+  if ((launch_layernorm(x_in, t_cap, rows_in, d, w->ln1_w, w->ln1_b, w->ln_eps, xn, stream)) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  if ((launch_linear(xn, t_cap, rows_in, d, w->w_qkv, 3 * d, w->b_qkv, nullptr, DORA_EPI_BIAS,
+                         qkv, status, stream)) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  if ((launch_varlen_attn(qkv, cu_in, batch, max_seqlen, t_cap, w->heads, 0.125f, o, status,
+                              stream)) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  if ((launch_linear(o, t_cap, rows_in, d, w->w_proj, d, w->b_proj, x_in,
+                         DORA_EPI_BIAS_RESIDUAL, hattn, status, stream)) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  // H_keep: delete, compact, LayerNorm' in one pass
+  const uint16_t* hk = hattn;
+  const int32_t* rows_mid = rows_in;
+  if (scores) {
+    if ((launch_select_keep(scores, cu_in, keep_counts, batch, max_seqlen, kept, cu_out,
+                                status, stream)) != cudaSuccess)
+      return DORA_ERR_CUDA;
+    if ((launch_compact(hattn, d, kept, cu_out, batch, t_cap, ids_in, w->ln2_w, w->ln2_b,
+                            w->ln_eps, hkeep, ids_out, xn, status, stream)) != cudaSuccess)
+      return DORA_ERR_CUDA;
+    hk = hkeep;
+    rows_mid = cu_out + batch;
+  } else {
+    if ((launch_layernorm(hattn, t_cap, rows_in, d, w->ln2_w, w->ln2_b, w->ln_eps, xn,
+                              stream)) != cudaSuccess)
+      return DORA_ERR_CUDA;
+  }
+  // H_next = H_keep + MLP(LayerNorm'(H_keep))
+  if ((launch_linear(xn, t_cap, rows_mid, d, w->w_fc1, w->mlp_dim, w->b_fc1, nullptr,
+                         DORA_EPI_BIAS_GELU, u, status, stream)) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  if ((launch_linear(u, t_cap, rows_mid, w->mlp_dim, w->w_fc2, d, w->b_fc2, hk,
+                         DORA_EPI_BIAS_RESIDUAL, x_out, status, stream)) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  return DORA_OK;
+}
+
+int dora_read_status(const int32_t* status_dev, int32_t* code) {
+  DORA_CHECK_ARG(status_dev && code);
+  if (cudaDeviceSynchronize() != cudaSuccess) return DORA_ERR_CUDA;
+  if (cudaMemcpy(code, status_dev, sizeof(int32_t), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  return DORA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,400 @@
+// Token selection, stream compaction (optionally fused with LayerNorm'),
+// row LayerNorm and the synthetic score gather.  All are bandwidth- or
+// latency-bound integer/copy work: no tensor cores.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dora_ptx.cuh"
+#include "token_ops.cuh"
+
+namespace dora {
+
+// ---------------------------------------------------------------------------
+// helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int warp_sum(int v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ float warp_sumf(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Block-wide sum; `scratch` holds >= 32 ints.  All threads get the result.
+__device__ int block_sum(int v, int* scratch) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = (blockDim.x + 31) >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) scratch[warp] = v;
+  __syncthreads();
+  int t = (threadIdx.x < nw) ? scratch[threadIdx.x] : 0;
+  if (warp == 0) t = warp_sum(t);
+  if (threadIdx.x == 0) scratch[0] = t;
+  __syncthreads();
+  const int r = scratch[0];
+  __syncthreads();
+  return r;
+}
+
+// Block-wide exclusive prefix sum of one int per thread (thread order).
+__device__ int block_exclusive_scan(int v, int* scratch) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nw = (blockDim.x + 31) >> 5;
+  int inc = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += t;
+  }
+  __syncthreads();
+  if (lane == 31) scratch[warp] = inc;
+  __syncthreads();
+  if (warp == 0) {
+    int w = (lane < nw) ? scratch[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += t;
+    }
+    if (lane < nw) scratch[lane] = w;   // inclusive over warps
+  }
+  __syncthreads();
+  const int warp_base = (warp == 0) ? 0 : scratch[warp - 1];
+  const int r = warp_base + inc - v;
+  __syncthreads();
+  return r;
+}
+
+// Monotone map of fp32 scores to uint32: unsigned order of keys equals the
+// order of the values, -0 == +0, every NaN above +inf.
+__device__ __forceinline__ uint32_t score_key(float s) {
+  uint32_t b = __float_as_uint(s);
+  if (b == 0x80000000u) b = 0u;
+  uint32_t k = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+  if (s != s) k = 0xFFFFFFFFu;
+  return k;
+}
+
+// Tokens image i keeps after clamping; every CTA evaluates it identically.
+__device__ __forceinline__ int clamped_keep(int n, int m, int max_seqlen) {
+  if (n > max_seqlen || n <= 0) return 0;
+  return m < 1 ? 1 : (m > n ? n : m);
+}
+
+// ---------------------------------------------------------------------------
+// K1: per-image deterministic top-k deletion
+// ---------------------------------------------------------------------------
+// One CTA per image.  Each visual candidate j counts how many candidates
+// precede it in the order (score key, index); it is kept when that rank is
+// below m - 1.  Kept flags are then scanned to write ascending indices.
+__global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
+    const float* __restrict__ scores, const int32_t* __restrict__ cu_in,
+    const int32_t* __restrict__ keep_counts, int32_t batch, int32_t max_seqlen,
+    int32_t* __restrict__ kept_idx, int32_t* __restrict__ cu_out, int32_t* status) {
+  extern __shared__ uint32_t keys[];            // [max_seqlen]
+  __shared__ int scratch[33];
+  const int i = blockIdx.x;
+  const int tid = threadIdx.x;
+
+  // output offset of this image: sum of the clamped keep counts before it
+  int part = 0;
+  for (int t = tid; t < i; t += blockDim.x)
+    part += clamped_keep(cu_in[t + 1] - cu_in[t], keep_counts[t], max_seqlen);
+  const int off = block_sum(part, scratch);
+
+  const int lo = cu_in[i];
+  const int n = cu_in[i + 1] - lo;
+  const int m = keep_counts[i];
+  const int me = clamped_keep(n, m, max_seqlen);
+  if (tid == 0) {
+    if (n > max_seqlen) record_status(status, DORA_ERR_DEVICE_SEQLEN);
+    else if (n < 0 || (n > 0 && me != m) || (n == 0 && m != 0))
+      record_status(status, DORA_ERR_DEVICE_BAD_COUNT);
+    cu_out[i + 1] = off + me;
+    if (i == 0) cu_out[0] = 0;
+  }
+  if (me == 0) return;
+
+  for (int j = tid; j < n; j += blockDim.x) keys[j] = score_key(scores[lo + j]);
+  __syncthreads();
+
+  // Each thread owns a contiguous segment of candidate indices so that the
+  // flag scan below preserves index order.
+  const int per = (n + blockDim.x - 1) / blockDim.x;
+  const int j0 = tid * per;
+  const int j1 = min(n, j0 + per);
+  uint32_t keepmask = 0;     // bit q set when index j0 + q is kept (per <= 32)
+  int cnt = 0;
+  const int need = me - 1;   // visual tokens to keep
+  for (int j = j0; j < j1; ++j) {
+    bool kept;
+    if (j == 0) {
+      kept = true;           // CLS
+    } else {
+      const uint32_t kj = keys[j];
+      int rank = 0;
+      for (int t = 1; t < n; ++t) {
+        const uint32_t kt = keys[t];
+        rank += (kt < kj) | ((kt == kj) & (t < j));
+      }
+      kept = rank < need;
+    }
+    if (kept) {
+      keepmask |= 1u << (j - j0);
+      ++cnt;
+    }
+  }
+  const int pos = block_exclusive_scan(cnt, scratch);
+  int w = off + pos;
+  for (int j = j0; j < j1; ++j)
+    if (keepmask & (1u << (j - j0))) kept_idx[w++] = lo + j;
+}
+
+// ---------------------------------------------------------------------------
+// K2: compaction (+ LayerNorm'), one warp per output row
+// ---------------------------------------------------------------------------
+template <bool kLN>
+__global__ void __launch_bounds__(kRowThreads) compact_kernel(
+    const uint4* __restrict__ x, int32_t chunks /* dim / 8 */, const int32_t* __restrict__ kept_idx,
+    const int32_t* __restrict__ cu_out, int32_t batch, int32_t t_in_cap,
+    const int32_t* __restrict__ ids_in, const uint4* __restrict__ ln_w,
+    const uint4* __restrict__ ln_b, float eps, uint4* __restrict__ packed,
+    int32_t* __restrict__ ids_out, uint4* __restrict__ ln_out, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  int t_out = cu_out[batch];
+  if (t_out > t_in_cap || t_out < 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) record_status(status, DORA_ERR_DEVICE_SEQLEN);
+    t_out = t_out < 0 ? 0 : t_in_cap;
+  }
+  const float inv_dim = 1.0f / static_cast<float>(chunks * 8);
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < t_out; r += warps) {
+    const int src = kept_idx[r];
+    if (src < 0 || src >= t_in_cap) {
+      if (lane == 0) record_status(status, DORA_ERR_DEVICE_SEQLEN);
+      continue;
+    }
+    if (ids_out != nullptr && lane == 0) ids_out[r] = ids_in[src];
+    const uint4* srow = x + static_cast<size_t>(src) * chunks;
+    uint4* drow = packed + static_cast<size_t>(r) * chunks;
+    uint4 v[kMaxChunksPerLane];
+#pragma unroll
+    for (int q = 0; q < kMaxChunksPerLane; ++q) {
+      const int c = lane + 32 * q;
+      if (c < chunks) v[q] = __ldg(srow + c);
+    }
+#pragma unroll
+    for (int q = 0; q < kMaxChunksPerLane; ++q) {
+      const int c = lane + 32 * q;
+      if (c < chunks) drow[c] = v[q];
+    }
+    if constexpr (kLN) {
+      float sum = 0.f;
+#pragma unroll
+      for (int q = 0; q < kMaxChunksPerLane; ++q) {
+        if (lane + 32 * q < chunks) {
+          const uint32_t* w = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) sum += bf16_lo(w[e]) + bf16_hi(w[e]);
+        }
+      }
+      const float mean = warp_sumf(sum) * inv_dim;
+      float sq = 0.f;
+#pragma unroll
+      for (int q = 0; q < kMaxChunksPerLane; ++q) {
+        if (lane + 32 * q < chunks) {
+          const uint32_t* w = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float a = bf16_lo(w[e]) - mean, b = bf16_hi(w[e]) - mean;
+            sq += a * a + b * b;
+          }
+        }
+      }
+      const float rstd = rsqrtf(warp_sumf(sq) * inv_dim + eps);
+      uint4* lrow = ln_out + static_cast<size_t>(r) * chunks;
+#pragma unroll
+      for (int q = 0; q < kMaxChunksPerLane; ++q) {
+        const int c = lane + 32 * q;
+        if (c < chunks) {
+          const uint4 gw = __ldg(ln_w + c), gb = __ldg(ln_b + c);
+          const uint32_t* w = reinterpret_cast<const uint32_t*>(&v[q]);
+          const uint32_t* g = reinterpret_cast<const uint32_t*>(&gw);
+          const uint32_t* bb = reinterpret_cast<const uint32_t*>(&gb);
+          uint4 o;
+          uint32_t* ow = reinterpret_cast<uint32_t*>(&o);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float a = (bf16_lo(w[e]) - mean) * rstd * bf16_lo(g[e]) + bf16_lo(bb[e]);
+            const float b = (bf16_hi(w[e]) - mean) * rstd * bf16_hi(g[e]) + bf16_hi(bb[e]);
+            ow[e] = pack_bf16x2(a, b);
+          }
+          lrow[c] = o;
+        }
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// K5: LayerNorm, one warp per row
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kRowThreads) layernorm_kernel(
+    const uint4* __restrict__ x, int32_t rows_cap, const int32_t* __restrict__ rows_dev,
+    int32_t chunks, const uint4* __restrict__ w, const uint4* __restrict__ b, float eps,
+    uint4* __restrict__ y) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  int rows = rows_cap;
+  if (rows_dev != nullptr) rows = min(rows_cap, max(0, *rows_dev));
+  const float inv_dim = 1.0f / static_cast<float>(chunks * 8);
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += warps) {
+    const uint4* srow = x + static_cast<size_t>(r) * chunks;
+    uint4 v[kMaxChunksPerLane];
+    float sum = 0.f;
+#pragma unroll
+    for (int q = 0; q < kMaxChunksPerLane; ++q) {
+      const int c = lane + 32 * q;
+      if (c < chunks) {
+        v[q] = __ldg(srow + c);
+        const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) sum += bf16_lo(u[e]) + bf16_hi(u[e]);
+      }
+    }
+    const float mean = warp_sumf(sum) * inv_dim;
+    float sq = 0.f;
+#pragma unroll
+    for (int q = 0; q < kMaxChunksPerLane; ++q) {
+      if (lane + 32 * q < chunks) {
+        const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float a = bf16_lo(u[e]) - mean, c2 = bf16_hi(u[e]) - mean;
+          sq += a * a + c2 * c2;
+        }
+      }
+    }
+    const float rstd = rsqrtf(warp_sumf(sq) * inv_dim + eps);
+    uint4* drow = y + static_cast<size_t>(r) * chunks;
+#pragma unroll
+    for (int q = 0; q < kMaxChunksPerLane; ++q) {
+      const int c = lane + 32 * q;
+      if (c < chunks) {
+        const uint4 gw = __ldg(w + c), gb = __ldg(b + c);
+        const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+        const uint32_t* g = reinterpret_cast<const uint32_t*>(&gw);
+        const uint32_t* bb = reinterpret_cast<const uint32_t*>(&gb);
+        uint4 o;
+        uint32_t* ow = reinterpret_cast<uint32_t*>(&o);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float a = (bf16_lo(u[e]) - mean) * rstd * bf16_lo(g[e]) + bf16_lo(bb[e]);
+          const float c2 = (bf16_hi(u[e]) - mean) * rstd * bf16_hi(g[e]) + bf16_hi(bb[e]);
+          ow[e] = pack_bf16x2(a, c2);
+        }
+        drow[c] = o;
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// synthetic actor stand-in: row-aligned scores from per-image id tables
+// ---------------------------------------------------------------------------
+__global__ void gather_scores_kernel(const float* __restrict__ table, int32_t stride,
+                                     const int32_t* __restrict__ ids,
+                                     const int32_t* __restrict__ cu, float* __restrict__ scores,
+                                     int32_t* status) {
+  const int i = blockIdx.x;
+  const int lo = cu[i], hi = cu[i + 1];
+  const float* row = table + static_cast<size_t>(i) * stride;
+  for (int r = lo + threadIdx.x; r < hi; r += blockDim.x) {
+    const int id = ids[r];
+    float s;
+    if (id >= 0 && id < stride) {
+      s = row[id];
+    } else {
+      s = __int_as_float(0x7FC00000);
+      record_status(status, DORA_ERR_DEVICE_SEQLEN);
+    }
+    scores[r] = s;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// launchers
+// ---------------------------------------------------------------------------
+static int row_grid(int64_t rows) {
+  const int64_t warps_per_cta = kRowThreads / 32;
+  int64_t g = (rows + warps_per_cta - 1) / warps_per_cta;
+  const int64_t cap = 152LL * 16;       // grid-stride beyond ~16 CTAs per SM
+  if (g > cap) g = cap;
+  if (g < 1) g = 1;
+  return static_cast<int>(g);
+}
+
+cudaError_t launch_select_keep(const float* scores, const int32_t* cu_in,
+                               const int32_t* keep_counts, int32_t batch, int32_t max_seqlen,
+                               int32_t* kept_idx, int32_t* cu_out, int32_t* status,
+                               cudaStream_t stream) {
+  if (batch == 0) return cudaSuccess;
+  const size_t smem = static_cast<size_t>(max_seqlen) * sizeof(uint32_t);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(select_keep_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  select_keep_kernel<<<batch, kSelectThreads, smem, stream>>>(scores, cu_in, keep_counts, batch,
+                                                              max_seqlen, kept_idx, cu_out,
+                                                              status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compact(const uint16_t* x, int32_t dim, const int32_t* kept_idx,
+                           const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
+                           const int32_t* ids_in, const uint16_t* ln_w, const uint16_t* ln_b,
+                           float eps, uint16_t* packed, int32_t* ids_out, uint16_t* ln_out,
+                           int32_t* status, cudaStream_t stream) {
+  const int grid = row_grid(t_in_cap);
+  const int chunks = dim / 8;
+  if (ln_out != nullptr) {
+    compact_kernel<true><<<grid, kRowThreads, 0, stream>>>(
+        reinterpret_cast<const uint4*>(x), chunks, kept_idx, cu_out, batch, t_in_cap, ids_in,
+        reinterpret_cast<const uint4*>(ln_w), reinterpret_cast<const uint4*>(ln_b), eps,
+        reinterpret_cast<uint4*>(packed), ids_out, reinterpret_cast<uint4*>(ln_out), status);
+  } else {
+    compact_kernel<false><<<grid, kRowThreads, 0, stream>>>(
+        reinterpret_cast<const uint4*>(x), chunks, kept_idx, cu_out, batch, t_in_cap, ids_in,
+        nullptr, nullptr, 0.f, reinterpret_cast<uint4*>(packed), ids_out, nullptr, status);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_layernorm(const uint16_t* x, int32_t rows_cap, const int32_t* rows_dev,
+                             int32_t dim, const uint16_t* w, const uint16_t* b, float eps,
+                             uint16_t* y, cudaStream_t stream) {
+  if (rows_cap == 0) return cudaSuccess;
+  layernorm_kernel<<<row_grid(rows_cap), kRowThreads, 0, stream>>>(
+      reinterpret_cast<const uint4*>(x), rows_cap, rows_dev, dim / 8,
+      reinterpret_cast<const uint4*>(w), reinterpret_cast<const uint4*>(b), eps,
+      reinterpret_cast<uint4*>(y));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_scores(const float* table, int32_t stride, const int32_t* ids,
+                                 const int32_t* cu, int32_t batch, float* scores, int32_t* status,
+                                 cudaStream_t stream) {
+  if (batch == 0) return cudaSuccess;
+  gather_scores_kernel<<<batch, 256, 0, stream>>>(table, stride, ids, cu, scores, status);
+  return cudaGetLastError();
+}
+
+}  // namespace dora

@@ -1,0 +1,83 @@
+"""Host-only checks of the C ABI: the library builds, loads, exports every
+symbol the header declares, and rejects bad arguments before touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import __graft_entry__ as G
+import paper_2609_34325_gb300 as P
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    G.build()
+    return P.load_library()
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "dora.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(dora_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_entry_points():
+    decl = _declared_functions()
+    for name in ("dora_select_keep", "dora_compact", "dora_varlen_attn", "dora_pruned_block",
+                 "dora_workspace_size", "dora_read_status"):
+        assert name in decl
+    assert sorted(P.EXPORTED_SYMBOLS) == decl
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    assert P.dora_version() == 1
+    assert P.dora_status_string(0) == "ok"
+    assert "timed out" in P.dora_status_string(4)
+    assert P.dora_status_string(99) == "unknown status"
+
+
+def test_host_validation_without_gpu(lib):
+    # every failure below is decided from the arguments, before any CUDA call
+    assert lib.dora_select_keep(None, None, None, 1, 197, None, None, None, None) == 1
+    assert lib.dora_select_keep(None, 8, 8, 1, 1 << 20, 8, 8, None, None) == 1
+    assert lib.dora_varlen_attn(16, 16, 1, 197, 197, 3, 32, 0.0, 16, None, None) == 2
+    assert lib.dora_varlen_attn(16, 16, 1, 197, 197, 3, 64, -1.0, 16, None, None) == 1
+    assert lib.dora_varlen_attn(17, 16, 1, 197, 197, 3, 64, 0.0, 16, None, None) == 1
+    assert lib.dora_linear(16, 128, None, 100, 16, 128, None, None, 0, 16, None, None) == 1
+    assert lib.dora_linear(16, 128, None, 128, 16, 100, None, None, 0, 16, None, None) == 1
+    assert lib.dora_linear(16, 128, None, 128, 16, 128, None, None, 2, 16, None, None) == 1
+    assert lib.dora_linear(16, 128, None, 128, 16, 128, None, None, 7, 16, None, None) == 1
+    assert lib.dora_compact(16, 12, 16, 16, 1, 10, None, 16, None, None, None) == 1
+    assert lib.dora_layernorm(16, 4, None, 4096, 16, 16, 1e-6, 16, None) == 1
+    assert lib.dora_gather_scores(16, 0, 16, 16, 1, 16, None, None) == 1
+    assert lib.dora_read_status(None, None) == 1
+    assert lib.dora_pruned_block(None, None, None, 1, 197, 197, None, None, None, None, None,
+                                 None, None, None, 0, None) == 1
+
+
+def test_block_weights_struct_and_workspace(lib):
+    import torch
+    dims = dict(dim=768, heads=12, mlp_dim=3072)
+    w = P._BlockWeightsC(*([16] * 12), 768, 12, 3072, 1e-6)
+    n = lib.dora_workspace_size(50432, 256, ctypes.byref(w))
+    t, d, m = 50432, 768, 3072
+    assert n >= t * d * 2 * 7 + t * m * 2 + t * 4
+    assert n < t * d * 2 * 7 + t * m * 2 + t * 4 + 64 * 1024
+    assert lib.dora_workspace_size(-1, 1, ctypes.byref(w)) == 0
+    assert dims["dim"] == dims["heads"] * 64
+    del torch
+
+
+def test_python_binding_rejects_cpu_tensors(lib):
+    import torch
+    x = torch.zeros(4, 8, dtype=torch.bfloat16)
+    with pytest.raises(TypeError):
+        P.dora_layernorm(x, x[0], x[0], 1e-6, x)

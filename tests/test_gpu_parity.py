@@ -1,0 +1,482 @@
+"""GPU parity: every entry point of include/dora.h, called through the C ABI,
+against the fp64 oracle on the same seeded inputs.  Integer and byte outputs
+(kept_idx, cu_seqlens, ids, packed rows) must match bit for bit; floating
+outputs within |err| <= 2e-2 or |err| <= 1e-2 |ref|."""
+import numpy as np
+import pytest
+import torch
+
+import __graft_entry__ as G
+import dora_synth as S
+import oracle as O
+import paper_2609_34325_gb300 as P
+from helpers import assert_close, bf, bits, dev, f32, f64, i32, sub_batch
+
+pytestmark = pytest.mark.gpu
+
+CFGS = ("cfg1", "cfg2", "cfg3", "cfg4", "cfg5")
+SENT = -7
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    G.build()
+    P.load_library()
+    torch.cuda.set_device(0)
+
+
+def _status():
+    return torch.zeros(1, dtype=torch.int32, device=dev())
+
+
+# ---------------------------------------------------------------------------
+# select_keep
+# ---------------------------------------------------------------------------
+
+def _run_select(scores, cu, keeps, max_seqlen):
+    t_in = int(cu[-1])
+    b = len(cu) - 1
+    kept = torch.full((max(t_in, 1),), SENT, dtype=torch.int32, device=dev())
+    cu_out = torch.full((b + 1,), SENT, dtype=torch.int32, device=dev())
+    st = _status()
+    P.dora_select_keep(f32(scores), i32(cu), i32(keeps), max_seqlen, kept, cu_out, st)
+    torch.cuda.synchronize()
+    return kept.cpu().numpy(), cu_out.cpu().numpy(), int(st.item())
+
+
+def _check_select(scores, cu, keeps, max_seqlen=None):
+    lens = np.diff(cu)
+    ms = int(lens.max()) if max_seqlen is None else max_seqlen
+    kept, cu_out, st = _run_select(scores, cu, keeps, ms)
+    rk, rcu, rst = O.select_keep(scores, cu, keeps)
+    assert np.array_equal(cu_out, rcu)
+    t_out = int(rcu[-1])
+    assert np.array_equal(kept[:t_out], rk)
+    assert np.all(kept[t_out:] == SENT)            # nothing written past T_out
+    assert st == rst
+    return t_out
+
+
+@pytest.mark.parametrize("name", CFGS)
+def test_select_keep_configs(name):
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    keeps, _ = S.keep_schedule(cfg, 0)
+    for j, blk in enumerate(cfg.prune_blocks[:2]):
+        table = S.score_table(cfg, blk, 0)
+        # the second step uses the packed layout produced by the first
+        if j == 0:
+            lcu, lids = cu, ids
+        scores = O.gather_scores(table, lcu, lids)
+        _check_select(scores, lcu, keeps[j], cfg.n_tokens)
+        rk, rcu, _ = O.select_keep(scores, lcu, keeps[j])
+        lcu, lids = rcu, lids[rk]
+
+
+def _edge_lengths():
+    return np.array([1, 2, 15, 16, 17, 31, 32, 33, 64, 127, 128, 129, 197, 255, 256, 257, 577])
+
+
+@pytest.mark.parametrize("kind", ["uniform", "ties", "special", "allequal"])
+def test_select_keep_edges(kind):
+    rng = np.random.default_rng(42)
+    lens = _edge_lengths()
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    if kind == "uniform":
+        s = rng.random(t).astype(np.float32)
+    elif kind == "ties":
+        s = rng.choice(np.array([0.0, 0.25, 0.5], np.float32), size=t)
+    elif kind == "allequal":
+        s = np.full(t, 0.125, np.float32)
+    else:
+        pal = np.array([0.0, -0.0, np.nan, -np.nan, np.inf, -np.inf, 1.0, -1.0, 1e-38, -1e-38],
+                       dtype=np.float32)
+        s = rng.choice(pal, size=t)
+        s[rng.random(t) < 0.02] = np.float32(np.nan)
+    for mode in ("one", "all", "random"):
+        if mode == "one":
+            keeps = np.ones_like(lens)
+        elif mode == "all":
+            keeps = lens.copy()
+        else:
+            keeps = np.array([rng.integers(1, n + 1) for n in lens])
+        _check_select(s, cu, keeps)
+
+
+def test_select_keep_bad_counts_and_empty_images():
+    lens = np.array([5, 0, 9, 3, 12])
+    cu = O.cu_from_counts(lens)
+    s = np.random.default_rng(3).random(int(cu[-1])).astype(np.float32)
+    keeps = np.array([0, 0, 20, 3, -4])       # 0 (<1), empty ok, >n, ok, negative
+    _check_select(s, cu, keeps)
+    _, _, st = _run_select(s, cu, keeps, 12)
+    assert st == O.DORA_ERR_DEVICE_BAD_COUNT
+
+
+def test_select_keep_longer_than_max_seqlen_flags():
+    lens = np.array([10, 40, 10])
+    cu = O.cu_from_counts(lens)
+    s = np.random.default_rng(4).random(60).astype(np.float32)
+    kept, cu_out, st = _run_select(s, cu, np.array([5, 5, 5]), 32)
+    assert st == 6
+    assert cu_out.tolist() == [0, 5, 5, 10]     # the long image keeps nothing
+
+
+def test_select_keep_large_batch_b1024():
+    rng = np.random.default_rng(5)
+    lens = rng.integers(1, 198, size=1024)
+    cu = O.cu_from_counts(lens)
+    s = rng.random(int(cu[-1])).astype(np.float32)
+    keeps = np.array([rng.integers(1, n + 1) for n in lens])
+    _check_select(s, cu, keeps, 197)
+
+
+# ---------------------------------------------------------------------------
+# compaction
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name", CFGS)
+def test_compact_bit_exact(name):
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    keeps, _ = S.keep_schedule(cfg, 1)
+    scores = O.gather_scores(S.score_table(cfg, cfg.prune_blocks[0], 1), cu, ids)
+    rk, rcu, _ = O.select_keep(scores, cu, keeps[0])
+    t_in, t_out = int(cu[-1]), int(rcu[-1])
+    rng = np.random.default_rng(6)
+    x = rng.integers(0, 65536, size=(t_in, cfg.dim), dtype=np.uint16)   # any bit pattern
+    packed = torch.zeros(t_in, cfg.dim, dtype=torch.bfloat16, device=dev())
+    packed.view(torch.int16).fill_(SENT)
+    ids_out = torch.full((t_in,), SENT, dtype=torch.int32, device=dev())
+    st = _status()
+    kept_d = torch.zeros(t_in, dtype=torch.int32, device=dev())
+    kept_d[:t_out] = i32(rk)
+    P.dora_compact(bf(x), kept_d, i32(rcu), packed, ids_in=i32(ids), ids_out=ids_out, status=st)
+    torch.cuda.synchronize()
+    ref_packed, ref_ids = O.compact(x, rk, ids)
+    got = bits(packed)
+    assert np.array_equal(got[:t_out], ref_packed)
+    assert np.all(got[t_out:].view(np.int16) == SENT)
+    assert np.array_equal(ids_out.cpu().numpy()[:t_out], ref_ids)
+    assert int(st.item()) == 0
+
+
+@pytest.mark.parametrize("name", ["cfg1", "cfg3", "cfg4"])
+def test_compact_ln_fused(name):
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    keeps, _ = S.keep_schedule(cfg, 2)
+    scores = O.gather_scores(S.score_table(cfg, cfg.prune_blocks[0], 2), cu, ids)
+    rk, rcu, _ = O.select_keep(scores, cu, keeps[0])
+    t_in, t_out = int(cu[-1]), int(rcu[-1])
+    x = S.activations_bf16(cfg, 2)
+    wb = S.block_weights(cfg, 0, 2, random_affine=True)
+    packed = torch.zeros(t_in, cfg.dim, dtype=torch.bfloat16, device=dev())
+    ln = torch.zeros_like(packed)
+    kept_d = torch.zeros(t_in, dtype=torch.int32, device=dev())
+    kept_d[:t_out] = i32(rk)
+    P.dora_compact_ln(bf(x), kept_d, i32(rcu), bf(wb["ln2_w"]), bf(wb["ln2_b"]), cfg.ln_eps,
+                      packed, ln)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits(packed)[:t_out], x[rk])
+    ref = O.layernorm(O.bf16_to_f64(x[rk]), O.bf16_to_f64(wb["ln2_w"]),
+                      O.bf16_to_f64(wb["ln2_b"]), cfg.ln_eps)
+    assert_close(f64(ln[:t_out]), ref, "compact_ln")
+
+
+def test_compact_empty_output():
+    cu_out = i32(np.zeros(4))
+    x = torch.zeros(10, 64, dtype=torch.bfloat16, device=dev())
+    packed = torch.full_like(x, 3.0)
+    P.dora_compact(x, torch.zeros(10, dtype=torch.int32, device=dev()), cu_out, packed)
+    torch.cuda.synchronize()
+    assert torch.all(packed == 3.0)
+
+
+# ---------------------------------------------------------------------------
+# LayerNorm
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("dim", [64, 192, 384, 768, 1024, 2048])
+def test_layernorm(dim):
+    rng = np.random.default_rng(dim)
+    rows_cap, rows = 1000, 777
+    x = S.f32_to_bf16_bits(rng.standard_normal((rows_cap, dim)) * 3 + 1)
+    w = S.f32_to_bf16_bits(1 + 0.1 * rng.standard_normal(dim))
+    b = S.f32_to_bf16_bits(0.1 * rng.standard_normal(dim))
+    y = torch.full((rows_cap, dim), 5.0, dtype=torch.bfloat16, device=dev())
+    P.dora_layernorm(bf(x), bf(w), bf(b), 1e-6, y, rows_dev=i32([rows]))
+    torch.cuda.synchronize()
+    ref = O.layernorm(O.bf16_to_f64(x[:rows]), O.bf16_to_f64(w), O.bf16_to_f64(b), 1e-6)
+    assert_close(f64(y[:rows]), ref, f"layernorm d={dim}")
+    assert torch.all(y[rows:] == 5.0)
+
+
+# ---------------------------------------------------------------------------
+# linear (tcgen05 GEMM)
+# ---------------------------------------------------------------------------
+
+LINEAR_CASES = [
+    # m_cap, m_live, k, n, epilogue
+    (128, 128, 64, 128, 0),
+    (300, 300, 192, 576, 0),       # ragged M, N not a multiple of 256
+    (1576, 1576, 192, 576, 0),     # cfg1 QKV
+    (1576, 1200, 192, 768, 1),     # cfg1 fc1 after a deletion
+    (1576, 1200, 768, 192, 2),     # cfg1 fc2
+    (12608, 7904, 384, 1152, 0),   # cfg2 QKV shape, fewer live rows
+    (2000, 1999, 768, 2304, 0),
+    (2000, 1001, 768, 3072, 1),
+    (2000, 1500, 3072, 768, 2),
+    (777, 777, 1024, 4096, 1),
+    (777, 640, 4096, 1024, 2),
+    (129, 1, 64, 32, 2),
+    (256, 0, 64, 256, 0),
+]
+
+
+@pytest.mark.parametrize("m_cap,m_live,k,n,epi", LINEAR_CASES)
+def test_linear(m_cap, m_live, k, n, epi):
+    rng = np.random.default_rng(m_cap * 7 + n + epi)
+    x = S.f32_to_bf16_bits(rng.standard_normal((m_cap, k)))
+    w = S.f32_to_bf16_bits(0.02 * rng.standard_normal((n, k)))
+    b = S.f32_to_bf16_bits(0.1 * rng.standard_normal(n))
+    r = S.f32_to_bf16_bits(rng.standard_normal((m_cap, n)))
+    y = torch.full((m_cap, n), 7.0, dtype=torch.bfloat16, device=dev())
+    st = _status()
+    P.dora_linear(bf(x), bf(w), y, bias=bf(b), residual=bf(r) if epi == 2 else None,
+                  epilogue=epi, m_dev=i32([m_live]), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ref = O.linear(O.bf16_to_f64(x[:m_live]), O.bf16_to_f64(w), O.bf16_to_f64(b))
+    if epi == 1:
+        ref = O.gelu(ref)
+    if epi == 2:
+        ref = ref + O.bf16_to_f64(r[:m_live])
+    assert_close(f64(y[:m_live]), ref, f"linear {m_cap}x{n}x{k} epi{epi}")
+    assert torch.all(y[m_live:] == 7.0)
+
+
+def test_linear_no_bias_full_rows():
+    rng = np.random.default_rng(9)
+    x = S.f32_to_bf16_bits(rng.standard_normal((512, 256)))
+    w = S.f32_to_bf16_bits(0.05 * rng.standard_normal((512, 256)))
+    y = torch.zeros(512, 512, dtype=torch.bfloat16, device=dev())
+    P.dora_linear(bf(x), bf(w), y)
+    torch.cuda.synchronize()
+    ref = O.bf16_to_f64(x) @ O.bf16_to_f64(w).T
+    assert_close(f64(y), ref, "linear no bias")
+
+
+# ---------------------------------------------------------------------------
+# varlen attention (tcgen05)
+# ---------------------------------------------------------------------------
+
+def _run_attn(qkv_bits, cu, heads, max_seqlen, t_cap=None):
+    t = qkv_bits.shape[0] if t_cap is None else t_cap
+    out = torch.full((t, heads * 64), 9.0, dtype=torch.bfloat16, device=dev())
+    st = _status()
+    P.dora_varlen_attn(bf(qkv_bits), i32(cu), max_seqlen, heads, out, status=st)
+    torch.cuda.synchronize()
+    return out, int(st.item())
+
+
+def _check_attn(lens, heads, seed, tail_nan=0):
+    rng = np.random.default_rng(seed)
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    qkv = S.f32_to_bf16_bits(rng.standard_normal((t + tail_nan, 3 * heads * 64)))
+    if tail_nan:
+        qkv[t:] = 0x7FC0            # NaN rows past the last image
+    out, st = _run_attn(qkv, cu, heads, int(max(lens)))
+    assert st == 0
+    ref = O.varlen_attention(qkv[:t], cu, heads)
+    assert_close(f64(out[:t]), ref, f"attn lens={list(lens)[:6]}")
+    if tail_nan:
+        assert torch.all(out[t:] == 9.0)
+
+
+@pytest.mark.parametrize("name", ["cfg1", "cfg2", "cfg3", "cfg4"])
+def test_attention_configs(name):
+    cfg = S.get_config(name)
+    keeps, _ = S.keep_schedule(cfg, 3)
+    _check_attn(np.full(cfg.batch, cfg.n_tokens), cfg.heads, 1)      # dense blocks
+    _check_attn(keeps[0], cfg.heads, 2)                               # after a deletion
+
+
+def test_attention_cfg5_long_sequences():
+    cfg = S.get_config("cfg5", batch=12)
+    keeps, _ = S.keep_schedule(cfg, 4)
+    _check_attn(np.full(4, 577), cfg.heads, 3)
+    _check_attn(keeps[1], cfg.heads, 4)
+
+
+def test_attention_edge_lengths_and_nan_tail():
+    _check_attn(np.array([1]), 1, 5)
+    _check_attn(np.array([1, 1, 1]), 2, 6)
+    _check_attn(np.array([16, 17, 31, 32, 33, 127, 128, 129]), 3, 7)
+    _check_attn(np.array([255, 256, 257, 383, 384, 385, 600]), 2, 8)
+    _check_attn(np.array([197, 5, 130]), 12, 9, tail_nan=70)
+
+
+def test_attention_empty_images_and_long_image_flag():
+    lens = np.array([0, 20, 0, 33])
+    _check_attn(lens, 2, 10)
+    cu = O.cu_from_counts(np.array([10, 300]))
+    qkv = S.f32_to_bf16_bits(np.random.default_rng(11).standard_normal((310, 3 * 64)))
+    _, st = _run_attn(qkv, cu, 1, 128)
+    assert st == 6
+
+
+def test_attention_matches_dense_when_unpruned():
+    """k = 0: packed attention equals dense batched attention (torch SDPA on
+    the same bf16 values, fp64) on the GPU path too."""
+    b, n, h = 4, 197, 3
+    rng = np.random.default_rng(12)
+    qkv = S.f32_to_bf16_bits(rng.standard_normal((b * n, 3 * h * 64)))
+    out, _ = _run_attn(qkv, np.arange(b + 1) * n, h, n)
+    a = torch.from_numpy(O.bf16_to_f64(qkv).reshape(b, n, 3, h, 64))
+    q, k, v = (a[:, :, j].permute(0, 2, 1, 3) for j in range(3))
+    dense = torch.nn.functional.scaled_dot_product_attention(q, k, v).permute(0, 2, 1, 3)
+    assert_close(f64(out), dense.reshape(b * n, h * 64).numpy(), "dense")
+
+
+# ---------------------------------------------------------------------------
+# the pruned block and the forward
+# ---------------------------------------------------------------------------
+
+def _device_weights(cfg, wb):
+    return P.BlockWeights({k: bf(v) for k, v in wb.items()}, cfg.dim, cfg.heads, cfg.mlp_dim,
+                          cfg.ln_eps)
+
+
+def _run_block(cfg, x_bits, cu, ids, w, scores=None, keeps=None, t_cap=None):
+    t_cap = t_cap or x_bits.shape[0]
+    ws = P.alloc_workspace(t_cap, cfg.batch, w)
+    x_out = torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev())
+    cu_out = torch.zeros(len(cu), dtype=torch.int32, device=dev())
+    ids_out = torch.full((t_cap,), SENT, dtype=torch.int32, device=dev())
+    kept = torch.full((t_cap,), SENT, dtype=torch.int32, device=dev())
+    xin = torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev())
+    xin[:x_bits.shape[0]] = bf(x_bits)
+    P.dora_pruned_block(xin, i32(cu), w, int(np.diff(cu).max()), x_out, ws, ids_in=i32(ids),
+                        scores=None if scores is None else f32(scores),
+                        keep_counts=None if keeps is None else i32(keeps), cu_out=cu_out,
+                        ids_out=ids_out, kept_idx=kept)
+    torch.cuda.synchronize()
+    st = P.dora_read_status(P.dora_workspace_status(ws))
+    return dict(x_out=x_out, cu_out=cu_out.cpu().numpy(), ids_out=ids_out.cpu().numpy(),
+                kept=kept.cpu().numpy(), status=st)
+
+
+def _check_block_images(cfg, x_bits, cu, ids, wb, scores, keeps, r, images):
+    """Oracle on a sub-batch of images (images are independent)."""
+    rows, lcu = sub_batch(cu, images)
+    wf = O.decode_weights(wb)
+    sub_scores = None if scores is None else scores[rows]
+    sub_keeps = None if keeps is None else np.asarray(keeps)[list(images)]
+    ref = O.pruned_block(O.bf16_to_f64(x_bits[rows]), lcu, ids[rows], wf, cfg.heads, cfg.ln_eps,
+                         sub_scores, sub_keeps)
+    cu_out = r["cu_out"] if scores is not None else cu
+    got_rows = np.concatenate([np.arange(cu_out[i], cu_out[i + 1]) for i in images])
+    assert_close(f64(r["x_out"])[got_rows], ref["x_out"], f"block {cfg.name} imgs {images}")
+
+
+@pytest.mark.parametrize("name", ["cfg1", "cfg2"])
+def test_block_full_oracle(name):
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    x = S.activations_bf16(cfg, 20)
+    wb = S.block_weights(cfg, 0, 20, random_affine=True)
+    keeps, _ = S.keep_schedule(cfg, 20)
+    scores = O.gather_scores(S.score_table(cfg, 0, 20), cu, ids)
+    w = _device_weights(cfg, wb)
+    r = _run_block(cfg, x, cu, ids, w, scores, keeps[0])
+    assert r["status"] == 0
+    ref = O.pruned_block(O.bf16_to_f64(x), cu, ids, O.decode_weights(wb), cfg.heads, cfg.ln_eps,
+                         scores, keeps[0])
+    t_out = int(ref["cu_out"][-1])
+    assert np.array_equal(r["cu_out"], ref["cu_out"])
+    assert np.array_equal(r["kept"][:t_out], ref["kept_idx"])
+    assert np.array_equal(r["ids_out"][:t_out], ref["ids_out"])
+    assert_close(f64(r["x_out"][:t_out]), ref["x_out"], f"block {name}")
+    # no deletion: the output boundaries are the input's and every row is computed
+    r0 = _run_block(cfg, x, cu, ids, w)
+    ref0 = O.pruned_block(O.bf16_to_f64(x), cu, ids, O.decode_weights(wb), cfg.heads, cfg.ln_eps)
+    assert_close(f64(r0["x_out"][:int(cu[-1])]), ref0["x_out"], f"dense block {name}")
+    # pruned rows equal the dense block's rows at the kept positions (Eq. 1)
+    assert np.array_equal(bits(r["x_out"][:t_out]), bits(r0["x_out"])[ref["kept_idx"]])
+
+
+@pytest.mark.parametrize("name", ["cfg3", "cfg4", "cfg5"])
+def test_block_full_size_sampled_images(name):
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    x = S.activations_bf16(cfg, 21)
+    blk = cfg.prune_blocks[0]
+    wb = S.block_weights(cfg, blk, 21, random_affine=True)
+    keeps, _ = S.keep_schedule(cfg, 21)
+    scores = O.gather_scores(S.score_table(cfg, blk, 21), cu, ids)
+    r = _run_block(cfg, x, cu, ids, _device_weights(cfg, wb), scores, keeps[0])
+    assert r["status"] == 0
+    rk, rcu, _ = O.select_keep(scores, cu, keeps[0])
+    assert np.array_equal(r["cu_out"], rcu)
+    assert np.array_equal(r["kept"][:int(rcu[-1])], rk)
+    assert np.array_equal(r["ids_out"][:int(rcu[-1])], ids[rk])
+    b = cfg.batch
+    _check_block_images(cfg, x, cu, ids, wb, scores, keeps[0], r, [0, b // 2, b - 1])
+
+
+def test_forward_deit_b_shape_per_block():
+    """Twelve DeiT-B-shape blocks pruned at 3/6/9 through the C ABI.  The token
+    trajectory (cu, ids, kept) must equal the oracle's bit for bit end to end;
+    each block's output is checked against the oracle fed the same block input
+    on sampled images."""
+    cfg = S.get_config("cfg3", batch=16)
+    cu, ids = S.initial_layout(cfg)
+    t_cap = int(cu[-1])
+    x = S.activations_bf16(cfg, 22)
+    keeps, _ = S.keep_schedule(cfg, 22)
+    sched = dict(zip(cfg.prune_blocks, keeps))
+    cur = torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev())
+    cur[:] = bf(x)
+    cu_d, ids_d = i32(cu), i32(ids)
+    host_cu, host_ids = cu.copy(), ids.copy()
+    for l in range(cfg.depth):
+        wb = S.block_weights(cfg, l, 22)
+        w = _device_weights(cfg, wb)
+        ws = P.alloc_workspace(t_cap, cfg.batch, w)
+        nxt = torch.zeros_like(cur)
+        x_in_bits = bits(cur)
+        kw = {}
+        if l in sched:
+            table = S.score_table(cfg, l, 22)
+            sc = torch.zeros(t_cap, dtype=torch.float32, device=dev())
+            P.dora_gather_scores(f32(table), ids_d, cu_d, sc)
+            cu_o = torch.zeros_like(cu_d)
+            ids_o = torch.zeros_like(ids_d)
+            kept = torch.zeros_like(ids_d)
+            kw = dict(scores=sc, keep_counts=i32(sched[l]), cu_out=cu_o, ids_out=ids_o,
+                      kept_idx=kept)
+        P.dora_pruned_block(cur, cu_d, w, cfg.n_tokens, nxt, ws, ids_in=ids_d, **kw)
+        torch.cuda.synchronize()
+        assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+        scores = None
+        if l in sched:
+            scores = O.gather_scores(table, host_cu, host_ids)
+            assert np.array_equal(sc.cpu().numpy()[:int(host_cu[-1])], scores)
+            rk, rcu, _ = O.select_keep(scores, host_cu, sched[l])
+            assert np.array_equal(cu_o.cpu().numpy(), rcu)
+            assert np.array_equal(kept.cpu().numpy()[:int(rcu[-1])], rk)
+            assert np.array_equal(ids_o.cpu().numpy()[:int(rcu[-1])], host_ids[rk])
+        r = dict(x_out=nxt, cu_out=(cu_o.cpu().numpy() if l in sched else host_cu))
+        imgs = [l % cfg.batch]
+        _check_block_images(cfg, x_in_bits, host_cu, host_ids, wb, scores,
+                            sched.get(l), r, imgs)
+        if l in sched:
+            host_cu, host_ids = rcu, host_ids[rk]
+            cu_d, ids_d = cu_o, ids_o
+        cur = nxt
+    assert np.array_equal(np.diff(host_cu), keeps[-1])
