@@ -1,0 +1,622 @@
+#!/usr/bin/env python
+"""Pruned ViT forward throughput on GB300 through the libdora C ABI.
+
+Workload (default): DeiT-Base shape, batch 256 per GPU, 197 tokens, D=768,
+12 heads, MLP 3072, 12 blocks, hard pruning at blocks 3/6/9 with per-image
+removal counts drawn so the batch-mean token-layer compression (Eq. 4) is
+about 0.38; deletion scores are synthetic per-image tables keyed by original
+token id.  One step = one forward of the whole batch: at each pruning block
+the score gather (actor stand-in) and dora_pruned_block, elsewhere
+dora_pruned_block without deletion.
+
+Prints one JSON line.  ``--impl reference`` times the fp64 CPU oracle on the
+same workload instead (bounded samples, host cores only).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import dora_synth as S  # noqa: E402
+from paper_2609_34325_gb300 import accounting as A  # noqa: E402
+
+METRIC = "pruned ViT forward images/sec on 1 GB300; varlen-attn % bf16 peak; compact GB/s"
+UNIT = "images/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+# DRAM traffic per GEMM launch from an ncu capture (dram__bytes_read.sum +
+# dram__bytes_write.sum), keyed by the sha256 of the kernel source it was
+# taken on; reported as null once the source changes.
+NCU_TRAFFIC = {}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="cfg3")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--input-sets", type=int, default=3)
+    ap.add_argument("--cpu-images", type=int, default=2)
+    ap.add_argument("--no-extras", action="store_true",
+                    help="headline loop only (no dense, e2e, per-kernel or CPU legs)")
+    ap.add_argument("--graph", action="store_true", help="replay the step as a CUDA graph")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def sha256_of(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+# ---------------------------------------------------------------------------
+# workload (host side, shared by both arms)
+# ---------------------------------------------------------------------------
+class HostWorkload:
+    def __init__(self, cfg, seed, n_sets):
+        self.cfg = cfg
+        self.cu0, self.ids0 = S.initial_layout(cfg)
+        self.sets = []
+        for r in range(n_sets):
+            s = seed + 7919 * r
+            keeps, befores = S.keep_schedule(cfg, s)
+            tables = [S.score_table(cfg, blk, s) for blk in cfg.prune_blocks]
+            self.sets.append(dict(seed=s, x=S.activations_bf16(cfg, s), keeps=keeps,
+                                  befores=befores, tables=tables))
+        self.weights = [S.block_weights(cfg, l, seed) for l in range(cfg.depth)]
+
+    def lengths_per_block(self, r):
+        """Token count of every image entering each block, for set r."""
+        cfg = self.cfg
+        sched = dict(zip(cfg.prune_blocks, self.sets[r]["keeps"]))
+        n = np.full(cfg.batch, cfg.n_tokens, dtype=np.int64)
+        out = []
+        for l in range(cfg.depth):
+            m = sched[l].astype(np.int64) if l in sched else n
+            out.append((n.copy(), m.copy()))
+            n = m
+        return out
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.lines, self.proc, self.gpu_id = [], None, gpu_id
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.gpu_id, "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append((time.time(), ln.strip()))
+
+    def stop(self, t0, t1):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], None, set()
+        for ts, ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9 or not (t0 - 0.05 <= ts <= t1 + 0.15):
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+            for name, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def gpu_uuid_arg(torch, dev_index):
+    try:
+        u = str(torch.cuda.get_device_properties(dev_index).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return str(dev_index)
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        return _run_gpu_on_stream(args, rank, world, local_rank, dev, stream)
+
+
+def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
+    import torch
+    import paper_2609_34325_gb300 as P
+
+    P.load_library()
+    cfg = S.get_config(args.config)
+    peaks, peak_src = load_peaks()
+    hw = HostWorkload(cfg, args.seed + 100003 * rank, args.input_sets)
+    t_cap = cfg.batch * cfg.n_tokens
+
+    def bf(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    def i32(a):
+        return torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).to(dev)
+
+    blocks = [P.BlockWeights({k: bf(v) for k, v in w.items()}, cfg.dim, cfg.heads, cfg.mlp_dim,
+                             cfg.ln_eps) for w in hw.weights]
+    sets = [dict(x=bf(s["x"]), keeps=[i32(k) for k in s["keeps"]],
+                 tables=[torch.from_numpy(t).to(dev) for t in s["tables"]]) for s in hw.sets]
+    cu0, ids0 = i32(hw.cu0), i32(hw.ids0)
+    ws = P.alloc_workspace(t_cap, cfg.batch, blocks[0], dev)
+    xbuf = [torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    cubuf = [torch.zeros(cfg.batch + 1, dtype=torch.int32, device=dev) for _ in range(2)]
+    idbuf = [torch.zeros(t_cap, dtype=torch.int32, device=dev) for _ in range(2)]
+    scores = torch.zeros(t_cap, dtype=torch.float32, device=dev)
+    kept = torch.zeros(t_cap, dtype=torch.int32, device=dev)
+    prune = list(cfg.prune_blocks)
+    launches_per_step = {True: 0, False: 0}
+
+    def forward(inp, pruned=True):
+        x, cu, ids = inp["x"], cu0, ids0
+        n = 0
+        for l in range(cfg.depth):
+            out = xbuf[l % 2]
+            if pruned and l in prune:
+                j = prune.index(l)
+                P.dora_gather_scores(inp["tables"][j], ids, cu, scores, stream=stream)
+                P.dora_pruned_block(x, cu, blocks[l], cfg.n_tokens, out, ws, ids_in=ids,
+                                    scores=scores, keep_counts=inp["keeps"][j],
+                                    cu_out=cubuf[j % 2], ids_out=idbuf[j % 2], kept_idx=kept,
+                                    stream=stream)
+                cu, ids = cubuf[j % 2], idbuf[j % 2]
+                n += 1 + 8
+            else:
+                P.dora_pruned_block(x, cu, blocks[l], cfg.n_tokens, out, ws, ids_in=ids,
+                                    stream=stream)
+                n += 7
+            x = out
+        launches_per_step[pruned] = n
+        return x, cu
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    def max_over_ranks(v):
+        if world == 1:
+            return v
+        import torch.distributed as dist
+        t = torch.tensor([v], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def timed(step_fn, steps, warmup, sample_clocks=False):
+        for i in range(warmup):
+            step_fn(i)
+        torch.cuda.synchronize()
+        sampler = ClockSampler(gpu_uuid_arg(torch, local_rank)) if sample_clocks else None
+        if sampler:
+            sampler.start()
+            time.sleep(0.4)
+        barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        w0 = time.time()
+        e0.record(stream)
+        for i in range(steps):
+            step_fn(i)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        w1 = time.time()
+        barrier()
+        ms = e0.elapsed_time(e1)
+        clocks = sampler.stop(w0, w1) if sampler else None
+        return max_over_ranks(ms / 1000.0), clocks
+
+    nsets = len(sets)
+    graph = None
+    if args.graph:
+        # one graph per input set: the step is launch-only and capture-safe
+        graphs = []
+        for r in range(nsets):
+            forward(sets[r])
+            torch.cuda.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                forward(sets[r])
+            graphs.append(g)
+        graph = graphs
+
+    def step_pruned(i):
+        if graph is not None:
+            graph[i % nsets].replay()
+        else:
+            forward(sets[i % nsets], True)
+
+    secs, clocks = timed(step_pruned, args.steps, max(args.warmup, 3), sample_clocks=True)
+    images = cfg.batch * args.steps * world
+    value = images / secs
+    st = P.dora_read_status(P.dora_workspace_status(ws))
+    result = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3),
+        "ms_per_step": round(1000 * secs / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded bf16 N(0,1) activations, N(0,0.02) weights, U(0,1) score "
+                "tables); no trained weights or images",
+        "config": {
+            "workload": f"{cfg.name}: DeiT-B shape, batch {cfg.batch}/GPU, N={cfg.n_tokens}, "
+                        f"D={cfg.dim}, H={cfg.heads}, MLP {cfg.mlp_dim}, {cfg.depth} blocks, "
+                        f"prune at {'/'.join(map(str, cfg.prune_blocks))}",
+            "global_batch": cfg.batch * world, "seq_len": cfg.n_tokens,
+            "parallelism": f"dp{world} (independent replicas, no collective)",
+            "l2": f"{nsets} input sets cycled; each step also streams ~1 GB of weights and "
+                  "intermediates, far above the 129 MB L2",
+            "cuda_graph": bool(args.graph),
+        },
+        "clocks": clocks,
+        "gpu_launches": launches_per_step[True] * args.steps,
+        "device_status": st,
+    }
+    if args.no_extras:
+        return result, None
+
+    # unpruned dense forward: same kernels, no deletion
+    dsecs, _ = timed(lambda i: forward(sets[i % nsets], False), args.steps,
+                     max(args.warmup, 3))
+    result["dense"] = {"value": round(cfg.batch * args.steps * world / dsecs, 1), "unit": UNIT,
+                       "ms_per_step": round(1000 * dsecs / args.steps, 4)}
+    result["speedup_vs_dense"] = round(dsecs / secs, 4)
+
+    # end to end through the C ABI with host buffers
+    pin = [dict(x=torch.from_numpy(s["x"].view(np.int16)).view(torch.bfloat16).pin_memory(),
+                keeps=[torch.from_numpy(k.astype(np.int32)).pin_memory() for k in s["keeps"]],
+                tables=[torch.from_numpy(t).pin_memory() for t in s["tables"]])
+           for s in hw.sets]
+    dev_in = dict(x=torch.empty_like(sets[0]["x"]),
+                  keeps=[torch.empty_like(k) for k in sets[0]["keeps"]],
+                  tables=[torch.empty_like(t) for t in sets[0]["tables"]])
+    host_out = torch.empty(t_cap, cfg.dim, dtype=torch.bfloat16).pin_memory()
+    host_cu = torch.empty(cfg.batch + 1, dtype=torch.int32).pin_memory()
+    h2d = (pin[0]["x"].numel() * 2 + sum(k.numel() * 4 for k in pin[0]["keeps"])
+           + sum(t.numel() * 4 for t in pin[0]["tables"]))
+    d2h = host_out.numel() * 2 + host_cu.numel() * 4
+
+    def step_e2e(i):
+        src = pin[i % nsets]
+        dev_in["x"].copy_(src["x"], non_blocking=True)
+        for a, b in zip(dev_in["keeps"], src["keeps"]):
+            a.copy_(b, non_blocking=True)
+        for a, b in zip(dev_in["tables"], src["tables"]):
+            a.copy_(b, non_blocking=True)
+        x, cu = forward(dev_in, True)
+        host_out.copy_(x, non_blocking=True)
+        host_cu.copy_(cu, non_blocking=True)
+
+    esteps = max(3, min(args.steps, 50))
+    esecs, _ = timed(step_e2e, esteps, 3)
+    result["e2e"] = {"value": round(cfg.batch * esteps * world / esecs, 1), "unit": UNIT,
+                     "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                     "ms_per_step": round(1000 * esecs / esteps, 4)}
+
+    # per-kernel pass: the same step driven kernel by kernel with events
+    kern = profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap,
+                           steps=max(3, min(args.steps, 20)))
+    result.update(roofline_report(kern, peaks, peak_src))
+    return result, hw
+
+
+def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
+    """Run the pruned step launch by launch through the fine-grained entry
+    points (the same kernels dora_pruned_block launches), bracketing each
+    launch with CUDA events on the launching stream.  Returns per-class times
+    and algorithmic work."""
+    d, m = cfg.dim, cfg.mlp_dim
+    bf16 = torch.bfloat16
+    xn = torch.zeros(t_cap, d, dtype=bf16, device=dev)
+    qkv = torch.zeros(t_cap, 3 * d, dtype=bf16, device=dev)
+    o = torch.zeros(t_cap, d, dtype=bf16, device=dev)
+    hattn = torch.zeros(t_cap, d, dtype=bf16, device=dev)
+    hkeep = torch.zeros(t_cap, d, dtype=bf16, device=dev)
+    u = torch.zeros(t_cap, m, dtype=bf16, device=dev)
+    xb = [torch.zeros(t_cap, d, dtype=bf16, device=dev) for _ in range(2)]
+    cub = [torch.zeros(cfg.batch + 1, dtype=torch.int32, device=dev) for _ in range(2)]
+    idb = [torch.zeros(t_cap, dtype=torch.int32, device=dev) for _ in range(2)]
+    kept = torch.zeros(t_cap, dtype=torch.int32, device=dev)
+    scores = torch.zeros(t_cap, dtype=torch.float32, device=dev)
+    cu0 = torch.from_numpy(hw.cu0).to(dev)
+    ids0 = torch.from_numpy(hw.ids0).to(dev)
+    prune = list(cfg.prune_blocks)
+    B = cfg.batch
+    records = []   # (class, start_event, end_event, work dict)
+
+    def ev():
+        return torch.cuda.Event(enable_timing=True)
+
+    def launch(cls, fn, work):
+        a, b = ev(), ev()
+        a.record(stream)
+        fn()
+        b.record(stream)
+        records.append((cls, a, b, work))
+
+    for it in range(steps + 1):
+        r = it % len(sets)
+        inp = sets[r]
+        lens = hw.lengths_per_block(r)
+        x, cu, ids = inp["x"], cu0, ids0
+        if it == 1:
+            torch.cuda.synchronize()
+            records.clear()
+        for l in range(cfg.depth):
+            w = blocks[l].tensors
+            n_in, n_out = lens[l]
+            T, To = int(n_in.sum()), int(n_out.sum())
+            rows = cu[B:]
+            launch("layernorm", lambda: P.dora_layernorm(x, w["ln1_w"], w["ln1_b"], cfg.ln_eps,
+                                                        xn, rows_dev=rows, stream=stream),
+                   dict(bytes=4.0 * T * d))
+            launch("gemm", lambda: P.dora_linear(xn, w["w_qkv"], qkv, bias=w["b_qkv"],
+                                                m_dev=rows, stream=stream),
+                   dict(flops=2.0 * T * 3 * d * d, bytes=2.0 * (T * d + 3 * d * d + 3 * T * d)))
+            launch("attention", lambda: P.dora_varlen_attn(qkv, cu, cfg.n_tokens, cfg.heads, o,
+                                                          stream=stream),
+                   dict(flops=A.attention_flops(n_in, cfg.heads), bytes=A.attention_bytes(T, d)))
+            launch("gemm", lambda: P.dora_linear(o, w["w_proj"], hattn, bias=w["b_proj"],
+                                                residual=x, epilogue=P.EPI_BIAS_RESIDUAL,
+                                                m_dev=rows, stream=stream),
+                   dict(flops=2.0 * T * d * d, bytes=2.0 * (3 * T * d + d * d)))
+            out = xb[l % 2]
+            if l in prune:
+                j = prune.index(l)
+                cuo, ido = cub[j % 2], idb[j % 2]
+                launch("gather_scores",
+                       lambda: P.dora_gather_scores(inp["tables"][j], ids, cu, scores,
+                                                    stream=stream),
+                       dict(bytes=12.0 * T))
+                launch("select_keep",
+                       lambda: P.dora_select_keep(scores, cu, inp["keeps"][j], cfg.n_tokens,
+                                                  kept, cuo, stream=stream),
+                       dict(bytes=4.0 * T + 4.0 * To + 8.0 * (B + 1) + 4.0 * B))
+                launch("compact_ln",
+                       lambda: P.dora_compact_ln(hattn, kept, cuo, w["ln2_w"], w["ln2_b"],
+                                                 cfg.ln_eps, hkeep, xn, ids_in=ids, ids_out=ido,
+                                                 stream=stream),
+                       dict(bytes=3.0 * 2 * To * d + 4.0 * To + 8.0 * To + 4.0 * (B + 1)))
+                hk, rows2 = hkeep, cuo[B:]
+                cu, ids = cuo, ido
+            else:
+                launch("layernorm", lambda: P.dora_layernorm(hattn, w["ln2_w"], w["ln2_b"],
+                                                            cfg.ln_eps, xn, rows_dev=rows,
+                                                            stream=stream),
+                       dict(bytes=4.0 * T * d))
+                hk, rows2 = hattn, rows
+            launch("gemm", lambda: P.dora_linear(xn, w["w_fc1"], u, bias=w["b_fc1"],
+                                                epilogue=P.EPI_BIAS_GELU, m_dev=rows2,
+                                                stream=stream),
+                   dict(flops=2.0 * To * d * m, bytes=2.0 * (To * d + d * m + To * m)))
+            launch("gemm", lambda: P.dora_linear(u, w["w_fc2"], out, bias=w["b_fc2"],
+                                                residual=hk, epilogue=P.EPI_BIAS_RESIDUAL,
+                                                m_dev=rows2, stream=stream),
+                   dict(flops=2.0 * To * m * d, bytes=2.0 * (To * m + m * d + 2 * To * d)))
+            x = out
+    torch.cuda.synchronize()
+    agg = {}
+    for cls, a, b, work in records:
+        e = agg.setdefault(cls, dict(ms=0.0, launches=0, flops=0.0, bytes=0.0))
+        e["ms"] += a.elapsed_time(b)
+        e["launches"] += 1
+        e["flops"] += work.get("flops", 0.0)
+        e["bytes"] += work.get("bytes", 0.0)
+    total = sum(e["ms"] for e in agg.values())
+    for e in agg.values():
+        e["share"] = e["ms"] / total if total else 0.0
+        e["ms"] /= steps
+        e["launches"] //= steps
+        e["flops"] /= steps
+        e["bytes"] /= steps
+    return agg
+
+
+def roofline_report(kern, peaks, peak_src):
+    tag = f"of {peak_src}"
+    g = kern["gemm"]
+    gemm_tf = g["flops"] / (g["ms"] * 1e-3) / 1e12
+    src = os.path.join(ROOT, "paper_2609_34325_gb300", "csrc", "gemm_tcgen05.cu")
+    tr = NCU_TRAFFIC.get(sha256_of(src))
+    out = {"roofline": {"kernel": "gemm_tcgen05 (QKV/proj/fc1/fc2)", "bound": "tensor",
+                        "achieved": round(gemm_tf, 1), "peak": peaks["bf16_tflops_sustained"],
+                        "unit": "TFLOP/s", "frac": round(gemm_tf / peaks["bf16_tflops_sustained"], 4),
+                        "peak_kind": f"bf16 sustained ({tag})",
+                        "frac_of_burst": round(gemm_tf / peaks["bf16_tflops"], 4),
+                        "traffic": tr,
+                        "algorithmic_bytes_per_launch": round(g["bytes"] / g["launches"]),
+                        "share_of_step": round(g["share"], 4)}}
+    a = kern["attention"]
+    at_tf = a["flops"] / (a["ms"] * 1e-3) / 1e12
+    ai = a["flops"] / a["bytes"]
+    attain = min(peaks["bf16_tflops"], ai * peaks["hbm_gbs"] / 1e3)
+    out["roofline_attention"] = {
+        "bound": "tensor", "achieved": round(at_tf, 1), "peak": peaks["bf16_tflops"],
+        "unit": "TFLOP/s", "frac": round(at_tf / peaks["bf16_tflops"], 4),
+        "peak_kind": f"bf16 burst ({tag})", "arith_intensity": round(ai, 1),
+        "attainable_from_hbm": round(attain, 1), "frac_of_attainable": round(at_tf / attain, 4),
+        "share_of_step": round(a["share"], 4)}
+    c = kern["compact_ln"]
+    c_gbs = c["bytes"] / (c["ms"] * 1e-3) / 1e9
+    s = kern["select_keep"]
+    sel_gbs = s["bytes"] / (s["ms"] * 1e-3) / 1e9
+    out["roofline_compact"] = {
+        "kernel": "compact_ln (compaction fused with LayerNorm')", "bound": "hbm",
+        "achieved": round(c_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+        "frac": round(c_gbs / peaks["hbm_gbs"], 4), "peak_kind": f"HBM copy ({tag})",
+        "select_keep_gbs": round(sel_gbs, 1), "select_keep_us": round(1000 * s["ms"] / s["launches"], 2),
+        "compact_us": round(1000 * c["ms"] / c["launches"], 2),
+        "share_of_step": round(c["share"] + s["share"], 4)}
+    out["kernels"] = {k: {"ms_per_step": round(v["ms"], 4), "launches_per_step": v["launches"],
+                          "share": round(v["share"], 4)} for k, v in sorted(kern.items())}
+    return out
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle legs
+# ---------------------------------------------------------------------------
+def oracle_sample(hw, r, images, blocks_subset=None):
+    """Run the fp64 oracle forward on the chosen images of input set r.
+    Returns seconds and the number of image-blocks processed."""
+    import oracle as O
+    cfg = hw.cfg
+    s = hw.sets[r]
+    rows = np.concatenate([np.arange(hw.cu0[i], hw.cu0[i + 1]) for i in images])
+    lcu = np.arange(len(images) + 1, dtype=np.int64) * cfg.n_tokens
+    x = O.bf16_to_f64(s["x"][rows])
+    ids = hw.ids0[rows]
+    layers = range(cfg.depth) if blocks_subset is None else blocks_subset
+    sched = {blk: j for j, blk in enumerate(cfg.prune_blocks)}
+    wf = {l: O.decode_weights(hw.weights[l]) for l in layers}
+    t0 = time.perf_counter()
+    cu = lcu
+    for l in layers:
+        if l in sched:
+            j = sched[l]
+            table = s["tables"][j][list(images)]
+            keep = s["keeps"][j][list(images)]
+            sc = O.gather_scores(table, cu, ids)
+            res = O.pruned_block(x, cu, ids, wf[l], cfg.heads, cfg.ln_eps, sc, keep)
+        else:
+            res = O.pruned_block(x, cu, ids, wf[l], cfg.heads, cfg.ln_eps)
+        if blocks_subset is None:
+            x, cu, ids = res["x_out"], res["cu_out"], res["ids_out"]
+    return time.perf_counter() - t0, len(images) * len(list(layers))
+
+
+def cpu_baseline(hw, n_images):
+    cfg = hw.cfg
+    cores = len(os.sched_getaffinity(0))
+    imgs = list(range(n_images))
+    secs, _ = oracle_sample(hw, 0, imgs)
+    return {"value": round(n_images / secs, 4), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{n_images} of {cfg.batch} images through all {cfg.depth} blocks "
+                      f"(fp64 numpy oracle, BLAS threads = {cores} host cores)",
+            "seconds": round(secs, 2)}
+
+
+def run_reference(args, rank, world):
+    if world > 1 and rank != 0:
+        return None
+    cfg = S.get_config(args.config)
+    hw = HostWorkload(cfg, args.seed, 1)
+    cores = len(os.sched_getaffinity(0))
+    # one step = image (step % B) through block (step % depth) of the same
+    # workload: 1/depth of an image-forward, so the run stays bounded
+    def step(i):
+        img = (i // cfg.depth) % cfg.batch
+        l = i % cfg.depth
+        return oracle_sample(hw, 0, [img], blocks_subset=[l])[0]
+
+    for i in range(max(args.warmup, 0)):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(args.warmup + i)
+    secs = time.perf_counter() - t0
+    value = (args.steps / cfg.depth) / secs
+    sample = (f"each step: 1 image through 1 of {cfg.depth} blocks (pruning blocks with their "
+              f"deletion), cycling blocks and images; fp64 numpy oracle on {cores} host cores")
+    return {"metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1000 * secs / max(args.steps, 1), 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg.name, "global_batch": cfg.batch, "seq_len": cfg.n_tokens,
+                       "parallelism": "host cores"},
+            "impl": "reference",
+            "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        res = run_reference(args, rank, world)
+        if res is not None:
+            print(json.dumps(res), flush=True)
+        return
+    res, hw = run_gpu(args, rank, world, local_rank)
+    if rank == 0:
+        if hw is not None:
+            res["cpu_baseline"] = cpu_baseline(hw, args.cpu_images)
+            keeps = hw.sets[0]["keeps"]
+            c = S.compression_from_counts(hw.cfg, keeps, hw.sets[0]["befores"])
+            sched = dict(zip(hw.cfg.prune_blocks, keeps))
+            fl = A.trajectory_flops(hw.cfg.depth, hw.cfg.dim, hw.cfg.mlp_dim, hw.cfg.n_tokens,
+                                    sched)
+            dense = A.trajectory_flops(hw.cfg.depth, hw.cfg.dim, hw.cfg.mlp_dim,
+                                       hw.cfg.n_tokens, {})
+            res["workload_stats"] = {"compression_C_mean": round(float(c.mean()), 4),
+                                     "block_gflops_per_image_pruned": round(float(fl.mean()) / 1e9, 3),
+                                     "block_gflops_per_image_dense": round(float(dense.mean()) / 1e9, 3)}
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
