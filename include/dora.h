@@ -55,6 +55,8 @@ enum dora_status {
   DORA_ERR_DEVICE_BAD_COUNT = 5,   /* device: keep count outside [1, n_i]; clamped */
   DORA_ERR_DEVICE_SEQLEN = 6,      /* device: an image is longer than max_seqlen,
                                       or a row index/count exceeds a capacity */
+  DORA_ERR_SCRATCH_TOO_SMALL = 7,  /* dora_pruned_block_noalloc: the block needs more
+                                      than DORA_NOALLOC_SCRATCH_BYTES of scratch */
 };
 
 /* Epilogues of dora_linear. */
@@ -242,6 +244,47 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
 
 /* Device address of the status word inside a dora_pruned_block workspace. */
 int32_t* dora_workspace_status(void* workspace);
+
+/*
+ * dora_pruned_block_noalloc -- dora_pruned_block for callers that cannot
+ * allocate device memory.  The paper has no counterpart: this is a deployment
+ * convenience of this library.
+ *
+ * Who needs it: code that must not call cudaMalloc at the point where it runs
+ * the block -- paths that may never synchronise the device (cudaMalloc and
+ * cudaFree can), plugins whose host framework owns all device memory and
+ * forbids side allocations, processes that reserved the whole device up
+ * front.  Such callers pass only inputs and outputs; the block's intermediates
+ * live in a scratch array that the library itself holds in device memory.
+ *
+ * Arguments are those of dora_pruned_block minus the workspace, plus
+ * `status` (nullable device int32) which receives the block's status word.
+ *
+ * Limits and behaviour:
+ *  - The scratch array holds DORA_NOALLOC_SCRATCH_BYTES (32 MiB) on every GPU
+ *    that loads the library, for the life of the process.  A block whose
+ *    dora_workspace_size(t_cap, batch, w) exceeds it is rejected with
+ *    DORA_ERR_SCRATCH_TOO_SMALL before anything is launched (32 MiB fits e.g.
+ *    a DeiT-Tiny-shape batch of 8 x 197 tokens, or about 1,900 token rows of
+ *    a DeiT-Base-shape block).
+ *  - The first call on a device looks up the device address of the scratch
+ *    array (cudaGetSymbolAddress) with that device current; make that first
+ *    call before any stream capture on the device.
+ *  - No cudaMalloc, cudaFree or other allocating routine is called.
+ *  - Every call on a device shares the same scratch, which keeps the previous
+ *    call's contents: the status word in it is cleared at the start of each
+ *    call and everything else is written before it is read.  Calls whose work
+ *    overlaps on the GPU (different streams, or different host threads,
+ *    without ordering between them) race on the scratch and give wrong
+ *    results: order them on one stream.
+ */
+#define DORA_NOALLOC_SCRATCH_BYTES (32u << 20)
+int dora_pruned_block_noalloc(const dora_bf16* x_in, const int32_t* cu_in,
+                              const int32_t* ids_in, int32_t batch, int32_t max_seqlen,
+                              int32_t t_cap, const dora_block_weights* w, const float* scores,
+                              const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
+                              int32_t* ids_out, int32_t* kept_idx, int32_t* status,
+                              dora_stream_t stream);
 
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug

@@ -19,13 +19,15 @@ __all__ = [
     "dora_select_keep", "dora_compact", "dora_compact_ln", "dora_layernorm", "dora_linear",
     "dora_varlen_attn", "dora_gather_scores", "BlockWeights", "dora_workspace_size",
     "dora_pruned_block", "dora_workspace_status", "dora_read_status", "alloc_workspace",
+    "dora_pruned_block_noalloc", "NOALLOC_SCRATCH_BYTES",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 EPI_BIAS, EPI_BIAS_GELU, EPI_BIAS_RESIDUAL = 0, 1, 2
 STATUS_NAMES = {0: "DORA_OK", 1: "DORA_ERR_INVALID_ARG", 2: "DORA_ERR_UNSUPPORTED",
                 3: "DORA_ERR_CUDA", 4: "DORA_ERR_TIMEOUT", 5: "DORA_ERR_DEVICE_BAD_COUNT",
-                6: "DORA_ERR_DEVICE_SEQLEN"}
+                6: "DORA_ERR_DEVICE_SEQLEN", 7: "DORA_ERR_SCRATCH_TOO_SMALL"}
+NOALLOC_SCRATCH_BYTES = 32 << 20
 
 _vp, _i32, _f32, _sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_float, ctypes.c_size_t
 _SIGS = {
@@ -45,6 +47,8 @@ _SIGS = {
     "dora_pruned_block": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp, _vp,
                                          _vp, _vp, _vp, _vp, _sz, _vp]),
     "dora_workspace_status": (_vp, [_vp]),
+    "dora_pruned_block_noalloc": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
+                                                 _vp, _vp, _vp, _vp, _vp, _vp]),
     "dora_read_status": (ctypes.c_int, [_vp, _vp]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
@@ -272,6 +276,30 @@ def dora_pruned_block(x_in, cu_in, weights: BlockWeights, max_seqlen, x_out, wor
         ctypes.byref(weights.c), _ptr(scores), _ptr(keep_counts), _ptr(x_out), _ptr(cu_out),
         _ptr(ids_out), _ptr(kept_idx), _ptr(workspace), workspace.numel(), _stream(stream)),
         "dora_pruned_block")
+
+
+def dora_pruned_block_noalloc(x_in, cu_in, weights: BlockWeights, max_seqlen, x_out,
+                              ids_in=None, scores=None, keep_counts=None, cu_out=None,
+                              ids_out=None, kept_idx=None, status=None, stream=None):
+    """dora_pruned_block without a workspace argument, for callers that cannot
+    allocate device memory when they run the block: the intermediates live in
+    a 32 MiB scratch array the library holds on each GPU.  Blocks needing more
+    raise DoraError (DORA_ERR_SCRATCH_TOO_SMALL).  Calls on one device share
+    that scratch, so keep them ordered on one stream.  ``status`` (optional
+    int32 CUDA tensor) receives the block's device status word."""
+    _req(x_in, torch.bfloat16, "x_in")
+    _req(x_out, torch.bfloat16, "x_out")
+    _req(cu_in, torch.int32, "cu_in")
+    for n, t in (("ids_in", ids_in), ("keep_counts", keep_counts), ("cu_out", cu_out),
+                 ("ids_out", ids_out), ("kept_idx", kept_idx), ("status", status)):
+        _req(t, torch.int32, n, optional=True)
+    _req(scores, torch.float32, "scores", optional=True)
+    t_cap = x_in.shape[0]
+    _check(load_library().dora_pruned_block_noalloc(
+        _ptr(x_in), _ptr(cu_in), _ptr(ids_in), cu_in.numel() - 1, int(max_seqlen), t_cap,
+        ctypes.byref(weights.c), _ptr(scores), _ptr(keep_counts), _ptr(x_out), _ptr(cu_out),
+        _ptr(ids_out), _ptr(kept_idx), _ptr(status), _stream(stream)),
+        "dora_pruned_block_noalloc")
 
 
 def dora_workspace_status(workspace) -> int:

@@ -105,6 +105,7 @@ const char* dora_status_string(int code) {
     case DORA_ERR_TIMEOUT: return "device wait timed out";
     case DORA_ERR_DEVICE_BAD_COUNT: return "keep count out of range (clamped)";
     case DORA_ERR_DEVICE_SEQLEN: return "sequence longer than max_seqlen or index past capacity";
+    case DORA_ERR_SCRATCH_TOO_SMALL: return "block needs more scratch than the no-alloc entry holds";
     default: return "unknown status";
   }
 }
