@@ -408,13 +408,13 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
             launch("layernorm", lambda: P.dora_layernorm(x, w["ln1_w"], w["ln1_b"], cfg.ln_eps,
                                                         xn, rows_dev=rows, stream=stream),
                    dict(bytes=4.0 * T * d))
-            launch("gemm", lambda: P.dora_linear(xn, w["w_qkv"], qkv, bias=w["b_qkv"],
+            launch("gemm_qkv", lambda: P.dora_linear(xn, w["w_qkv"], qkv, bias=w["b_qkv"],
                                                 m_dev=rows, stream=stream),
                    dict(flops=2.0 * T * 3 * d * d, bytes=2.0 * (T * d + 3 * d * d + 3 * T * d)))
             launch("attention", lambda: P.dora_varlen_attn(qkv, cu, cfg.n_tokens, cfg.heads, o,
                                                           stream=stream),
                    dict(flops=A.attention_flops(n_in, cfg.heads), bytes=A.attention_bytes(T, d)))
-            launch("gemm", lambda: P.dora_linear(o, w["w_proj"], hattn, bias=w["b_proj"],
+            launch("gemm_proj", lambda: P.dora_linear(o, w["w_proj"], hattn, bias=w["b_proj"],
                                                 residual=x, epilogue=P.EPI_BIAS_RESIDUAL,
                                                 m_dev=rows, stream=stream),
                    dict(flops=2.0 * T * d * d, bytes=2.0 * (3 * T * d + d * d)))
@@ -443,11 +443,11 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
                                                             stream=stream),
                        dict(bytes=4.0 * T * d))
                 hk, rows2 = hattn, rows
-            launch("gemm", lambda: P.dora_linear(xn, w["w_fc1"], u, bias=w["b_fc1"],
+            launch("gemm_fc1", lambda: P.dora_linear(xn, w["w_fc1"], u, bias=w["b_fc1"],
                                                 epilogue=P.EPI_BIAS_GELU, m_dev=rows2,
                                                 stream=stream),
                    dict(flops=2.0 * To * d * m, bytes=2.0 * (To * d + d * m + To * m)))
-            launch("gemm", lambda: P.dora_linear(u, w["w_fc2"], out, bias=w["b_fc2"],
+            launch("gemm_fc2", lambda: P.dora_linear(u, w["w_fc2"], out, bias=w["b_fc2"],
                                                 residual=hk, epilogue=P.EPI_BIAS_RESIDUAL,
                                                 m_dev=rows2, stream=stream),
                    dict(flops=2.0 * To * m * d, bytes=2.0 * (To * m + m * d + 2 * To * d)))
@@ -460,13 +460,20 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
         e["launches"] += 1
         e["flops"] += work.get("flops", 0.0)
         e["bytes"] += work.get("bytes", 0.0)
+    gemm = dict(ms=0.0, launches=0, flops=0.0, bytes=0.0)
+    for k in [k for k in agg if k.startswith("gemm_")]:
+        for f in gemm:
+            gemm[f] += agg[k][f]
     total = sum(e["ms"] for e in agg.values())
-    for e in agg.values():
+    agg["gemm"] = gemm
+    for k, e in agg.items():
         e["share"] = e["ms"] / total if total else 0.0
         e["ms"] /= steps
         e["launches"] //= steps
         e["flops"] /= steps
         e["bytes"] /= steps
+        if e["flops"]:
+            e["tflops"] = e["flops"] / (e["ms"] * 1e-3) / 1e12
     return agg
 
 
@@ -506,7 +513,9 @@ def roofline_report(kern, peaks, peak_src):
         "compact_us": round(1000 * c["ms"] / c["launches"], 2),
         "share_of_step": round(c["share"] + s["share"], 4)}
     out["kernels"] = {k: {"ms_per_step": round(v["ms"], 4), "launches_per_step": v["launches"],
-                          "share": round(v["share"], 4)} for k, v in sorted(kern.items())}
+                          "share": round(v["share"], 4),
+                          **({"tflops": round(v["tflops"], 1)} if "tflops" in v else {})}
+                      for k, v in sorted(kern.items())}
     return out
 
 

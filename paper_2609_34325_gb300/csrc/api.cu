@@ -52,7 +52,8 @@ int num_sms() {
 }
 
 int encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t outer,
-                        uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer) {
+                        uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer,
+                        int swizzle_bytes) {
   {
     std::lock_guard<std::mutex> lk(g_mu);
     if (g_encode == nullptr) {
@@ -71,7 +72,8 @@ int encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t ou
   cuuint32_t estr[2] = {1, 1};
   CUresult r = g_encode(reinterpret_cast<CUtensorMap*>(map), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
                         const_cast<void*>(base), dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? 0 : static_cast<int>(r);
 }

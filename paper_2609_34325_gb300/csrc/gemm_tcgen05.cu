@@ -2,15 +2,22 @@
 //   Y[M, N] = epi(X[M, K] W[N, K]^T + b)      (nn.Linear layout)
 // used for the QKV, projection and MLP linears of the pruned block (Eq. 1).
 //
-// Design (one persistent CTA per SM):
-//   warp 0     TMA producer: 128x64 X tile + BNx64 W tile per stage into a
-//              4-stage shared-memory ring (128-byte swizzle).
+// Design (one persistent CTA per SM, CTAs paired in clusters of two):
+//   The two CTAs of a cluster work on vertically adjacent output tiles
+//   (M-tiles 2p and 2p+1 of the same N-tile), so they need the same W tile.
+//   warp 0     TMA producer: the CTA's own 128x64 X tile, plus one half of the
+//              shared BNx64 W tile multicast into both CTAs, per stage of a
+//              4-stage shared-memory ring (128-byte swizzle).  Each W byte is
+//              read from L2 once per pair.
 //   warp 1     MMA issuer: one thread issues tcgen05.mma (M=128, N=BN, K=16)
 //              into one of two TMEM accumulators (2 x BN fp32 columns), so
 //              the epilogue of tile t overlaps the main loop of tile t+1.
-//   warps 2-9  epilogue: tcgen05.ld the accumulator (each thread owns one
-//              row, each warp half the columns), add bias, GELU or residual,
-//              round to bf16, store.
+//   warps 2-17 epilogue: tcgen05.ld the accumulator (each thread owns one
+//              row; four warps share a TMEM lane quarter, each a quarter of the
+//              columns), release the accumulator at once, then add bias, GELU
+//              or residual, round to bf16, stage each 32x32 chunk in shared
+//              memory (64-byte swizzle) and write it with a TMA tensor store.
+//              The tile that straddles the live row count stores row by row.
 // The live row count M may come from device memory (rows left after a
 // deletion); tiles past it are never scheduled.  Every wait is bounded.
 #include <cuda.h>
@@ -27,13 +34,18 @@ namespace gemm {
 constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int kStages = 4;
-constexpr int kEpiWarps = 8;
+constexpr int kEpiWarps = 16;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
+constexpr int kCluster = 2;
+constexpr uint16_t kPairMask = 0x3;
+
+constexpr int kStageChunk = 32 * 32;   // one warp's 32 rows x 32 columns, bf16
 
 template <int BN>
 struct Smem {
   uint16_t a[kStages][BM * BK];   // 16 KB per stage
   uint16_t b[kStages][BN * BK];   // BN * 128 B per stage
+  uint16_t out[kEpiWarps][kStageChunk];   // 2 KB per epilogue warp
   uint64_t full[kStages];
   uint64_t empty[kStages];
   uint64_t acc_full[2];
@@ -45,11 +57,38 @@ struct Smem {
   int consumed;
 };
 
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// GELU(x) = x * Phi(x), Phi(x) = (1 + erf(x / sqrt 2)) / 2, with erf from
+// formula 7.1.26 of Abramowitz & Stegun, Handbook of Mathematical Functions
+// (|erf error| <= 1.5e-7): for z >= 0,
+//     erf(z) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-z^2),
+//     t = 1 / (1 + p z).
+// With z = |x| / sqrt 2 and q = (1 - erf(z)) / 2:  Phi = 1 - q for x >= 0,
+// q for x < 0.  The constants below fold in the 1/sqrt 2 and the 1/2.
+__device__ __forceinline__ float gelu_erf(float x) {
+  constexpr float kP = 0.3275911f * 0.70710678118654752f;
+  constexpr float kA1 = 0.5f * 0.254829592f, kA2 = 0.5f * -0.284496736f,
+                  kA3 = 0.5f * 1.421413741f, kA4 = 0.5f * -1.453152027f,
+                  kA5 = 0.5f * 1.061405429f;
+  constexpr float kNegHalfLog2e = -0.72134752044448170f;   // exp(-x^2/2) = 2^(x^2 * this)
+  const float t = rcp_approx(fmaf(kP, fabsf(x), 1.0f));
+  const float poly = t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, kA5, kA4), kA3), kA2), kA1);
+  const float q = poly * ex2_approx(x * x * kNegHalfLog2e);
+  return x * (x >= 0.0f ? 1.0f - q : q);
+}
+
+// Epilogue arithmetic of one 32-column chunk of one row; returns 16 packed
+// bf16x2 words.  R is read only for the residual epilogue (row < M).
 template <int EPI>
-__device__ __forceinline__ void epilogue_store(const uint32_t (&r)[32], uint16_t* __restrict__ Y,
-                                               const uint16_t* __restrict__ bias,
-                                               const uint16_t* __restrict__ R, int row, int gcol,
-                                               int N) {
+__device__ __forceinline__ void epilogue_math(const uint32_t (&r)[32], uint32_t (&o)[16],
+                                              const uint16_t* __restrict__ bias,
+                                              const uint16_t* __restrict__ R, int row, int gcol,
+                                              int N, bool row_ok) {
   float v[32];
 #pragma unroll
   for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(r[e]);
@@ -68,38 +107,32 @@ __device__ __forceinline__ void epilogue_store(const uint32_t (&r)[32], uint16_t
   }
   if constexpr (EPI == DORA_EPI_BIAS_GELU) {
 #pragma unroll
-    for (int e = 0; e < 32; ++e) v[e] = 0.5f * v[e] * (1.0f + erff(v[e] * 0.70710678118654752f));
+    for (int e = 0; e < 32; ++e) v[e] = gelu_erf(v[e]);
   }
-  const size_t off = static_cast<size_t>(row) * N + gcol;
   if constexpr (EPI == DORA_EPI_BIAS_RESIDUAL) {
-    const uint4* rp = reinterpret_cast<const uint4*>(R + off);
+    if (row_ok) {
+      const uint4* rp = reinterpret_cast<const uint4*>(R + static_cast<size_t>(row) * N + gcol);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const uint4 rr = __ldg(rp + q);
-      const uint32_t* w = reinterpret_cast<const uint32_t*>(&rr);
+      for (int q = 0; q < 4; ++q) {
+        const uint4 rr = __ldg(rp + q);
+        const uint32_t* w = reinterpret_cast<const uint32_t*>(&rr);
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        v[q * 8 + 2 * e] += bf16_lo(w[e]);
-        v[q * 8 + 2 * e + 1] += bf16_hi(w[e]);
+        for (int e = 0; e < 4; ++e) {
+          v[q * 8 + 2 * e] += bf16_lo(w[e]);
+          v[q * 8 + 2 * e + 1] += bf16_hi(w[e]);
+        }
       }
     }
   }
-  uint4* yp = reinterpret_cast<uint4*>(Y + off);
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    uint4 o;
-    o.x = pack_bf16x2(v[q * 8 + 0], v[q * 8 + 1]);
-    o.y = pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]);
-    o.z = pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]);
-    o.w = pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]);
-    yp[q] = o;
-  }
+  for (int e = 0; e < 16; ++e) o[e] = pack_bf16x2(v[2 * e], v[2 * e + 1]);
 }
 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                uint16_t* __restrict__ Y, const uint16_t* __restrict__ bias,
+                const __grid_constant__ CUtensorMap tmY, uint16_t* __restrict__ Y,
+                const uint16_t* __restrict__ bias,
                 const uint16_t* __restrict__ R, int m_cap, const int32_t* __restrict__ m_dev,
                 int N, int K, int32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -115,15 +148,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int v = *m_dev;
     M = v < 0 ? 0 : (v > m_cap ? m_cap : v);
   }
+  // Work is a list of tile pairs: pair p covers M-tiles 2*(p / n_tiles) and
+  // 2*(p / n_tiles) + 1 of N-tile p % n_tiles; CTA `rank` of cluster c takes
+  // the M-tile 2*(p / n_tiles) + rank of pairs c, c + clusters, ...
+  // Both CTAs of a cluster walk the same pairs in lockstep.
+  const int rank = static_cast<int>(cluster_ctarank());
+  const int cid = blockIdx.x / kCluster;
+  const int n_clusters = gridDim.x / kCluster;
   const int n_tiles = (N + BN - 1) / BN;
-  const int num_tiles = ((M + BM - 1) / BM) * n_tiles;
+  const int m_pairs = (M + 2 * BM - 1) / (2 * BM);
+  const int num_pairs = m_pairs * n_tiles;
   const int kb_count = K / BK;
   constexpr uint32_t kTmemCols = 2 * BN;
+  constexpr int kHalfB = BN / 2;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&s.full[i], 1);
-      mbar_init(&s.empty[i], 1);
+      mbar_init(&s.empty[i], kCluster);      // both CTAs' MMAs release a stage
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s.acc_full[i], 1);
@@ -136,10 +178,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_barrier_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(&tmY);
   }
   if (warp == 1) tmem_alloc(&s.tmem_base, kTmemCols);
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();              // peers' barriers are initialised before any multicast
   tc_fence_after();
   const uint32_t tmem = s.tmem_base;
   volatile int* abort = &s.abort_flag;
@@ -148,9 +191,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       int it = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
-        const int mt = tile / n_tiles;
-        const int nt = tile - mt * n_tiles;
+      for (int pr = cid; ok && pr < num_pairs; pr += n_clusters) {
+        const int mt = 2 * (pr / n_tiles) + rank;
+        const int nt = pr % n_tiles;
         for (int kb = 0; kb < kb_count; ++kb) {
           const int st = it % kStages;
           const uint32_t ph = (it / kStages) & 1;
@@ -160,7 +203,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           mbar_arrive_expect_tx(&s.full[st], (BM + BN) * BK * 2);
           tma_load_2d(s.a[st], &tmA, &s.full[st], kb * BK, mt * BM);
-          tma_load_2d(s.b[st], &tmB, &s.full[st], kb * BK, nt * BN);
+          tma_load_2d_multicast(s.b[st] + rank * kHalfB * BK, &tmB, &s.full[st], kb * BK,
+                                nt * BN + rank * kHalfB, kPairMask);
           ++it;
         }
       }
@@ -171,7 +215,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc = idesc_bf16(BM, BN, false);
       int it = 0, ti = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++ti) {
+      for (int pr = cid; ok && pr < num_pairs; pr += n_clusters, ++ti) {
         const int acc = ti & 1;
         const uint32_t aph = (ti >> 1) & 1;
         if (!mbar_wait(&s.acc_empty[acc], aph ^ 1, abort)) break;
@@ -190,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             mma_bf16_ss(d, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
-          mma_commit(&s.empty[st]);
+          mma_commit_multicast(&s.empty[st], kPairMask);   // both CTAs' W halves free
           ++it;
         }
         if (ok) mma_commit(&s.acc_full[acc]);
@@ -200,31 +244,65 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_limited(&s.drain, 0, kWaitLimitNs);
     }
   } else {
+    constexpr int kCols = BN / 4;                 // columns per epilogue warp
+    constexpr int kChunks = kCols / 32;
     const int q = warp & 3;                       // TMEM lanes this warp may read
-    const int half = (warp - 2) >> 2;             // which half of the columns
+    const int slot = (warp - 2) >> 2;             // which quarter of the columns
     const uint32_t lane_sel = static_cast<uint32_t>(q * 32) << 16;
     int ti = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++ti) {
+    for (int pr = cid; pr < num_pairs; pr += n_clusters, ++ti) {
       const int acc = ti & 1;
       const uint32_t aph = (ti >> 1) & 1;
       if (!mbar_wait_warp(&s.acc_full[acc], aph, abort)) break;
       tc_fence_after();
-      const int mt = tile / n_tiles;
-      const int nt = tile - mt * n_tiles;
-      const int row = mt * BM + q * 32 + lane;
-#pragma unroll 1
-      for (int c = 0; c < BN / 2; c += 32) {
-        const int tcol = half * (BN / 2) + c;
-        uint32_t r[32];
-        tmem_ld32(tmem + lane_sel + static_cast<uint32_t>(acc * BN + tcol), r);
-        tmem_ld_wait();
-        const int gcol = nt * BN + tcol;
-        if (row < M && gcol < N) epilogue_store<EPI>(r, Y, bias, R, row, gcol, N);
-      }
+      const int mt = 2 * (pr / n_tiles) + rank;
+      const int nt = pr % n_tiles;
+      const int row0 = mt * BM + q * 32;          // first row of this warp
+      const int row = row0 + lane;
+      const bool whole = row0 + 32 <= M;           // all 32 rows live: TMA store
+      uint32_t r[kChunks][32];
+#pragma unroll
+      for (int c = 0; c < kChunks; ++c)
+        tmem_ld32(tmem + lane_sel + static_cast<uint32_t>(acc * BN + slot * kCols + c * 32),
+                  r[c]);
+      tmem_ld_wait();
+      // the accumulator is in registers: hand it back to the MMA warp now
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&s.acc_empty[acc]);
+      uint16_t* stage = s.out[warp - 2];
+#pragma unroll
+      for (int c = 0; c < kChunks; ++c) {
+        const int gcol = nt * BN + slot * kCols + c * 32;
+        if (gcol >= N || row0 >= M) continue;      // warp-uniform
+        uint32_t o[16];
+        epilogue_math<EPI>(r[c], o, bias, R, row, gcol, N, row < M);
+        if (whole) {
+          // row `lane` of the 32x32 chunk, 64-byte swizzle: 16-byte piece j
+          // of row l sits at piece j ^ ((l >> 1) & 3)
+          if (lane == 0) bulk_wait_group_read0();  // previous store has read the stage
+          __syncwarp();
+          uint8_t* rowp = reinterpret_cast<uint8_t*>(stage) + lane * 64;
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            *reinterpret_cast<uint4*>(rowp + ((j ^ ((lane >> 1) & 3)) << 4)) =
+                make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tmY, stage, gcol, row0);
+            bulk_commit_group();
+          }
+        } else if (row < M) {
+          uint4* yp = reinterpret_cast<uint4*>(Y + static_cast<size_t>(row) * N + gcol);
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            yp[j] = make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
+        }
+      }
     }
+    if (lane == 0) bulk_wait_group0();             // stores done before the CTA exits
+    __syncwarp();
   }
 
   __syncwarp();
@@ -236,6 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // let every TMA load that was issued but never consumed land first
       for (int it = s.consumed; it < s.issued; ++it)
         mbar_wait_limited(&s.full[it % kStages], (it / kStages) & 1, 100ull * 1000 * 1000);
+      __nanosleep(50000);      // the peer's last multicast halves
     }
     __syncthreads();
   }
@@ -243,10 +322,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  cluster_sync();              // no CTA leaves while its peer may still signal it
 }
 
 template <int BN, int EPI>
-static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb, uint16_t* y,
+static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
+                                 const CUtensorMap& ty, uint16_t* y,
                                  const uint16_t* bias, const uint16_t* residual, int m_cap,
                                  const int32_t* m_dev, int n, int k, int32_t* status,
                                  cudaStream_t stream) {
@@ -255,26 +336,52 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb, u
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  const long tiles = static_cast<long>((m_cap + BM - 1) / BM) * ((n + BN - 1) / BN);
-  const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
-  kern<<<grid, kThreads, smem, stream>>>(ta, tb, y, bias, residual, m_cap, m_dev, n, k, status);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kCluster;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // as many co-resident clusters as fit, capped by the tile pairs of m_cap
+  static int max_clusters[64] = {0};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev < 0 || dev >= 64) dev = 0;
+  if (max_clusters[dev] == 0) {
+    cfg.gridDim = dim3(kCluster * (num_sms() / kCluster));
+    int c = 0;
+    e = cudaOccupancyMaxActiveClusters(&c, kern, &cfg);
+    if (e != cudaSuccess) return e;
+    max_clusters[dev] = c > 0 ? c : 1;
+  }
+  const long pairs =
+      static_cast<long>((m_cap + 2 * BM - 1) / (2 * BM)) * ((n + BN - 1) / BN);
+  const long clusters = pairs < max_clusters[dev] ? pairs : max_clusters[dev];
+  cfg.gridDim = dim3(static_cast<unsigned>(kCluster * clusters));
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, ty, y, bias, residual, m_cap, m_dev, n, k,
+                            status);
 }
 
 template <int BN>
-static cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, uint16_t* y,
+static cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& ty,
+                             uint16_t* y,
                              const uint16_t* bias, const uint16_t* residual, int epi, int m_cap,
                              const int32_t* m_dev, int n, int k, int32_t* status,
                              cudaStream_t stream) {
   switch (epi) {
     case DORA_EPI_BIAS_GELU:
-      return launch_bn_epi<BN, DORA_EPI_BIAS_GELU>(ta, tb, y, bias, residual, m_cap, m_dev, n, k,
+      return launch_bn_epi<BN, DORA_EPI_BIAS_GELU>(ta, tb, ty, y, bias, residual, m_cap, m_dev, n, k,
                                                    status, stream);
     case DORA_EPI_BIAS_RESIDUAL:
-      return launch_bn_epi<BN, DORA_EPI_BIAS_RESIDUAL>(ta, tb, y, bias, residual, m_cap, m_dev, n,
+      return launch_bn_epi<BN, DORA_EPI_BIAS_RESIDUAL>(ta, tb, ty, y, bias, residual, m_cap, m_dev, n,
                                                        k, status, stream);
     default:
-      return launch_bn_epi<BN, DORA_EPI_BIAS>(ta, tb, y, bias, residual, m_cap, m_dev, n, k,
+      return launch_bn_epi<BN, DORA_EPI_BIAS>(ta, tb, ty, y, bias, residual, m_cap, m_dev, n, k,
                                               status, stream);
   }
 }
@@ -287,17 +394,20 @@ cudaError_t launch_linear(const uint16_t* x, int32_t m_cap, const int32_t* m_dev
                           int32_t* status, cudaStream_t stream) {
   if (m_cap == 0) return cudaSuccess;
   const int bn = (n % 256 == 0) ? 256 : 128;
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, ty;
   if (encode_tmap_2d_bf16(&ta, x, static_cast<uint64_t>(k), static_cast<uint64_t>(m_cap),
                           static_cast<uint64_t>(k) * 2, gemm::BK, gemm::BM) != 0)
     return cudaErrorInvalidValue;
   if (encode_tmap_2d_bf16(&tb, w, static_cast<uint64_t>(k), static_cast<uint64_t>(n),
-                          static_cast<uint64_t>(k) * 2, gemm::BK, static_cast<uint32_t>(bn)) != 0)
+                          static_cast<uint64_t>(k) * 2, gemm::BK, static_cast<uint32_t>(bn / 2)) != 0)
+    return cudaErrorInvalidValue;
+  if (encode_tmap_2d_bf16(&ty, y, static_cast<uint64_t>(n), static_cast<uint64_t>(m_cap),
+                          static_cast<uint64_t>(n) * 2, 32, 32, 64) != 0)
     return cudaErrorInvalidValue;
   if (bn == 256)
-    return gemm::launch_bn<256>(ta, tb, y, bias, residual, epilogue, m_cap, m_dev, n, k, status,
+    return gemm::launch_bn<256>(ta, tb, ty, y, bias, residual, epilogue, m_cap, m_dev, n, k, status,
                                 stream);
-  return gemm::launch_bn<128>(ta, tb, y, bias, residual, epilogue, m_cap, m_dev, n, k, status,
+  return gemm::launch_bn<128>(ta, tb, ty, y, bias, residual, epilogue, m_cap, m_dev, n, k, status,
                               stream);
 }
 

@@ -43,8 +43,10 @@ cudaError_t launch_varlen_attn(const uint16_t* qkv, const int32_t* cu, int32_t b
                                uint16_t* out, int32_t* status, cudaStream_t stream);
 
 // Tensor-map encoding through the driver entry point (no libcuda link).
+// swizzle_bytes: 128 (default) or 64 (CU_TENSOR_MAP_SWIZZLE_128B / _64B).
 int encode_tmap_2d_bf16(void* map, const void* base, uint64_t inner, uint64_t outer,
-                        uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer);
+                        uint64_t row_pitch_bytes, uint32_t box_inner, uint32_t box_outer,
+                        int swizzle_bytes = 128);
 
 int num_sms();
 

@@ -259,6 +259,27 @@ def test_linear(m_cap, m_live, k, n, epi):
     assert torch.all(y[m_live:] == 7.0)
 
 
+def test_linear_gelu_epilogue_within_one_bf16_ulp():
+    """The GELU epilogue against exact-erf GELU on a dense grid: x has one
+    nonzero column and W routes it to every output, so each output is
+    GELU(v) of an exactly known v; the result must be within one bf16 ulp,
+    plus the approximation's absolute bound (|x| * 0.75e-7 <= 1e-6 here) that
+    matters only in the far tail where GELU itself is below 1e-6."""
+    m, k, n = 4096, 64, 32
+    v = S.bf16_bits_to_f32(S.f32_to_bf16_bits(np.linspace(-9.0, 9.0, m))).astype(np.float64)
+    x = np.zeros((m, k))
+    x[:, 0] = v
+    w = np.zeros((n, k))
+    w[:, 0] = 1.0
+    y = torch.zeros(m, n, dtype=torch.bfloat16, device=dev())
+    P.dora_linear(bf(S.f32_to_bf16_bits(x)), bf(S.f32_to_bf16_bits(w)), y,
+                  epilogue=P.EPI_BIAS_GELU)
+    torch.cuda.synchronize()
+    ref = O.gelu(v)[:, None]
+    err = np.abs(f64(y) - ref)
+    assert np.all(err <= 2.0 ** -7 * np.abs(ref) + 1e-6), float(err.max())
+
+
 def test_linear_no_bias_full_rows():
     rng = np.random.default_rng(9)
     x = S.f32_to_bf16_bits(rng.standard_normal((512, 256)))
