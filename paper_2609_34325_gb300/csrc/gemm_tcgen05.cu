@@ -12,12 +12,13 @@
 //   warp 1     MMA issuer: one thread issues tcgen05.mma (M=128, N=BN, K=16)
 //              into one of two TMEM accumulators (2 x BN fp32 columns), so
 //              the epilogue of tile t overlaps the main loop of tile t+1.
-//   warps 2-17 epilogue: tcgen05.ld the accumulator (each thread owns one
-//              row; four warps share a TMEM lane quarter, each a quarter of the
-//              columns), release the accumulator at once, then add bias, GELU
-//              or residual, round to bf16, stage each 32x32 chunk in shared
-//              memory (64-byte swizzle) and write it with a TMA tensor store.
-//              The tile that straddles the live row count stores row by row.
+//   epilogue warps (2 .. 1 + kEpiWarps): tcgen05.ld the accumulator (each
+//              thread owns one row; the warps of a TMEM lane quarter split the
+//              columns), release it once in registers, add bias, GELU or
+//              residual, round to bf16, stage each 32x32 chunk in one of two
+//              shared-memory buffers (64-byte swizzle) and write it with a TMA
+//              tensor store.  The tile that straddles the live row count
+//              stores row by row.
 // The live row count M may come from device memory (rows left after a
 // deletion); tiles past it are never scheduled.  Every wait is bounded.
 #include <cuda.h>
@@ -34,18 +35,25 @@ namespace gemm {
 constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int kStages = 4;
-constexpr int kEpiWarps = 16;
-constexpr int kThreads = 64 + 32 * kEpiWarps;
+// Epilogue warps per CTA (a multiple of 4: one per TMEM lane quarter) and
+// staging buffers per warp, chosen per epilogue: the ALU-heavy GELU epilogue
+// wants more warps, the others fewer warps with double-buffered stores.
+template <int EPI>
+struct EpiCfg {
+  static constexpr int kWarps = EPI == DORA_EPI_BIAS_GELU ? 16 : 8;
+  static constexpr int kBufs = kWarps == 16 ? 1 : 2;
+  static constexpr int kThreads = 64 + 32 * kWarps;
+};
 constexpr int kCluster = 2;
 constexpr uint16_t kPairMask = 0x3;
 
 constexpr int kStageChunk = 32 * 32;   // one warp's 32 rows x 32 columns, bf16
 
-template <int BN>
+template <int BN, int EPI>
 struct Smem {
   uint16_t a[kStages][BM * BK];   // 16 KB per stage
   uint16_t b[kStages][BN * BK];   // BN * 128 B per stage
-  uint16_t out[kEpiWarps][kStageChunk];   // 2 KB per epilogue warp
+  uint16_t out[EpiCfg<EPI>::kWarps][EpiCfg<EPI>::kBufs][kStageChunk];   // 2 KB each
   uint64_t full[kStages];
   uint64_t empty[kStages];
   uint64_t acc_full[2];
@@ -70,20 +78,30 @@ __device__ __forceinline__ float rcp_approx(float x) {
 //     t = 1 / (1 + p z).
 // With z = |x| / sqrt 2 and q = (1 - erf(z)) / 2:  Phi = 1 - q for x >= 0,
 // q for x < 0.  The constants below fold in the 1/sqrt 2 and the 1/2.
-__device__ __forceinline__ float gelu_erf(float x) {
-  constexpr float kP = 0.3275911f * 0.70710678118654752f;
-  constexpr float kA1 = 0.5f * 0.254829592f, kA2 = 0.5f * -0.284496736f,
-                  kA3 = 0.5f * 1.421413741f, kA4 = 0.5f * -1.453152027f,
-                  kA5 = 0.5f * 1.061405429f;
-  constexpr float kNegHalfLog2e = -0.72134752044448170f;   // exp(-x^2/2) = 2^(x^2 * this)
-  const float t = rcp_approx(fmaf(kP, fabsf(x), 1.0f));
-  const float poly = t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, kA5, kA4), kA3), kA2), kA1);
-  const float q = poly * ex2_approx(x * x * kNegHalfLog2e);
-  return x * (x >= 0.0f ? 1.0f - q : q);
+// Evaluated on two values at once with the paired fp32 instructions
+// (fma/mul.rn.f32x2): the epilogue's ALU work is what limits this GEMM.
+__device__ __forceinline__ void gelu_erf2(float& x0, float& x1) {
+  const uint64_t P2 = f2_pack(0.3275911f * 0.70710678118654752f, 0.3275911f * 0.70710678118654752f);
+  const uint64_t ONE2 = f2_pack(1.0f, 1.0f);
+  const uint64_t A1 = f2_pack(0.5f * 0.254829592f, 0.5f * 0.254829592f);
+  const uint64_t A2 = f2_pack(0.5f * -0.284496736f, 0.5f * -0.284496736f);
+  const uint64_t A3 = f2_pack(0.5f * 1.421413741f, 0.5f * 1.421413741f);
+  const uint64_t A4 = f2_pack(0.5f * -1.453152027f, 0.5f * -1.453152027f);
+  const uint64_t A5 = f2_pack(0.5f * 1.061405429f, 0.5f * 1.061405429f);
+  const uint64_t C2 = f2_pack(-0.72134752044448170f, -0.72134752044448170f);
+  const uint64_t X = f2_pack(x0, x1);
+  float d0, d1;
+  f2_unpack(f2_fma(P2, f2_pack(fabsf(x0), fabsf(x1)), ONE2), d0, d1);
+  const uint64_t T = f2_pack(rcp_approx(d0), rcp_approx(d1));
+  const uint64_t poly =
+      f2_mul(T, f2_fma(T, f2_fma(T, f2_fma(T, f2_fma(T, A5, A4), A3), A2), A1));
+  float e0, e1;
+  f2_unpack(f2_mul(f2_mul(X, X), C2), e0, e1);
+  float q0, q1;
+  f2_unpack(f2_mul(poly, f2_pack(ex2_approx(e0), ex2_approx(e1))), q0, q1);
+  f2_unpack(f2_mul(X, f2_pack(x0 >= 0.0f ? 1.0f - q0 : q0, x1 >= 0.0f ? 1.0f - q1 : q1)), x0, x1);
 }
 
-// Epilogue arithmetic of one 32-column chunk of one row; returns 16 packed
-// bf16x2 words.  R is read only for the residual epilogue (row < M).
 template <int EPI>
 __device__ __forceinline__ void epilogue_math(const uint32_t (&r)[32], uint32_t (&o)[16],
                                               const uint16_t* __restrict__ bias,
@@ -100,14 +118,15 @@ __device__ __forceinline__ void epilogue_math(const uint32_t (&r)[32], uint32_t 
       const uint32_t* w = reinterpret_cast<const uint32_t*>(&bb);
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
-        v[q * 8 + 2 * e] += bf16_lo(w[e]);
-        v[q * 8 + 2 * e + 1] += bf16_hi(w[e]);
+        float& a = v[q * 8 + 2 * e];
+        float& b = v[q * 8 + 2 * e + 1];
+        f2_unpack(f2_add(f2_pack(a, b), f2_pack(bf16_lo(w[e]), bf16_hi(w[e]))), a, b);
       }
     }
   }
   if constexpr (EPI == DORA_EPI_BIAS_GELU) {
 #pragma unroll
-    for (int e = 0; e < 32; ++e) v[e] = gelu_erf(v[e]);
+    for (int e = 0; e < 32; e += 2) gelu_erf2(v[e], v[e + 1]);
   }
   if constexpr (EPI == DORA_EPI_BIAS_RESIDUAL) {
     if (row_ok) {
@@ -118,8 +137,9 @@ __device__ __forceinline__ void epilogue_math(const uint32_t (&r)[32], uint32_t 
         const uint32_t* w = reinterpret_cast<const uint32_t*>(&rr);
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          v[q * 8 + 2 * e] += bf16_lo(w[e]);
-          v[q * 8 + 2 * e + 1] += bf16_hi(w[e]);
+          float& a = v[q * 8 + 2 * e];
+          float& b = v[q * 8 + 2 * e + 1];
+          f2_unpack(f2_add(f2_pack(a, b), f2_pack(bf16_lo(w[e]), bf16_hi(w[e]))), a, b);
         }
       }
     }
@@ -129,7 +149,7 @@ __device__ __forceinline__ void epilogue_math(const uint32_t (&r)[32], uint32_t 
 }
 
 template <int BN, int EPI>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmY, uint16_t* __restrict__ Y,
                 const uint16_t* __restrict__ bias,
@@ -140,7 +160,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) record_status(status, DORA_ERR_UNSUPPORTED);
     return;
   }
-  Smem<BN>& s = *reinterpret_cast<Smem<BN>*>(smem_raw);
+  Smem<BN, EPI>& s = *reinterpret_cast<Smem<BN, EPI>*>(smem_raw);
+  constexpr int kEpiWarps = EpiCfg<EPI>::kWarps;
+  constexpr int kBufs = EpiCfg<EPI>::kBufs;
+  constexpr int kColGroups = kEpiWarps / 4;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   int M = m_cap;
@@ -244,11 +267,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_limited(&s.drain, 0, kWaitLimitNs);
     }
   } else {
-    constexpr int kCols = BN / 4;                 // columns per epilogue warp
+    constexpr int kCols = BN / kColGroups;        // columns per epilogue warp
     constexpr int kChunks = kCols / 32;
+    constexpr int kBatch = kChunks < 2 ? kChunks : 2;   // chunks per TMEM load
     const int q = warp & 3;                       // TMEM lanes this warp may read
-    const int slot = (warp - 2) >> 2;             // which quarter of the columns
+    const int slot = (warp - 2) >> 2;             // which column slice
     const uint32_t lane_sel = static_cast<uint32_t>(q * 32) << 16;
+    int buf = 0;                                  // staging buffer to write next
     int ti = 0;
     for (int pr = cid; pr < num_pairs; pr += n_clusters, ++ti) {
       const int acc = ti & 1;
@@ -259,45 +284,56 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int nt = pr % n_tiles;
       const int row0 = mt * BM + q * 32;          // first row of this warp
       const int row = row0 + lane;
-      const bool whole = row0 + 32 <= M;           // all 32 rows live: TMA store
-      uint32_t r[kChunks][32];
+      const bool whole = row0 + 32 <= M;          // all 32 rows live: TMA store
+#pragma unroll 1
+      for (int cb = 0; cb < kChunks; cb += kBatch) {
+        uint32_t r[kBatch][32];
 #pragma unroll
-      for (int c = 0; c < kChunks; ++c)
-        tmem_ld32(tmem + lane_sel + static_cast<uint32_t>(acc * BN + slot * kCols + c * 32),
-                  r[c]);
-      tmem_ld_wait();
-      // the accumulator is in registers: hand it back to the MMA warp now
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s.acc_empty[acc]);
-      uint16_t* stage = s.out[warp - 2];
-#pragma unroll
-      for (int c = 0; c < kChunks; ++c) {
-        const int gcol = nt * BN + slot * kCols + c * 32;
-        if (gcol >= N || row0 >= M) continue;      // warp-uniform
-        uint32_t o[16];
-        epilogue_math<EPI>(r[c], o, bias, R, row, gcol, N, row < M);
-        if (whole) {
-          // row `lane` of the 32x32 chunk, 64-byte swizzle: 16-byte piece j
-          // of row l sits at piece j ^ ((l >> 1) & 3)
-          if (lane == 0) bulk_wait_group_read0();  // previous store has read the stage
+        for (int c = 0; c < kBatch; ++c)
+          tmem_ld32(tmem + lane_sel +
+                        static_cast<uint32_t>(acc * BN + slot * kCols + (cb + c) * 32),
+                    r[c]);
+        tmem_ld_wait();
+        if (cb + kBatch == kChunks) {
+          // the accumulator is in registers: hand it back to the MMA warp
+          tc_fence_before();
           __syncwarp();
-          uint8_t* rowp = reinterpret_cast<uint8_t*>(stage) + lane * 64;
+          if (lane == 0) mbar_arrive(&s.acc_empty[acc]);
+        }
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            *reinterpret_cast<uint4*>(rowp + ((j ^ ((lane >> 1) & 3)) << 4)) =
-                make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            tma_store_2d(&tmY, stage, gcol, row0);
-            bulk_commit_group();
+        for (int c = 0; c < kBatch; ++c) {
+          const int gcol = nt * BN + slot * kCols + (cb + c) * 32;
+          if (gcol >= N || row0 >= M) continue;    // warp-uniform
+          uint32_t o[16];
+          epilogue_math<EPI>(r[c], o, bias, R, row, gcol, N, row < M);
+          if (whole) {
+            // row `lane` of the 32x32 chunk, 64-byte swizzle: 16-byte piece j
+            // of row l sits at piece j ^ ((l >> 1) & 3).  The store issued two
+            // chunks ago from this buffer must have read it.
+            uint16_t* stage = s.out[warp - 2][buf];
+            if (lane == 0) {
+              if constexpr (kBufs == 2) bulk_wait_group_read1();
+              else bulk_wait_group_read0();
+            }
+            __syncwarp();
+            uint8_t* rowp = reinterpret_cast<uint8_t*>(stage) + lane * 64;
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              *reinterpret_cast<uint4*>(rowp + ((j ^ ((lane >> 1) & 3)) << 4)) =
+                  make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tmY, stage, gcol, row0);
+              bulk_commit_group();
+            }
+            buf = (buf + 1) % kBufs;
+          } else if (row < M) {
+            uint4* yp = reinterpret_cast<uint4*>(Y + static_cast<size_t>(row) * N + gcol);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              yp[j] = make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
           }
-        } else if (row < M) {
-          uint4* yp = reinterpret_cast<uint4*>(Y + static_cast<size_t>(row) * N + gcol);
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            yp[j] = make_uint4(o[4 * j], o[4 * j + 1], o[4 * j + 2], o[4 * j + 3]);
         }
       }
     }
@@ -331,7 +367,7 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
                                  const uint16_t* bias, const uint16_t* residual, int m_cap,
                                  const int32_t* m_dev, int n, int k, int32_t* status,
                                  cudaStream_t stream) {
-  const size_t smem = sizeof(Smem<BN>);
+  const size_t smem = sizeof(Smem<BN, EPI>);
   auto kern = gemm_kernel<BN, EPI>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
@@ -342,7 +378,7 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
   attr[0].val.clusterDim.x = kCluster;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(EpiCfg<EPI>::kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cfg.attrs = attr;
