@@ -102,48 +102,33 @@ __device__ __forceinline__ void gelu_erf2(float& x0, float& x1) {
   f2_unpack(f2_mul(X, f2_pack(x0 >= 0.0f ? 1.0f - q0 : q0, x1 >= 0.0f ? 1.0f - q1 : q1)), x0, x1);
 }
 
+// Adds 8 bf16 values (one 16-byte piece) to v[0..7] in fp32 pairs.
+__device__ __forceinline__ void add_bf16x8(float* v, const uint4& piece) {
+  const uint32_t* w = reinterpret_cast<const uint32_t*>(&piece);
+#pragma unroll
+  for (int e = 0; e < 4; ++e)
+    f2_unpack(f2_add(f2_pack(v[2 * e], v[2 * e + 1]), f2_pack(bf16_lo(w[e]), bf16_hi(w[e]))),
+              v[2 * e], v[2 * e + 1]);
+}
+
+// Bias and GELU of one 32-column chunk of one row, in fp32.
 template <int EPI>
-__device__ __forceinline__ void epilogue_math(const uint32_t (&r)[32], uint32_t (&o)[16],
-                                              const uint16_t* __restrict__ bias,
-                                              const uint16_t* __restrict__ R, int row, int gcol,
-                                              int N, bool row_ok) {
-  float v[32];
+__device__ __forceinline__ void epilogue_math(const uint32_t (&r)[32], float (&v)[32],
+                                              const uint16_t* __restrict__ bias, int gcol) {
 #pragma unroll
   for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(r[e]);
   if (bias != nullptr) {
     const uint4* bp = reinterpret_cast<const uint4*>(bias + gcol);
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const uint4 bb = __ldg(bp + q);
-      const uint32_t* w = reinterpret_cast<const uint32_t*>(&bb);
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        float& a = v[q * 8 + 2 * e];
-        float& b = v[q * 8 + 2 * e + 1];
-        f2_unpack(f2_add(f2_pack(a, b), f2_pack(bf16_lo(w[e]), bf16_hi(w[e]))), a, b);
-      }
-    }
+    for (int q = 0; q < 4; ++q) add_bf16x8(v + 8 * q, __ldg(bp + q));
   }
   if constexpr (EPI == DORA_EPI_BIAS_GELU) {
 #pragma unroll
     for (int e = 0; e < 32; e += 2) gelu_erf2(v[e], v[e + 1]);
   }
-  if constexpr (EPI == DORA_EPI_BIAS_RESIDUAL) {
-    if (row_ok) {
-      const uint4* rp = reinterpret_cast<const uint4*>(R + static_cast<size_t>(row) * N + gcol);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint4 rr = __ldg(rp + q);
-        const uint32_t* w = reinterpret_cast<const uint32_t*>(&rr);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          float& a = v[q * 8 + 2 * e];
-          float& b = v[q * 8 + 2 * e + 1];
-          f2_unpack(f2_add(f2_pack(a, b), f2_pack(bf16_lo(w[e]), bf16_hi(w[e]))), a, b);
-        }
-      }
-    }
-  }
+}
+
+__device__ __forceinline__ void pack_row(const float (&v)[32], uint32_t (&o)[16]) {
 #pragma unroll
   for (int e = 0; e < 16; ++e) o[e] = pack_bf16x2(v[2 * e], v[2 * e + 1]);
 }
@@ -287,6 +272,28 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
       const bool whole = row0 + 32 <= M;          // all 32 rows live: TMA store
 #pragma unroll 1
       for (int cb = 0; cb < kChunks; cb += kBatch) {
+        // Residual of whole 32-row chunks: loaded by the warp together, 8 rows
+        // x 64 contiguous bytes per instruction (piece p = lane + 32 i is
+        // row p / 4, 16-byte piece p % 4), before the TMEM load so its
+        // latency overlaps; it is transposed to rows through shared memory.
+        uint4 res[kBatch][4];
+        if constexpr (EPI == DORA_EPI_BIAS_RESIDUAL) {
+          if (whole) {
+#pragma unroll
+            for (int c = 0; c < kBatch; ++c) {
+              const int gcol = nt * BN + slot * kCols + (cb + c) * 32;
+              if (gcol < N) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                  const int pc = lane + 32 * i;
+                  res[c][i] = __ldg(reinterpret_cast<const uint4*>(
+                                        R + static_cast<size_t>(row0 + (pc >> 2)) * N + gcol) +
+                                    (pc & 3));
+                }
+              }
+            }
+          }
+        }
         uint32_t r[kBatch][32];
 #pragma unroll
         for (int c = 0; c < kBatch; ++c)
@@ -304,19 +311,35 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
         for (int c = 0; c < kBatch; ++c) {
           const int gcol = nt * BN + slot * kCols + (cb + c) * 32;
           if (gcol >= N || row0 >= M) continue;    // warp-uniform
+          float v[32];
           uint32_t o[16];
-          epilogue_math<EPI>(r[c], o, bias, R, row, gcol, N, row < M);
+          epilogue_math<EPI>(r[c], v, bias, gcol);
           if (whole) {
             // row `lane` of the 32x32 chunk, 64-byte swizzle: 16-byte piece j
-            // of row l sits at piece j ^ ((l >> 1) & 3).  The store issued two
-            // chunks ago from this buffer must have read it.
+            // of row l sits at piece j ^ ((l >> 1) & 3).  The store issued
+            // kBufs chunks ago from this buffer must have read it.
             uint16_t* stage = s.out[warp - 2][buf];
+            uint8_t* base = reinterpret_cast<uint8_t*>(stage);
             if (lane == 0) {
               if constexpr (kBufs == 2) bulk_wait_group_read1();
               else bulk_wait_group_read0();
             }
             __syncwarp();
-            uint8_t* rowp = reinterpret_cast<uint8_t*>(stage) + lane * 64;
+            uint8_t* rowp = base + lane * 64;
+            if constexpr (EPI == DORA_EPI_BIAS_RESIDUAL) {
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const int pc = lane + 32 * i, rr = pc >> 2, j = pc & 3;
+                *reinterpret_cast<uint4*>(base + rr * 64 + ((j ^ ((rr >> 1) & 3)) << 4)) =
+                    res[c][i];
+              }
+              __syncwarp();
+#pragma unroll
+              for (int j = 0; j < 4; ++j)
+                add_bf16x8(v + 8 * j,
+                           *reinterpret_cast<const uint4*>(rowp + ((j ^ ((lane >> 1) & 3)) << 4)));
+            }
+            pack_row(v, o);
 #pragma unroll
             for (int j = 0; j < 4; ++j)
               *reinterpret_cast<uint4*>(rowp + ((j ^ ((lane >> 1) & 3)) << 4)) =
@@ -329,6 +352,12 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
             }
             buf = (buf + 1) % kBufs;
           } else if (row < M) {
+            if constexpr (EPI == DORA_EPI_BIAS_RESIDUAL) {
+              const uint4* rp = reinterpret_cast<const uint4*>(R + static_cast<size_t>(row) * N + gcol);
+#pragma unroll
+              for (int j = 0; j < 4; ++j) add_bf16x8(v + 8 * j, __ldg(rp + j));
+            }
+            pack_row(v, o);
             uint4* yp = reinterpret_cast<uint4*>(Y + static_cast<size_t>(row) * N + gcol);
 #pragma unroll
             for (int j = 0; j < 4; ++j)
