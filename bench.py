@@ -39,7 +39,10 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM traffic per GEMM launch from an ncu capture (dram__bytes_read.sum +
 # dram__bytes_write.sum), keyed by the sha256 of the kernel source it was
 # taken on; reported as null once the source changes.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    # profiles/gemm_tcgen05_deit_base_b256.md: 48 launches of one forward step
+    "3a170aa1d8db06deca78668d674cb29a90e837efaf9a5eba44d09e7729885705": 187774272,
+}
 
 
 def parse_args():
