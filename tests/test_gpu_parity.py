@@ -342,6 +342,28 @@ def test_attention_edge_lengths_and_nan_tail():
     _check_attn(np.array([197, 5, 130]), 12, 9, tail_nan=70)
 
 
+def test_attention_running_maximum_moves_between_key_chunks():
+    """Keys of later 128-key chunks scaled up (image 0: x4 then x8; image 2:
+    x6) so that the row maximum of a later chunk lies far above the first
+    chunk's and the online softmax has to move its reference; image 1 is the
+    reverse (first chunk dominant, later probabilities underflow)."""
+    lens = np.array([300, 200, 140])
+    heads = 2
+    rng = np.random.default_rng(13)
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    x = rng.standard_normal((t, 3 * heads * 64))
+    kcols = slice(heads * 64, 2 * heads * 64)
+    x[cu[0] + 128:cu[0] + 256, kcols] *= 4.0
+    x[cu[0] + 256:cu[1], kcols] *= 8.0
+    x[cu[1]:cu[1] + 128, kcols] *= 6.0
+    x[cu[2] + 128:cu[3], kcols] *= 6.0
+    qkv = S.f32_to_bf16_bits(x)
+    out, st = _run_attn(qkv, cu, heads, int(max(lens)))
+    assert st == 0
+    assert_close(f64(out), O.varlen_attention(qkv, cu, heads), "attn rescale")
+
+
 def test_attention_empty_images_and_long_image_flag():
     lens = np.array([0, 20, 0, 33])
     _check_attn(lens, 2, 10)
