@@ -5,31 +5,30 @@
 //
 // Work unit = (image, head, 128-row query tile); a unit walks its keys in
 // chunks of 128 ("steps").  One persistent CTA per SM owns a contiguous range
-// of image-heads, split by estimated cost.  The CTA's units alternate between
-// two warpgroups; each has its own MMA issuer, so the two run independently
-// and one's exponentials overlap the other's tensor-core work:
-//   warp 0       walks the CTA's steps two at a time (one per warpgroup), loads
-//                Q and K/V chunks by TMA (a chunk both warpgroups need in the
-//                same round is loaded once) and publishes a step descriptor per
-//                warpgroup and a unit descriptor for the epilogue.  No other
+// of image-heads, split by estimated cost, and runs its steps through a
+// pipeline in which no role waits on the softmax's own previous work:
+//   warp 0       walks the CTA's units, loads Q and K/V chunks by TMA (the two
+//                query tiles of an image of up to 256 tokens share the chunks),
+//                and publishes a descriptor per step and per unit.  No other
 //                role keeps unit bookkeeping.
-//   warps 1, 14  MMA issuers of warpgroups 0 and 1 (one thread each):
-//                S = Q K^T (M=128, N=keys rounded to 16, K=64) into the
-//                warpgroup's S columns, then O (+)= P V with P read from TMEM.
-//                A step's S is issued as soon as the previous S has been read,
-//                ahead of the previous step's PV.
-//   warps 2-9    softmax warpgroups, one thread per query row (TMEM lane):
-//                row maximum, 2^x, row sum; P (bf16) to its own TMEM columns.
-//                Within a unit the reference maximum is only raised when a
-//                later chunk exceeds it by more than 2^8, and then O is rescaled
-//                in TMEM; otherwise P stays below 2^8 in the old frame, which
-//                bf16 and fp32 hold exactly as well.  They also zero the V rows
-//                of a chunk's last 16-key group that lie past the image.
-//   warps 10-13  epilogue: once a unit's last PV is done, O is read from TMEM,
-//                divided by the row sum and stored; the O columns are handed
-//                back for the warpgroup's next unit.
-// TMEM (512 columns): warpgroup w owns [256w, 256w+256): S 0-127, P 128-191,
-// O 192-255.  Rows past the image are computed but never stored; keys past it
+//   warps 1, 2   MMA issuers (one thread each): warp 1 issues S(j) = Q K^T
+//                (M=128, N=keys rounded to 16, K=64) into S/P buffer j mod 2,
+//                once PV(j-2) is done with that buffer; warp 2 issues O (+)= P(j) V
+//                with P read from the same buffer, into O buffer (unit mod 2).
+//                A single issuing thread could not keep up with 12 MMAs a step.
+//   warps 4-11   softmax, two threads per query row (TMEM lane), 64 of a step's
+//                128 S columns each, held in registers: the half maxima are
+//                exchanged, then 2^x, partial row sum, and P (bf16) written over
+//                the S columns just read.  Within a unit
+//                the reference maximum is only raised when a later chunk exceeds
+//                it by more than 2^8, and then O is rescaled in TMEM; otherwise
+//                P stays below 2^8 in the old frame, which bf16 and fp32 hold
+//                exactly as well.  The softmax also zeroes the V rows of a
+//                chunk's last 16-key group that lie past the image.
+//   warps 12-15  epilogue: when a unit's last PV is done, O / row sum, staged
+//                through shared memory and stored four whole rows per store.
+// TMEM (512 columns): S/P buffers 0-127 and 128-255, O buffers 256-319 and
+// 320-383.  Rows past the image are computed but never stored; keys past it
 // are masked, and V rows past it are zeroed so stale data cannot leak through
 // 0 * NaN.
 #include <cuda.h>
@@ -48,59 +47,61 @@ constexpr int BQ = 128;         // query rows per unit
 constexpr int KC = 128;         // keys per step
 constexpr int HD = 64;
 constexpr int kStages = 4;      // K/V chunk ring
-constexpr int kDescRing = 8;    // step descriptors in flight per warpgroup
-constexpr int kUnitRing = 4;    // unit descriptors in flight per warpgroup
-constexpr int kThreads = 480;   // 15 warps
-constexpr int kIssuer0 = 1, kIssuer1 = 14;   // MMA issuer warps of warpgroups 0 and 1
+constexpr int kDescRing = 8;    // step descriptors in flight
+constexpr int kUnitRing = 4;    // unit descriptors in flight
+constexpr int kThreads = 512;   // 16 warps (3 idle): 128 registers a thread
+constexpr int kSoftWarp0 = 4;   // softmax warps 4-11: two per TMEM lane quarter
+constexpr int kEpiWarp0 = 12;   // epilogue warps 12-15
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleLog2 = 8.f;    // raise the reference maximum past 2^8
 constexpr uint32_t kSleepNs = 200000;  // waiting threads sleep instead of spinning
-__device__ __forceinline__ uint32_t tmem_s(int w) { return 256u * static_cast<uint32_t>(w); }
-__device__ __forceinline__ uint32_t tmem_p(int w) { return 256u * static_cast<uint32_t>(w) + 128u; }
-__device__ __forceinline__ uint32_t tmem_o(int w) { return 256u * static_cast<uint32_t>(w) + 192u; }
+__device__ __forceinline__ uint32_t tmem_sp(int b) { return 128u * static_cast<uint32_t>(b); }
+__device__ __forceinline__ uint32_t tmem_o(int b) { return 256u + 64u * static_cast<uint32_t>(b); }
 
 // Step descriptor (one 32-bit word).
 constexpr uint32_t kDStage = 0x3u;        // K/V stage
 constexpr uint32_t kDKvPar = 1u << 2;     // phase parity of that stage's load
 constexpr uint32_t kDFirst = 1u << 3;     // first key chunk of a unit
 constexpr uint32_t kDLast = 1u << 4;      // last key chunk of a unit
-constexpr uint32_t kDQbuf = 1u << 5;      // Q buffer of the unit
-constexpr uint32_t kDQPar = 1u << 6;      // phase parity of that Q load
-constexpr uint32_t kDPrevUnit = 1u << 7;  // the warpgroup had an earlier unit
-constexpr uint32_t kDSolo = 1u << 8;      // the only step reading this K/V load
-constexpr uint32_t kDEnd = 1u << 31;      // no more steps for this warpgroup
+constexpr uint32_t kDUPar = 1u << 5;      // unit parity: Q buffer and O buffer
+constexpr uint32_t kDQPar = 1u << 6;      // phase parity of the unit's Q load
+constexpr uint32_t kDRelease = 1u << 7;   // the K/V stage is free after this step's PV
+constexpr uint32_t kDOWait = 1u << 8;     // the O buffer held an earlier unit
+constexpr uint32_t kDOPar = 1u << 25;     // phase parity of that unit's O read-out
+constexpr uint32_t kDEnd = 1u << 31;      // no more steps
 __device__ __forceinline__ int d_kc(uint32_t d) { return static_cast<int>((d >> 9) & 0xFFu); }
 __device__ __forceinline__ int d_rows(uint32_t d) { return static_cast<int>((d >> 17) & 0xFFu); }
-constexpr uint32_t kUEnd = 0xFFFFFFFFu;   // unit descriptor: no more units
 
 struct Smem {
-  uint16_t q[2][2][BQ * HD];    // [warpgroup][buffer], 4 x 16 KB
+  uint16_t q[2][BQ * HD];       // 2 x 16 KB, by unit parity
   uint16_t k[kStages][KC * HD]; // 4 x 16 KB
   uint16_t v[kStages][KC * HD]; // 4 x 16 KB
-  float lsum[2][2][BQ];         // row sums [warpgroup][unit parity]
-  uint64_t q_full[2][2];
-  uint64_t q_empty[2][2];
+  uint4 ostage[4][32 * 8];      // per epilogue warp: 32 output rows of 128 bytes
+  float lsum[4][2][BQ];         // row sums of each column half, by unit mod 4
+  float mx[2][2][BQ];           // row maxima of each column half, by step parity
+  uint64_t q_full[2];
+  uint64_t q_empty[2];
   uint64_t kv_full[kStages];
-  uint64_t kv_empty[kStages];   // two arrivals: both readers' PVs (a solo reader arrives twice)
-  uint64_t s_full[2];           // S of warpgroup w computed
-  uint64_t s_free[2];           // ... and read (one arrival per warp)
-  uint64_t p_full[2];           // P written, O rescaled, V tail zeroed (one arrival per warp)
-  uint64_t p_free[2];           // PV done: P buffer free, O current
-  uint64_t o_done[2];           // last PV of a unit done
-  uint64_t o_free[2];           // O read by the epilogue (one arrival per warp)
-  uint64_t l_full[2][2];        // row sums of a unit written (one arrival per warp)
-  uint64_t sd_full[2][kDescRing];   // step descriptor published
-  uint64_t sd_empty[2][kDescRing];  // ... read by the issuer and the four softmax warps
-  uint64_t ud_full[2][kUnitRing];   // unit descriptor published
-  uint64_t ud_empty[2][kUnitRing];  // ... read by the four epilogue warps
+  uint64_t kv_empty[kStages];
+  uint64_t s_full[2];           // S of a step in S/P buffer b
+  uint64_t p_full[2];           // P written over it (one arrival per softmax warp)
+  uint64_t xbar[2][4];          // the two halves of a lane quarter exchanged their maxima
+  uint64_t p_free[2];           // PV of buffer b done
+  uint64_t o_done[2];           // last PV of a unit in O buffer b done
+  uint64_t o_free[2];           // O buffer b read out (one arrival per epilogue warp)
+  uint64_t l_full[4];           // row sums of a unit (one arrival per softmax warp)
+  uint64_t sd_full[kDescRing];  // step descriptor published
+  uint64_t sd_empty[kDescRing]; // ... read by both issuers and the eight softmax warps
+  uint64_t ud_full[kUnitRing];  // unit descriptor published
+  uint64_t ud_empty[kUnitRing]; // ... read by the four epilogue warps
   uint64_t drain[2];
-  uint32_t sdesc[2][kDescRing];
-  uint32_t urow[2][kUnitRing];      // first output row of the unit
-  uint32_t uhead[2][kUnitRing];     // head | rows << 16, or kUEnd
+  uint32_t sdesc[kDescRing];
+  uint32_t urow[kUnitRing];     // first output row of the unit
+  uint32_t uhead[kUnitRing];    // head | rows << 16
   uint32_t tmem_base;
   int abort_flag;
   int ih_begin, ih_end;
-  int q_issued[2], kv_issued;
+  int q_issued, kv_issued;
 };
 
 // Rows of image `img`, clamped to the buffer (0 when its start lies outside).
@@ -161,40 +162,6 @@ struct Walker {
       settle();
     }
   }
-};
-
-// The steps (unit, key chunk) of one softmax warpgroup: the CTA's units of
-// parity `wg`, each walked chunk by chunk.
-struct Steps {
-  Walker u;
-  int c, nch, ju;
-  bool has;
-  __device__ __forceinline__ void refresh() {
-    has = !u.done();
-    nch = has ? (u.n + KC - 1) / KC : 0;
-  }
-  __device__ __forceinline__ void start(const int32_t* cu, int heads, int t_cap, int b, int e,
-                                        int wg) {
-    u.start(cu, heads, t_cap, b, e);
-    if (wg) u.next();
-    c = 0;
-    ju = 0;
-    refresh();
-  }
-  __device__ __forceinline__ void next_unit() {
-    c = 0;
-    ++ju;
-    u.next();
-    u.next();
-    refresh();
-  }
-  __device__ __forceinline__ void advance() {
-    if (++c < nch) return;
-    next_unit();
-  }
-  __device__ __forceinline__ int kc() const { return min(KC, u.n - c * KC); }
-  __device__ __forceinline__ int q_rows() const { return min(BQ, u.n - u.qt * BQ); }
-  __device__ __forceinline__ bool last() const { return c == nch - 1; }
 };
 
 // Whole warp: the CTA's image-head range.  Image-head ih belongs to CTA
@@ -296,24 +263,25 @@ __device__ __forceinline__ float max32(const uint32_t (&a)[32], float m) {
   return max3f(m0, m1, fmaxf(m2, m3));
 }
 
-// p = 2^(s * scale_log2 - m) for 32 keys: packed to bf16, summed into l.
-__device__ __forceinline__ void exp32(const uint32_t (&a)[32], float scale_log2, float neg_m,
-                                      uint32_t (&pk)[16], float& l) {
-  float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
+// p = 2^(s * scale_log2 - m) for 32 keys, summed into l and packed to bf16 in
+// place: pair (2k, 2k+1) lands in a[k], whose S value is already consumed.
+__device__ __forceinline__ void exp32_pack(uint32_t (&a)[32], float scale_log2, float neg_m,
+                                           float& l) {
+  float l0 = 0.f, l1 = 0.f;
 #pragma unroll
-  for (int e = 0; e < 32; e += 4) {
+  for (int e = 0; e < 32; e += 2) {
     const float p0 = ex2_approx(fmaf(__uint_as_float(a[e]), scale_log2, neg_m));
     const float p1 = ex2_approx(fmaf(__uint_as_float(a[e + 1]), scale_log2, neg_m));
-    const float p2 = ex2_approx(fmaf(__uint_as_float(a[e + 2]), scale_log2, neg_m));
-    const float p3 = ex2_approx(fmaf(__uint_as_float(a[e + 3]), scale_log2, neg_m));
     l0 += p0;
     l1 += p1;
-    l2 += p2;
-    l3 += p3;
-    pk[e >> 1] = pack_bf16x2(p0, p1);
-    pk[(e >> 1) + 1] = pack_bf16x2(p2, p3);
+    a[e >> 1] = pack_bf16x2(p0, p1);
   }
-  l += (l0 + l1) + (l2 + l3);
+  l += l0 + l1;
+}
+
+// The packed half of a block, as the 16-column store operand.
+__device__ __forceinline__ const uint32_t (&lo16(const uint32_t (&a)[32]))[16] {
+  return *reinterpret_cast<const uint32_t(*)[16]>(&a[0]);
 }
 
 // One arrival for the whole warp, after every lane's prior tcgen05 accesses.
@@ -345,34 +313,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       s.ih_end = static_cast<int>(e);
     }
   } else if (threadIdx.x == 64) {
-    for (int w = 0; w < 2; ++w) {
-      for (int b = 0; b < 2; ++b) {
-        mbar_init(&s.q_full[w][b], 1);
-        mbar_init(&s.q_empty[w][b], 1);
-        mbar_init(&s.l_full[w][b], 4);
-      }
-      mbar_init(&s.s_full[w], 1);
-      mbar_init(&s.s_free[w], 4);
-      mbar_init(&s.p_full[w], 4);
-      mbar_init(&s.p_free[w], 1);
-      mbar_init(&s.o_done[w], 1);
-      mbar_init(&s.o_free[w], 4);
-      for (int i = 0; i < kDescRing; ++i) {
-        mbar_init(&s.sd_full[w][i], 1);
-        mbar_init(&s.sd_empty[w][i], 5);
-      }
-      for (int i = 0; i < kUnitRing; ++i) {
-        mbar_init(&s.ud_full[w][i], 1);
-        mbar_init(&s.ud_empty[w][i], 4);
-      }
-      mbar_init(&s.drain[w], 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&s.q_full[b], 1);
+      mbar_init(&s.q_empty[b], 1);
+      mbar_init(&s.s_full[b], 1);
+      mbar_init(&s.p_full[b], 8);
+      for (int q = 0; q < 4; ++q) mbar_init(&s.xbar[b][q], 2);
+      mbar_init(&s.p_free[b], 1);
+      mbar_init(&s.o_done[b], 1);
+      mbar_init(&s.o_free[b], 4);
     }
+    for (int i = 0; i < 4; ++i) mbar_init(&s.l_full[i], 8);
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&s.kv_full[i], 1);
-      mbar_init(&s.kv_empty[i], 2);
+      mbar_init(&s.kv_empty[i], 1);
     }
+    for (int i = 0; i < kDescRing; ++i) {
+      mbar_init(&s.sd_full[i], 1);
+      mbar_init(&s.sd_empty[i], 10);
+    }
+    for (int i = 0; i < kUnitRing; ++i) {
+      mbar_init(&s.ud_full[i], 1);
+      mbar_init(&s.ud_empty[i], 4);
+    }
+    mbar_init(&s.drain[0], 1);
+    mbar_init(&s.drain[1], 1);
     s.abort_flag = 0;
-    s.q_issued[0] = s.q_issued[1] = s.kv_issued = 0;
+    s.q_issued = s.kv_issued = 0;
     fence_barrier_init();
     tma_prefetch_desc(&tm);
   }
@@ -387,362 +354,302 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ---------------- scheduler + TMA producer ----------------
     if (lane == 0) {
-      Steps st[2];
-      st[0].start(cu, heads, t_cap, ih_b, ih_e, 0);
-      st[1].start(cu, heads, t_cap, ih_b, ih_e, 1);
-      int loads = 0, qn[2] = {0, 0}, dn[2] = {0, 0}, un[2] = {0, 0};
-      bool ended[2] = {false, false};
+      Walker wk;
+      wk.start(cu, heads, t_cap, ih_b, ih_e);
+      int u = 0, loads = 0, dn = 0;
+      int prev_stage[2] = {0, 0}, prev_par[2] = {0, 0};
+      bool reuse_this = false;      // this unit reads the previous unit's K/V chunks
       bool ok = true;
-      auto desc = [&](int w, uint32_t d) -> bool {
-        const int i = dn[w] % kDescRing;
-        if (!mbar_wait_sleep(&s.sd_empty[w][i], ((dn[w] / kDescRing) & 1) ^ 1, abort, kSleepNs))
+      auto desc = [&](uint32_t d) -> bool {
+        const int i = dn % kDescRing;
+        if (!mbar_wait_sleep(&s.sd_empty[i], ((dn / kDescRing) & 1) ^ 1, abort, kSleepNs))
           return false;
-        s.sdesc[w][i] = d;
-        mbar_arrive(&s.sd_full[w][i]);
-        ++dn[w];
+        s.sdesc[i] = d;
+        mbar_arrive(&s.sd_full[i]);
+        ++dn;
         return true;
       };
-      auto unit = [&](int w, uint32_t row, uint32_t hd) -> bool {
-        const int i = un[w] % kUnitRing;
-        if (!mbar_wait_sleep(&s.ud_empty[w][i], ((un[w] / kUnitRing) & 1) ^ 1, abort, kSleepNs))
-          return false;
-        s.urow[w][i] = row;
-        s.uhead[w][i] = hd;
-        mbar_arrive(&s.ud_full[w][i]);
-        ++un[w];
-        return true;
-      };
-      while (ok && !(ended[0] && ended[1])) {
-        // this round: the next step of each warpgroup; one load when they share a chunk
-        const bool shared = !ended[0] && !ended[1] && st[0].has && st[1].has &&
-                            st[0].u.ih == st[1].u.ih && st[0].c == st[1].c;
-        int load0 = 0;
-        for (int w = 0; w < 2 && ok; ++w) {
-          if (ended[w]) continue;
-          Steps& x = st[w];
-          if (!x.has) {
-            ok = desc(w, kDEnd) && unit(w, 0u, kUEnd);
-            ended[w] = true;
-            continue;
-          }
-          const int rows = x.q_rows();
-          if (x.c == 0) {
-            if (!unit(w, static_cast<uint32_t>(x.u.lo + x.u.qt * BQ),
-                      static_cast<uint32_t>(x.u.head) | (static_cast<uint32_t>(rows) << 16))) {
-              ok = false;
-              break;
-            }
-            const int qb = qn[w] & 1;
-            if (!mbar_wait_sleep(&s.q_empty[w][qb], ((qn[w] >> 1) & 1) ^ 1, abort, kSleepNs)) {
-              ok = false;
-              break;
-            }
-            mbar_arrive_expect_tx(&s.q_full[w][qb], BQ * HD * 2);
-            tma_load_2d(s.q[w][qb], &tm, &s.q_full[w][qb], x.u.head * HD, x.u.lo + x.u.qt * BQ);
-            ++qn[w];
-          }
-          int ld = load0;
-          if (!(w == 1 && shared)) {
-            ld = loads;
-            const int stg = ld % kStages;
-            if (!mbar_wait_sleep(&s.kv_empty[stg], ((ld / kStages) & 1) ^ 1, abort, kSleepNs)) {
+      while (ok && !wk.done()) {
+        const int n = wk.n, nch = (n + KC - 1) / KC;
+        const int rows = min(BQ, n - wk.qt * BQ);
+        Walker nx = wk;
+        nx.next();
+        // the next unit (the image-head's other query tile) reads the same chunks
+        const bool reuse_next = !nx.done() && nx.ih == wk.ih && nch <= 2;
+        {
+          const int i = u % kUnitRing;
+          if (!mbar_wait_sleep(&s.ud_empty[i], ((u / kUnitRing) & 1) ^ 1, abort, kSleepNs)) break;
+          s.urow[i] = static_cast<uint32_t>(wk.lo + wk.qt * BQ);
+          s.uhead[i] = static_cast<uint32_t>(wk.head) | (static_cast<uint32_t>(rows) << 16);
+          mbar_arrive(&s.ud_full[i]);
+        }
+        const int qb = u & 1;
+        if (!mbar_wait_sleep(&s.q_empty[qb], ((u >> 1) & 1) ^ 1, abort, kSleepNs)) break;
+        mbar_arrive_expect_tx(&s.q_full[qb], BQ * HD * 2);
+        tma_load_2d(s.q[qb], &tm, &s.q_full[qb], wk.head * HD, wk.lo + wk.qt * BQ);
+        s.q_issued = u + 1;
+        int cur_stage[2] = {0, 0}, cur_par[2] = {0, 0};
+        for (int c = 0; ok && c < nch; ++c) {
+          int stg, par;
+          if (reuse_this) {
+            stg = prev_stage[c];
+            par = prev_par[c];
+          } else {
+            stg = loads % kStages;
+            par = (loads / kStages) & 1;
+            if (!mbar_wait_sleep(&s.kv_empty[stg], par ^ 1, abort, kSleepNs)) {
               ok = false;
               break;
             }
             mbar_arrive_expect_tx(&s.kv_full[stg], 2 * KC * HD * 2);
-            const int row = x.u.lo + x.c * KC;
-            tma_load_2d(s.k[stg], &tm, &s.kv_full[stg], dim + x.u.head * HD, row);
-            tma_load_2d(s.v[stg], &tm, &s.kv_full[stg], 2 * dim + x.u.head * HD, row);
+            const int row = wk.lo + c * KC;
+            tma_load_2d(s.k[stg], &tm, &s.kv_full[stg], dim + wk.head * HD, row);
+            tma_load_2d(s.v[stg], &tm, &s.kv_full[stg], 2 * dim + wk.head * HD, row);
             ++loads;
-            load0 = ld;
+            s.kv_issued = loads;
           }
-          const int qi = qn[w] - 1;                       // this unit's Q load
+          if (c < 2) {
+            cur_stage[c] = stg;
+            cur_par[c] = par;
+          }
           const uint32_t d =
-              static_cast<uint32_t>(ld % kStages) | (((ld / kStages) & 1) ? kDKvPar : 0u) |
-              (x.c == 0 ? kDFirst : 0u) | (x.last() ? kDLast : 0u) | ((qi & 1) ? kDQbuf : 0u) |
-              (((qi >> 1) & 1) ? kDQPar : 0u) | (x.ju > 0 ? kDPrevUnit : 0u) |
-              (shared ? 0u : kDSolo) | (static_cast<uint32_t>(x.kc()) << 9) |
+              static_cast<uint32_t>(stg) | (par ? kDKvPar : 0u) | (c == 0 ? kDFirst : 0u) |
+              (c == nch - 1 ? kDLast : 0u) | ((u & 1) ? kDUPar : 0u) |
+              (((u >> 1) & 1) ? kDQPar : 0u) | (reuse_next ? 0u : kDRelease) |
+              (u >= 2 ? kDOWait : 0u) | ((((u >> 1) - 1) & 1) ? kDOPar : 0u) |
+              (static_cast<uint32_t>(min(KC, n - c * KC)) << 9) |
               (static_cast<uint32_t>(rows) << 17);
-          if (!desc(w, d)) {
-            ok = false;
-            break;
-          }
-          x.advance();
+          ok = desc(d);
+        }
+        prev_stage[0] = cur_stage[0];
+        prev_stage[1] = cur_stage[1];
+        prev_par[0] = cur_par[0];
+        prev_par[1] = cur_par[1];
+        reuse_this = reuse_next;
+        ++u;
+        wk = nx;
+      }
+      if (ok && desc(kDEnd)) {
+        const int i = u % kUnitRing;      // no more units
+        if (mbar_wait_sleep(&s.ud_empty[i], ((u / kUnitRing) & 1) ^ 1, abort, kSleepNs)) {
+          s.uhead[i] = 0xFFFFFFFFu;
+          mbar_arrive(&s.ud_full[i]);
         }
       }
-      s.q_issued[0] = qn[0];
-      s.q_issued[1] = qn[1];
-      s.kv_issued = loads;
     }
-  } else if (warp == kIssuer0 || warp == kIssuer1) {
-    // ---------------- MMA issuer of warpgroup w (lane 0) ----------------
-    const int w = warp == kIssuer0 ? 0 : 1;
+  } else if (warp == 1 || warp == 2) {
+    // ---------------- MMA issuers: warp 1 issues S, warp 2 issues PV (lane 0) ----------------
+    // Each reads every step descriptor.  The only order between the two is
+    // explicit: S(j+2) waits until PV(j) has read S/P buffer j mod 2.
     if (lane == 0) {
-      constexpr uint32_t id_o = idesc_bf16(BQ, HD, true);
-      const uint32_t ts = tmem + tmem_s(w), tp = tmem + tmem_p(w), to = tmem + tmem_o(w);
-      int j = 0, ju = 0;
-      bool ok = true;
-      auto next_desc = [&](uint32_t& d) -> bool {
+      for (int j = 0;; ++j) {
         const int i = j % kDescRing;
-        if (!mbar_wait_sleep(&s.sd_full[w][i], (j / kDescRing) & 1, abort, kSleepNs)) return false;
-        d = s.sdesc[w][i];
-        mbar_arrive(&s.sd_empty[w][i]);
-        return true;
-      };
-      // S = Q K^T of step j
-      auto issue_s = [&](uint32_t d) -> bool {
+        if (!mbar_wait_sleep(&s.sd_full[i], (j / kDescRing) & 1, abort, kSleepNs)) break;
+        const uint32_t d = s.sdesc[i];
+        mbar_arrive(&s.sd_empty[i]);
+        if (d & kDEnd) break;
         const int stg = static_cast<int>(d & kDStage);
-        const uint32_t qb = (d & kDQbuf) ? 1u : 0u;
-        if ((d & kDFirst) &&
-            !mbar_wait_sleep(&s.q_full[w][qb], (d & kDQPar) ? 1u : 0u, abort, kSleepNs))
-          return false;
-        if (!mbar_wait_sleep(&s.kv_full[stg], (d & kDKvPar) ? 1u : 0u, abort, kSleepNs))
-          return false;
-        if (j > 0 && !mbar_wait_sleep(&s.s_free[w], (j - 1) & 1, abort, kSleepNs)) return false;
-        tc_fence_after();
-        const uint64_t qd = sdesc_sw128(smem_u32(s.q[w][qb]), 16, 1024);
-        const uint64_t kd = sdesc_sw128(smem_u32(s.k[stg]), 16, 1024);
-        const uint32_t id_s = idesc_bf16(BQ, (d_kc(d) + 15) & ~15, false);
-        mma_bf16_ss(ts, qd, kd, id_s, 0u);
-        mma_bf16_ss(ts, qd + 2, kd + 2, id_s, 1u);
-        mma_bf16_ss(ts, qd + 4, kd + 4, id_s, 1u);
-        mma_bf16_ss(ts, qd + 6, kd + 6, id_s, 1u);
-        mma_commit(&s.s_full[w]);
-        if (d & kDLast) mma_commit(&s.q_empty[w][qb]);
-        ++j;
-        return true;
-      };
-      // O (+)= P V of step jp
-      auto issue_pv = [&](uint32_t d, int jp) -> bool {
-        const bool first = (d & kDFirst) != 0;
-        if (first && (d & kDPrevUnit) &&
-            !mbar_wait_sleep(&s.o_free[w], (ju - 1) & 1, abort, kSleepNs))
-          return false;
-        if (!mbar_wait_sleep(&s.p_full[w], jp & 1, abort, kSleepNs)) return false;
-        tc_fence_after();
-        const int nk = (d_kc(d) + 15) >> 4;
-        const uint64_t vd = sdesc_sw128(smem_u32(s.v[d & kDStage]), 1024, 1024);
-        mma_bf16_ts(to, tp, vd, id_o, first ? 0u : 1u);
+        const int up = (d & kDUPar) ? 1 : 0;
+        const int b = j & 1;
+        if (warp == 1) {
+          // S(j) = Q K^T into S/P buffer b
+          if ((d & kDFirst) &&
+              !mbar_wait_sleep(&s.q_full[up], (d & kDQPar) ? 1u : 0u, abort, kSleepNs))
+            break;
+          if (!mbar_wait_sleep(&s.kv_full[stg], (d & kDKvPar) ? 1u : 0u, abort, kSleepNs)) break;
+          // the buffer's previous P has been read by its PV (step j - 2)
+          if (j >= 2 && !mbar_wait_sleep(&s.p_free[b], ((j - 2) >> 1) & 1, abort, kSleepNs))
+            break;
+          tc_fence_after();
+          const uint64_t qd = sdesc_sw128(smem_u32(s.q[up]), 16, 1024);
+          const uint64_t kd = sdesc_sw128(smem_u32(s.k[stg]), 16, 1024);
+          const uint32_t id_s = idesc_bf16(BQ, (d_kc(d) + 15) & ~15, false);
+          const uint32_t dt = tmem + tmem_sp(b);
+          mma_bf16_ss(dt, qd, kd, id_s, 0u);
+          mma_bf16_ss(dt, qd + 2, kd + 2, id_s, 1u);
+          mma_bf16_ss(dt, qd + 4, kd + 4, id_s, 1u);
+          mma_bf16_ss(dt, qd + 6, kd + 6, id_s, 1u);
+          mma_commit(&s.s_full[b]);
+          if (d & kDLast) mma_commit(&s.q_empty[up]);
+        } else {
+          // O (+)= P(j) V into O buffer up
+          constexpr uint32_t id_o = idesc_bf16(BQ, HD, true);
+          const bool first = (d & kDFirst) != 0;
+          if (first && (d & kDOWait) &&
+              !mbar_wait_sleep(&s.o_free[up], (d & kDOPar) ? 1u : 0u, abort, kSleepNs))
+            break;
+          if (!mbar_wait_sleep(&s.p_full[b], (j >> 1) & 1, abort, kSleepNs)) break;
+          tc_fence_after();
+          const int nk = (d_kc(d) + 15) >> 4;
+          const uint64_t vd = sdesc_sw128(smem_u32(s.v[stg]), 1024, 1024);
+          const uint32_t dt = tmem + tmem_o(up), at = tmem + tmem_sp(b);
+          mma_bf16_ts(dt, at, vd, id_o, first ? 0u : 1u);
 #pragma unroll
-        for (int kk = 1; kk < KC / 16; ++kk)   // 16 keys: 2048 bytes of V, 8 P columns
-          if (kk < nk) mma_bf16_ts(to, tp + 8u * kk, vd + 128u * kk, id_o, 1u);
-        mma_commit(&s.p_free[w]);
-        if (d & kDLast) {
-          mma_commit(&s.o_done[w]);
-          ++ju;
-        }
-        mma_commit(&s.kv_empty[d & kDStage]);
-        if (d & kDSolo) mma_commit(&s.kv_empty[d & kDStage]);
-        return true;
-      };
-      uint32_t dcur;
-      ok = next_desc(dcur);
-      if (ok && !(dcur & kDEnd)) {
-        ok = issue_s(dcur);
-        while (ok) {
-          uint32_t dn;
-          if (!next_desc(dn)) break;
-          const bool end = (dn & kDEnd) != 0;
-          if (!end && !issue_s(dn)) break;
-          if (!issue_pv(dcur, j - (end ? 1 : 2))) break;
-          if (end) break;
-          dcur = dn;
+          for (int kk = 1; kk < KC / 16; ++kk)   // 16 keys: 2048 bytes of V, 8 P columns
+            if (kk < nk) mma_bf16_ts(dt, at + 8u * kk, vd + 128u * kk, id_o, 1u);
+          mma_commit(&s.p_free[b]);
+          if (d & kDLast) mma_commit(&s.o_done[up]);
+          if (d & kDRelease) mma_commit(&s.kv_empty[stg]);
         }
       }
-      mma_commit(&s.drain[w]);
-      mbar_wait_limited(&s.drain[w], 0, kWaitLimitNs);
+      mma_commit(&s.drain[warp - 1]);
+      mbar_wait_limited(&s.drain[warp - 1], 0, kWaitLimitNs);
     }
-  } else if (warp < 10) {
-    // ---------------- softmax: warpgroup w, one thread per query row ----------------
-    const int w = (warp - 2) >> 2;
+  } else if (warp >= kSoftWarp0 && warp < kSoftWarp0 + 8) {
+    // ---------------- softmax: two threads per query row, 64 columns each ----------------
     const int quarter = warp & 3;
+    const int half = (warp - kSoftWarp0) >> 2;
     const int r = quarter * 32 + lane;                   // query row of the tile (TMEM lane)
     const uint32_t lane_sel = static_cast<uint32_t>(quarter * 32) << 16;
-    const uint32_t ts = tmem + lane_sel + tmem_s(w);
-    const uint32_t tp = tmem + lane_sel + tmem_p(w);
-    const uint32_t to = tmem + lane_sel + tmem_o(w);
-    float m_ref = 0.f, l = 0.f;
-    int ju = 0;
+    float m_ref = 0.f, l = 0.f;                          // l: this half's partial row sum
+    int u = 0;                                           // units finished
     auto step = [&](int j, uint32_t d) -> bool {
       const int kc = d_kc(d), kc16 = (kc + 15) & ~15;
-      const int nb = (kc + 31) >> 5;
+      const int kh = min(max(kc - 64 * half, 0), 64);    // keys in this thread's half
       const bool live = quarter * 32 < d_rows(d);        // warp-uniform
-      if (!mbar_wait_warp_sleep(&s.s_full[w], j & 1, abort, kSleepNs)) return false;
+      const int b = j & 1;
+      const uint32_t tsp = tmem + lane_sel + tmem_sp(b);
+      if (!mbar_wait_warp_sleep(&s.s_full[b], (j >> 1) & 1, abort, kSleepNs)) return false;
       tc_fence_after();
       // S is done, so the K/V load landed: zero V rows [kc, kc16) (whole 128-byte rows)
       if (kc < kc16) {
-        const int t = r;                                  // 0..127 over the warpgroup
+        const int t = half * BQ + r;
         if (t < (kc16 - kc) * 8)
           reinterpret_cast<uint4*>(s.v[d & kDStage])[kc * 8 + t] = make_uint4(0u, 0u, 0u, 0u);
         fence_proxy_async_smem();
       }
-      bool p_ok = j == 0;                                // P buffer known to be free
+      // this half's 64 S columns into registers (both blocks, always: arrays
+      // filled only conditionally would stay live across iterations)
+      uint32_t s0[32], s1[32];
+      float mloc = -INFINITY;
       if (live) {
-        float mloc = -INFINITY;
-        for (int b = 0; b < nb; ++b) {
-          uint32_t a[32];
-          tmem_ld32(ts + static_cast<uint32_t>(32 * b), a);
-          tmem_ld_wait();
-          mask_tail(a, kc - 32 * b);
-          mloc = max32(a, mloc);
-        }
-        const float mc = mloc * scale_log2;
+        tmem_ld32(tsp + static_cast<uint32_t>(64 * half), s0);
+        tmem_ld32(tsp + static_cast<uint32_t>(64 * half + 32), s1);
+        tmem_ld_wait();
+        mask_tail(s0, kh);
+        mask_tail(s1, kh - 32);
+        mloc = max32(s1, max32(s0, -INFINITY));
+      }
+      // exchange the half maxima with the other thread of the row
+      s.mx[b][half][r] = mloc;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.xbar[b][quarter]);
+      if (!mbar_wait_warp_sleep(&s.xbar[b][quarter], (j >> 1) & 1, abort, kSleepNs)) return false;
+      const float mc = fmaxf(mloc, s.mx[b][half ^ 1][r]) * scale_log2;
+      if (live) {
+        // reference maximum: set on a unit's first chunk, raised past 2^8
+        bool rescale = false;
+        float alpha = 1.f;
         if (d & kDFirst) {
           m_ref = mc;
           l = 0.f;
         } else {
           const bool need = mc > m_ref + kRescaleLog2;
-          if (__any_sync(0xffffffffu, need)) {
-            // raise the reference: O (complete up to the previous chunk) and l
-            if (!mbar_wait_warp_sleep(&s.p_free[w], (j - 1) & 1, abort, kSleepNs)) return false;
-            p_ok = true;
-            tc_fence_after();
-            const float m_new = need ? mc : m_ref;
-            const float alpha = ex2_approx(m_ref - m_new);
-#pragma unroll 1
-            for (int h = 0; h < 2; ++h) {
-              uint32_t o[32], o2[16];
-              tmem_ld32(to + static_cast<uint32_t>(32 * h), o);
-              tmem_ld_wait();
-#pragma unroll
-              for (int e = 0; e < 16; ++e) o2[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-              tmem_st16(to + static_cast<uint32_t>(32 * h), o2);
-#pragma unroll
-              for (int e = 0; e < 16; ++e) o2[e] = __float_as_uint(__uint_as_float(o[e + 16]) * alpha);
-              tmem_st16(to + static_cast<uint32_t>(32 * h + 16), o2);
-            }
+          rescale = __any_sync(0xffffffffu, need) != 0;
+          if (need) {
+            alpha = ex2_approx(m_ref - mc);
             l *= alpha;
-            m_ref = m_new;
+            m_ref = mc;
           }
         }
-        if (!p_ok) {
-          if (!mbar_wait_warp_sleep(&s.p_free[w], (j - 1) & 1, abort, kSleepNs)) return false;
+        // P over this half's S columns (16 columns per 32 keys)
+        if (kh > 0) {
+          exp32_pack(s0, scale_log2, -m_ref, l);
+          tmem_st16(tsp + static_cast<uint32_t>(32 * half), lo16(s0));
+        }
+        if (kh > 32) {
+          exp32_pack(s1, scale_log2, -m_ref, l);
+          tmem_st16(tsp + static_cast<uint32_t>(32 * half + 16), lo16(s1));
+        }
+        if (rescale) {
+          // O holds the chunks before this one once their PV is done: bring this
+          // half's 32 columns to the raised reference before this chunk's PV
+          if (!mbar_wait_warp_sleep(&s.p_free[b ^ 1], ((j - 1) >> 1) & 1, abort, kSleepNs))
+            return false;
           tc_fence_after();
-        }
-        for (int b = 0; b < nb; ++b) {
-          uint32_t a[32], pk[16];
-          tmem_ld32(ts + static_cast<uint32_t>(32 * b), a);
+          const uint32_t to = tmem + lane_sel + tmem_o((d & kDUPar) ? 1 : 0) +
+                              static_cast<uint32_t>(32 * half);
+          uint32_t o[32];
+          tmem_ld32(to, o);
           tmem_ld_wait();
-          if (b == nb - 1) warp_arrive(&s.s_free[w]);
-          mask_tail(a, kc - 32 * b);
-          exp32(a, scale_log2, -m_ref, pk, l);
-          tmem_st16(tp + static_cast<uint32_t>(16 * b), pk);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          tmem_st16(to, lo16(o));
+          tmem_st16(to + 16u, *reinterpret_cast<const uint32_t(*)[16]>(&o[16]));
         }
-        tmem_st_wait();
-      } else {
-        warp_arrive(&s.s_free[w]);
-        // arrive on p_full only after the previous PV: keeps phases apart
-        if (!p_ok && !mbar_wait_warp_sleep(&s.p_free[w], (j - 1) & 1, abort, kSleepNs)) return false;
       }
+      tmem_st_wait();
       if (d & kDLast) {
-        s.lsum[w][ju & 1][r] = l;
-        warp_arrive(&s.l_full[w][ju & 1]);
-        ++ju;
+        s.lsum[u & 3][half][r] = l;
+        warp_arrive(&s.l_full[u & 3]);
+        ++u;
       }
-      warp_arrive(&s.p_full[w]);
+      warp_arrive(&s.p_full[b]);
       return true;
     };
     for (int j = 0;; ++j) {
       const int i = j % kDescRing;
-      if (!mbar_wait_warp_sleep(&s.sd_full[w][i], (j / kDescRing) & 1, abort, kSleepNs)) break;
-      const uint32_t d = s.sdesc[w][i];
+      if (!mbar_wait_warp_sleep(&s.sd_full[i], (j / kDescRing) & 1, abort, kSleepNs)) break;
+      const uint32_t d = s.sdesc[i];
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s.sd_empty[w][i]);
+      if (lane == 0) mbar_arrive(&s.sd_empty[i]);
       if ((d & kDEnd) || !step(j, d)) break;
     }
-  } else {
-    // ---------------- epilogue: normalise and store O ----------------
+  } else if (warp >= kEpiWarp0) {
+    // ---------------- epilogue: O / row sum, stored four rows per instruction ----------------
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;
     const uint32_t lane_sel = static_cast<uint32_t>(quarter * 32) << 16;
-    int ue[2] = {0, 0};
-    bool have[2] = {false, false}, done[2] = {false, false};
-    uint32_t urow[2] = {0u, 0u}, uhd[2] = {0u, 0u};
-    uint64_t t0 = 0;
-    uint32_t spins = 0;
-    bool ok = true;
-    // Units finish out of order between the warpgroups: serve whichever is done.
-    while (ok && !(done[0] && done[1])) {
-      bool did = false;
-      for (int w = 0; w < 2 && ok; ++w) {
-        if (done[w]) continue;
-        const uint32_t hint = done[w ^ 1] ? 4096u : 256u;
-        if (!have[w]) {
-          const int i = ue[w] % kUnitRing;
-          if (!__all_sync(0xffffffffu,
-                          mbar_try_wait_hint(&s.ud_full[w][i], (ue[w] / kUnitRing) & 1, hint)))
-            continue;
-          urow[w] = s.urow[w][i];
-          uhd[w] = s.uhead[w][i];
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s.ud_empty[w][i]);
-          did = true;
-          if (uhd[w] == kUEnd) {
-            done[w] = true;
-            continue;
-          }
-          have[w] = true;
-        }
-        if (!__all_sync(0xffffffffu, mbar_try_wait_hint(&s.o_done[w], ue[w] & 1, hint))) continue;
-        const int ub = ue[w] & 1;
-        if (!mbar_wait_warp_sleep(&s.l_full[w][ub], (ue[w] >> 1) & 1, abort, kSleepNs)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const int q_rows = static_cast<int>(uhd[w] >> 16);
-        const int head = static_cast<int>(uhd[w] & 0xFFFFu);
-        const bool live = quarter * 32 < q_rows;
-        uint32_t oa[32], ob[32];
-        float lr = 1.f;
-        if (live) {
-          const uint32_t to = tmem + lane_sel + tmem_o(w);
-          tmem_ld32(to, oa);
-          tmem_ld32(to + 32u, ob);
-          tmem_ld_wait();
-          lr = s.lsum[w][ub][r];
-        }
-        warp_arrive(&s.o_free[w]);
-        if (live && r < q_rows) {
-          const float inv = 1.0f / lr;
-          uint4* dst = reinterpret_cast<uint4*>(
-              out + static_cast<size_t>(urow[w] + r) * dim + head * HD);
-#pragma unroll
-          for (int qd = 0; qd < 4; ++qd)
-            dst[qd] = make_uint4(
-                pack_bf16x2(__uint_as_float(oa[qd * 8 + 0]) * inv, __uint_as_float(oa[qd * 8 + 1]) * inv),
-                pack_bf16x2(__uint_as_float(oa[qd * 8 + 2]) * inv, __uint_as_float(oa[qd * 8 + 3]) * inv),
-                pack_bf16x2(__uint_as_float(oa[qd * 8 + 4]) * inv, __uint_as_float(oa[qd * 8 + 5]) * inv),
-                pack_bf16x2(__uint_as_float(oa[qd * 8 + 6]) * inv, __uint_as_float(oa[qd * 8 + 7]) * inv));
-#pragma unroll
-          for (int qd = 0; qd < 4; ++qd)
-            dst[4 + qd] = make_uint4(
-                pack_bf16x2(__uint_as_float(ob[qd * 8 + 0]) * inv, __uint_as_float(ob[qd * 8 + 1]) * inv),
-                pack_bf16x2(__uint_as_float(ob[qd * 8 + 2]) * inv, __uint_as_float(ob[qd * 8 + 3]) * inv),
-                pack_bf16x2(__uint_as_float(ob[qd * 8 + 4]) * inv, __uint_as_float(ob[qd * 8 + 5]) * inv),
-                pack_bf16x2(__uint_as_float(ob[qd * 8 + 6]) * inv, __uint_as_float(ob[qd * 8 + 7]) * inv));
-        }
-        have[w] = false;
-        ++ue[w];
-        did = true;
+    uint4* const stage = s.ostage[warp - kEpiWarp0];
+    for (int u = 0;; ++u) {
+      const int i = u % kUnitRing;
+      // one descriptor per unit, then an end marker
+      if (!mbar_wait_warp_sleep(&s.ud_full[i], (u / kUnitRing) & 1, abort, kSleepNs)) break;
+      const uint32_t row0 = s.urow[i], hd = s.uhead[i];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s.ud_empty[i]);
+      if (hd == 0xFFFFFFFFu) break;
+      const int ob = u & 1;
+      const int rows = static_cast<int>(hd >> 16), head = static_cast<int>(hd & 0xFFFFu);
+      if (!mbar_wait_warp_sleep(&s.o_done[ob], (u >> 1) & 1, abort, kSleepNs)) break;
+      if (!mbar_wait_warp_sleep(&s.l_full[u & 3], (u >> 2) & 1, abort, kSleepNs)) break;
+      tc_fence_after();
+      const bool live = quarter * 32 < rows;
+      uint32_t oa[32], ob2[32];
+      float inv = 1.f;
+      if (live) {
+        const uint32_t to = tmem + lane_sel + tmem_o(ob);
+        tmem_ld32(to, oa);
+        tmem_ld32(to + 32u, ob2);
+        tmem_ld_wait();
+        inv = 1.0f / (s.lsum[u & 3][0][r] + s.lsum[u & 3][1][r]);
       }
-      if (did) {
-        t0 = 0;
-        spins = 0;
-      } else if ((++spins & 15u) == 0u) {
-        // bounded idle time, decided by lane 0 for the whole warp
-        int quit = 0;
-        if (lane == 0) {
-          const uint64_t now = globaltimer_ns();
-          if (t0 == 0) t0 = now;
-          if (*abort) {
-            quit = 1;
-          } else if (now - t0 > kWaitLimitNs) {
-            *abort = 1;
-            quit = 1;
-          }
+      warp_arrive(&s.o_free[ob]);
+      if (live) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          stage[lane * 8 + (c ^ (lane & 7))] = make_uint4(
+              pack_bf16x2(__uint_as_float(oa[c * 8 + 0]) * inv, __uint_as_float(oa[c * 8 + 1]) * inv),
+              pack_bf16x2(__uint_as_float(oa[c * 8 + 2]) * inv, __uint_as_float(oa[c * 8 + 3]) * inv),
+              pack_bf16x2(__uint_as_float(oa[c * 8 + 4]) * inv, __uint_as_float(oa[c * 8 + 5]) * inv),
+              pack_bf16x2(__uint_as_float(oa[c * 8 + 6]) * inv, __uint_as_float(oa[c * 8 + 7]) * inv));
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          stage[lane * 8 + ((c + 4) ^ (lane & 7))] = make_uint4(
+              pack_bf16x2(__uint_as_float(ob2[c * 8 + 0]) * inv, __uint_as_float(ob2[c * 8 + 1]) * inv),
+              pack_bf16x2(__uint_as_float(ob2[c * 8 + 2]) * inv, __uint_as_float(ob2[c * 8 + 3]) * inv),
+              pack_bf16x2(__uint_as_float(ob2[c * 8 + 4]) * inv, __uint_as_float(ob2[c * 8 + 5]) * inv),
+              pack_bf16x2(__uint_as_float(ob2[c * 8 + 6]) * inv, __uint_as_float(ob2[c * 8 + 7]) * inv));
+        __syncwarp();
+        const int c = lane & 7;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+          const int row = 4 * t + (lane >> 3);             // of this warp's 32
+          if (quarter * 32 + row < rows)
+            *reinterpret_cast<uint4*>(out + static_cast<size_t>(row0 + quarter * 32 + row) * dim +
+                                      head * HD + c * 8) = stage[row * 8 + (c ^ (row & 7))];
         }
-        if (__shfl_sync(0xffffffffu, quit, 0)) ok = false;
+        __syncwarp();
       }
     }
   }
@@ -754,9 +661,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
       record_status(status, DORA_ERR_TIMEOUT);
       // let the last TMA load of every buffer land (earlier ones were consumed)
-      for (int w = 0; w < 2; ++w)
-        for (int c = max(0, s.q_issued[w] - 2); c < s.q_issued[w]; ++c)
-          mbar_wait_limited(&s.q_full[w][c & 1], (c >> 1) & 1, 100ull * 1000 * 1000);
+      for (int c = max(0, s.q_issued - 2); c < s.q_issued; ++c)
+        mbar_wait_limited(&s.q_full[c & 1], (c >> 1) & 1, 100ull * 1000 * 1000);
       for (int c = max(0, s.kv_issued - kStages); c < s.kv_issued; ++c)
         mbar_wait_limited(&s.kv_full[c % kStages], (c / kStages) & 1, 100ull * 1000 * 1000);
     }

@@ -124,7 +124,7 @@ __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity,
 // spinning, leaving the issue slots to the other warps of its SM sub-partition.
 __device__ __forceinline__ bool mbar_wait_sleep(uint64_t* bar, uint32_t parity,
                                                 volatile int* abort, uint32_t hint_ns) {
-  if (mbar_try_wait_hint(bar, parity, hint_ns)) return true;
+  if (mbar_try_wait(bar, parity)) return true;   // cheaper when already complete
   const uint64_t t0 = globaltimer_ns();
   while (true) {
     if (mbar_try_wait_hint(bar, parity, hint_ns)) return true;
@@ -300,6 +300,17 @@ __device__ __forceinline__ void mma_commit_multicast(uint64_t* bar, uint16_t cta
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
       " [%0], %1;" ::"r"(smem_u32(bar)), "h"(cta_mask)
       : "memory");
+}
+
+// Warp-collective: 16 consecutive 32-bit columns per lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
 }
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
