@@ -245,6 +245,63 @@ __global__ void __launch_bounds__(kRowThreads) compact_kernel(
 // ---------------------------------------------------------------------------
 // K5: LayerNorm, one warp per row
 // ---------------------------------------------------------------------------
+// Row statistics and normalisation of CPL 16-byte chunks per lane (the row
+// length is chunks * 8 <= 256 * CPL); two rows per warp at a time, so that
+// twice the bytes are in flight.
+template <int CPL>
+__device__ __forceinline__ void ln_row_stats(const uint4 (&v)[CPL], int lane, int chunks,
+                                             float inv_dim, float eps, float& mean, float& rstd) {
+  float sum = 0.f;
+#pragma unroll
+  for (int q = 0; q < CPL; ++q) {
+    if (lane + 32 * q < chunks) {
+      const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) sum += bf16_lo(u[e]) + bf16_hi(u[e]);
+    }
+  }
+  mean = warp_sumf(sum) * inv_dim;
+  float sq = 0.f;
+#pragma unroll
+  for (int q = 0; q < CPL; ++q) {
+    if (lane + 32 * q < chunks) {
+      const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a = bf16_lo(u[e]) - mean, c2 = bf16_hi(u[e]) - mean;
+        sq += a * a + c2 * c2;
+      }
+    }
+  }
+  rstd = rsqrtf(warp_sumf(sq) * inv_dim + eps);
+}
+
+template <int CPL>
+__device__ __forceinline__ void ln_row_store(const uint4 (&v)[CPL], int lane, int chunks,
+                                             float mean, float rstd, const uint4* __restrict__ w,
+                                             const uint4* __restrict__ b, uint4* __restrict__ drow) {
+#pragma unroll
+  for (int q = 0; q < CPL; ++q) {
+    const int c = lane + 32 * q;
+    if (c < chunks) {
+      const uint4 gw = __ldg(w + c), gb = __ldg(b + c);
+      const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+      const uint32_t* g = reinterpret_cast<const uint32_t*>(&gw);
+      const uint32_t* bb = reinterpret_cast<const uint32_t*>(&gb);
+      uint4 o;
+      uint32_t* ow = reinterpret_cast<uint32_t*>(&o);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a = (bf16_lo(u[e]) - mean) * rstd * bf16_lo(g[e]) + bf16_lo(bb[e]);
+        const float c2 = (bf16_hi(u[e]) - mean) * rstd * bf16_hi(g[e]) + bf16_hi(bb[e]);
+        ow[e] = pack_bf16x2(a, c2);
+      }
+      drow[c] = o;
+    }
+  }
+}
+
+template <int CPL>
 __global__ void __launch_bounds__(kRowThreads) layernorm_kernel(
     const uint4* __restrict__ x, int32_t rows_cap, const int32_t* __restrict__ rows_dev,
     int32_t chunks, const uint4* __restrict__ w, const uint4* __restrict__ b, float eps,
@@ -254,53 +311,24 @@ __global__ void __launch_bounds__(kRowThreads) layernorm_kernel(
   int rows = rows_cap;
   if (rows_dev != nullptr) rows = min(rows_cap, max(0, *rows_dev));
   const float inv_dim = 1.0f / static_cast<float>(chunks * 8);
-  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += warps) {
-    const uint4* srow = x + static_cast<size_t>(r) * chunks;
-    uint4 v[kMaxChunksPerLane];
-    float sum = 0.f;
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += 2 * warps) {
+    const int r2 = r + warps;                         // second row of this warp, if any
+    const bool two = r2 < rows;                       // warp-uniform
+    uint4 v[CPL], v2[CPL];
 #pragma unroll
-    for (int q = 0; q < kMaxChunksPerLane; ++q) {
+    for (int q = 0; q < CPL; ++q) {
       const int c = lane + 32 * q;
       if (c < chunks) {
-        v[q] = __ldg(srow + c);
-        const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) sum += bf16_lo(u[e]) + bf16_hi(u[e]);
+        v[q] = __ldg(x + static_cast<size_t>(r) * chunks + c);
+        if (two) v2[q] = __ldg(x + static_cast<size_t>(r2) * chunks + c);
       }
     }
-    const float mean = warp_sumf(sum) * inv_dim;
-    float sq = 0.f;
-#pragma unroll
-    for (int q = 0; q < kMaxChunksPerLane; ++q) {
-      if (lane + 32 * q < chunks) {
-        const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float a = bf16_lo(u[e]) - mean, c2 = bf16_hi(u[e]) - mean;
-          sq += a * a + c2 * c2;
-        }
-      }
-    }
-    const float rstd = rsqrtf(warp_sumf(sq) * inv_dim + eps);
-    uint4* drow = y + static_cast<size_t>(r) * chunks;
-#pragma unroll
-    for (int q = 0; q < kMaxChunksPerLane; ++q) {
-      const int c = lane + 32 * q;
-      if (c < chunks) {
-        const uint4 gw = __ldg(w + c), gb = __ldg(b + c);
-        const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
-        const uint32_t* g = reinterpret_cast<const uint32_t*>(&gw);
-        const uint32_t* bb = reinterpret_cast<const uint32_t*>(&gb);
-        uint4 o;
-        uint32_t* ow = reinterpret_cast<uint32_t*>(&o);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float a = (bf16_lo(u[e]) - mean) * rstd * bf16_lo(g[e]) + bf16_lo(bb[e]);
-          const float c2 = (bf16_hi(u[e]) - mean) * rstd * bf16_hi(g[e]) + bf16_hi(bb[e]);
-          ow[e] = pack_bf16x2(a, c2);
-        }
-        drow[c] = o;
-      }
+    float mean, rstd;
+    ln_row_stats<CPL>(v, lane, chunks, inv_dim, eps, mean, rstd);
+    ln_row_store<CPL>(v, lane, chunks, mean, rstd, w, b, y + static_cast<size_t>(r) * chunks);
+    if (two) {
+      ln_row_stats<CPL>(v2, lane, chunks, inv_dim, eps, mean, rstd);
+      ln_row_store<CPL>(v2, lane, chunks, mean, rstd, w, b, y + static_cast<size_t>(r2) * chunks);
     }
   }
 }
@@ -382,10 +410,20 @@ cudaError_t launch_layernorm(const uint16_t* x, int32_t rows_cap, const int32_t*
                              int32_t dim, const uint16_t* w, const uint16_t* b, float eps,
                              uint16_t* y, cudaStream_t stream) {
   if (rows_cap == 0) return cudaSuccess;
-  layernorm_kernel<<<row_grid(rows_cap), kRowThreads, 0, stream>>>(
-      reinterpret_cast<const uint4*>(x), rows_cap, rows_dev, dim / 8,
-      reinterpret_cast<const uint4*>(w), reinterpret_cast<const uint4*>(b), eps,
-      reinterpret_cast<uint4*>(y));
+  const int chunks = dim / 8;
+  const int grid = row_grid((rows_cap + 1) / 2);
+  const uint4* xx = reinterpret_cast<const uint4*>(x);
+  const uint4* ww = reinterpret_cast<const uint4*>(w);
+  const uint4* bb = reinterpret_cast<const uint4*>(b);
+  uint4* yy = reinterpret_cast<uint4*>(y);
+  // registers sized to the row: 16-byte chunks per lane
+  switch ((chunks + 31) / 32) {
+    case 1: layernorm_kernel<1><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    case 2: layernorm_kernel<2><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    case 3: layernorm_kernel<3><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    case 4: layernorm_kernel<4><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    default: layernorm_kernel<kMaxChunksPerLane><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+  }
   return cudaGetLastError();
 }
 
