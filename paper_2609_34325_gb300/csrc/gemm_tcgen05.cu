@@ -34,7 +34,16 @@ namespace gemm {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int kStages = 4;
+// Pair mode (BN = 256): one MMA of M = 256 spans both CTAs of the cluster,
+// each holding its own 128 rows of X and one half of the W tile, so a stage is
+// 32 KB instead of 48 and six fit; the shared memory read per MMA drops by a
+// third.  Otherwise one MMA per CTA, with W halves multicast.
+template <int BN, bool PAIR>
+struct Mode {
+  static constexpr bool kPair = PAIR;
+  static constexpr int kStages = kPair ? 6 : 4;
+  static constexpr int kBRows = kPair ? BN / 2 : BN;   // W rows held per CTA
+};
 // Epilogue warps per CTA (a multiple of 4: one per TMEM lane quarter) and
 // staging buffers per warp, chosen per epilogue: the ALU-heavy GELU epilogue
 // wants more warps, the others fewer warps with double-buffered stores.
@@ -49,13 +58,13 @@ constexpr uint16_t kPairMask = 0x3;
 
 constexpr int kStageChunk = 32 * 32;   // one warp's 32 rows x 32 columns, bf16
 
-template <int BN, int EPI>
+template <int BN, int EPI, bool PAIR>
 struct Smem {
-  uint16_t a[kStages][BM * BK];   // 16 KB per stage
-  uint16_t b[kStages][BN * BK];   // BN * 128 B per stage
+  uint16_t a[Mode<BN, PAIR>::kStages][BM * BK];                 // 16 KB per stage
+  uint16_t b[Mode<BN, PAIR>::kStages][Mode<BN, PAIR>::kBRows * BK];   // 16 or 32 KB per stage
   uint16_t out[EpiCfg<EPI>::kWarps][EpiCfg<EPI>::kBufs][kStageChunk];   // 2 KB each
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint64_t full[Mode<BN, PAIR>::kStages];
+  uint64_t empty[Mode<BN, PAIR>::kStages];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
@@ -133,7 +142,7 @@ __device__ __forceinline__ void pack_row(const float (&v)[32], uint32_t (&o)[16]
   for (int e = 0; e < 16; ++e) o[e] = pack_bf16x2(v[2 * e], v[2 * e + 1]);
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, bool PAIR>
 __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ CUtensorMap tmY, uint16_t* __restrict__ Y,
@@ -145,10 +154,12 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
     if (threadIdx.x == 0) record_status(status, DORA_ERR_UNSUPPORTED);
     return;
   }
-  Smem<BN, EPI>& s = *reinterpret_cast<Smem<BN, EPI>*>(smem_raw);
+  Smem<BN, EPI, PAIR>& s = *reinterpret_cast<Smem<BN, EPI, PAIR>*>(smem_raw);
   constexpr int kEpiWarps = EpiCfg<EPI>::kWarps;
   constexpr int kBufs = EpiCfg<EPI>::kBufs;
   constexpr int kColGroups = kEpiWarps / 4;
+  constexpr int kStages = Mode<BN, PAIR>::kStages;
+  constexpr bool kPair = Mode<BN, PAIR>::kPair;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   int M = m_cap;
@@ -173,11 +184,14 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&s.full[i], 1);
-      mbar_init(&s.empty[i], kCluster);      // both CTAs' MMAs release a stage
+      // pair mode: the first CTA's MMAs release both CTAs' stages; otherwise
+      // both CTAs' MMAs release a stage (its W halves came from both)
+      mbar_init(&s.empty[i], kPair ? 1 : kCluster);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s.acc_full[i], 1);
-      mbar_init(&s.acc_empty[i], kEpiWarps);
+      // pair mode: the epilogues of both CTAs hand the accumulator back to the first
+      mbar_init(&s.acc_empty[i], kPair ? 2 * kEpiWarps : kEpiWarps);
     }
     mbar_init(&s.drain, 1);
     s.abort_flag = 0;
@@ -188,7 +202,10 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
     tma_prefetch_desc(&tmB);
     tma_prefetch_desc(&tmY);
   }
-  if (warp == 1) tmem_alloc(&s.tmem_base, kTmemCols);
+  if (warp == 1) {
+    if constexpr (kPair) tmem_alloc_pair(&s.tmem_base, kTmemCols);
+    else tmem_alloc(&s.tmem_base, kTmemCols);
+  }
   tc_fence_before();
   cluster_sync();              // peers' barriers are initialised before any multicast
   tc_fence_after();
@@ -209,17 +226,58 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&s.full[st], (BM + BN) * BK * 2);
-          tma_load_2d(s.a[st], &tmA, &s.full[st], kb * BK, mt * BM);
-          tma_load_2d_multicast(s.b[st] + rank * kHalfB * BK, &tmB, &s.full[st], kb * BK,
-                                nt * BN + rank * kHalfB, kPairMask);
+          if constexpr (kPair) {
+            // this CTA's X rows and half of the W tile; the bytes of both CTAs
+            // are counted on the first CTA's barrier, which its MMA waits on
+            if (rank == 0) mbar_arrive_expect_tx(&s.full[st], 2 * (BM + Mode<BN, PAIR>::kBRows) * BK * 2);
+            tma_load_2d_pair(s.a[st], &tmA, &s.full[st], 0, kb * BK, mt * BM);
+            tma_load_2d_pair(s.b[st], &tmB, &s.full[st], 0, kb * BK, nt * BN + rank * kHalfB);
+          } else {
+            mbar_arrive_expect_tx(&s.full[st], (BM + BN) * BK * 2);
+            tma_load_2d(s.a[st], &tmA, &s.full[st], kb * BK, mt * BM);
+            tma_load_2d_multicast(s.b[st] + rank * kHalfB * BK, &tmB, &s.full[st], kb * BK,
+                                  nt * BN + rank * kHalfB, kPairMask);
+          }
           ++it;
         }
       }
       s.issued = it;
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && kPair && rank == 0) {
+      // pair MMA issuer: M = 256 over both CTAs, D in both CTAs' TMEM
+      constexpr uint32_t idesc = idesc_bf16(2 * BM, BN, false);
+      int it = 0, ti = 0;
+      bool ok = true;
+      for (int pr = cid; ok && pr < num_pairs; pr += n_clusters, ++ti) {
+        const int acc = ti & 1;
+        const uint32_t aph = (ti >> 1) & 1;
+        if (!mbar_wait(&s.acc_empty[acc], aph ^ 1, abort)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + static_cast<uint32_t>(acc * BN);
+        for (int kb = 0; kb < kb_count; ++kb) {
+          const int st = it % kStages;
+          const uint32_t ph = (it / kStages) & 1;
+          if (!mbar_wait(&s.full[st], ph, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = sdesc_sw128(smem_u32(s.a[st]), 16, 1024);
+          const uint64_t bd = sdesc_sw128(smem_u32(s.b[st]), 16, 1024);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            mma_bf16_ss_pair(d, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
+          mma_commit_pair(&s.empty[st], kPairMask);        // both CTAs' stages free
+          ++it;
+        }
+        if (ok) mma_commit_pair(&s.acc_full[acc], kPairMask);
+      }
+      s.consumed = it;
+      mma_commit_pair(&s.drain, 0x1);
+      mbar_wait_limited(&s.drain, 0, kWaitLimitNs);
+    } else if (lane == 0) {
+     if constexpr (!kPair) {
       constexpr uint32_t idesc = idesc_bf16(BM, BN, false);
       int it = 0, ti = 0;
       bool ok = true;
@@ -250,6 +308,7 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
       s.consumed = it;
       mma_commit(&s.drain);
       mbar_wait_limited(&s.drain, 0, kWaitLimitNs);
+     }
     }
   } else {
     constexpr int kCols = BN / kColGroups;        // columns per epilogue warp
@@ -305,7 +364,10 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
           // the accumulator is in registers: hand it back to the MMA warp
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&s.acc_empty[acc]);
+          if (lane == 0) {
+            if (kPair && rank != 0) mbar_arrive_remote(&s.acc_empty[acc], 0);
+            else mbar_arrive(&s.acc_empty[acc]);
+          }
         }
 #pragma unroll
         for (int c = 0; c < kBatch; ++c) {
@@ -377,27 +439,29 @@ __global__ void __launch_bounds__(EpiCfg<EPI>::kThreads, 1)
     if (threadIdx.x == 0) {
       record_status(status, DORA_ERR_TIMEOUT);
       // let every TMA load that was issued but never consumed land first
-      for (int it = s.consumed; it < s.issued; ++it)
-        mbar_wait_limited(&s.full[it % kStages], (it / kStages) & 1, 100ull * 1000 * 1000);
+      if (!kPair || rank == 0)
+        for (int it = s.consumed; it < s.issued; ++it)
+          mbar_wait_limited(&s.full[it % kStages], (it / kStages) & 1, 100ull * 1000 * 1000);
       __nanosleep(50000);      // the peer's last multicast halves
     }
     __syncthreads();
   }
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    if constexpr (kPair) tmem_dealloc_pair(tmem, kTmemCols);
+    else tmem_dealloc(tmem, kTmemCols);
   }
   cluster_sync();              // no CTA leaves while its peer may still signal it
 }
 
-template <int BN, int EPI>
+template <int BN, int EPI, bool PAIR>
 static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
                                  const CUtensorMap& ty, uint16_t* y,
                                  const uint16_t* bias, const uint16_t* residual, int m_cap,
                                  const int32_t* m_dev, int n, int k, int32_t* status,
                                  cudaStream_t stream) {
-  const size_t smem = sizeof(Smem<BN, EPI>);
-  auto kern = gemm_kernel<BN, EPI>;
+  const size_t smem = sizeof(Smem<BN, EPI, PAIR>);
+  auto kern = gemm_kernel<BN, EPI, PAIR>;
   cudaError_t e =
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -413,7 +477,7 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   // as many co-resident clusters as fit, capped by the tile pairs of m_cap
-  static int max_clusters[64] = {0};
+  static int max_clusters[64] = {0};   // per instantiation and device
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev < 0 || dev >= 64) dev = 0;
@@ -432,6 +496,9 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
                             status);
 }
 
+// Pair mode for BN = 256, except for the residual epilogue over a short K
+// (the projection linear), whose epilogue traffic then dominates: measured
+// slower in pair mode.
 template <int BN>
 static cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& ty,
                              uint16_t* y,
@@ -440,14 +507,17 @@ static cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const
                              cudaStream_t stream) {
   switch (epi) {
     case DORA_EPI_BIAS_GELU:
-      return launch_bn_epi<BN, DORA_EPI_BIAS_GELU>(ta, tb, ty, y, bias, residual, m_cap, m_dev, n, k,
-                                                   status, stream);
+      return launch_bn_epi<BN, DORA_EPI_BIAS_GELU, BN == 256>(ta, tb, ty, y, bias, residual, m_cap,
+                                                              m_dev, n, k, status, stream);
     case DORA_EPI_BIAS_RESIDUAL:
-      return launch_bn_epi<BN, DORA_EPI_BIAS_RESIDUAL>(ta, tb, ty, y, bias, residual, m_cap, m_dev, n,
-                                                       k, status, stream);
+      if (BN == 256 && k > 1024)
+        return launch_bn_epi<BN, DORA_EPI_BIAS_RESIDUAL, BN == 256>(ta, tb, ty, y, bias, residual,
+                                                                    m_cap, m_dev, n, k, status, stream);
+      return launch_bn_epi<BN, DORA_EPI_BIAS_RESIDUAL, false>(ta, tb, ty, y, bias, residual, m_cap,
+                                                              m_dev, n, k, status, stream);
     default:
-      return launch_bn_epi<BN, DORA_EPI_BIAS>(ta, tb, ty, y, bias, residual, m_cap, m_dev, n, k,
-                                              status, stream);
+      return launch_bn_epi<BN, DORA_EPI_BIAS, BN == 256>(ta, tb, ty, y, bias, residual, m_cap, m_dev,
+                                                         n, k, status, stream);
   }
 }
 
