@@ -196,8 +196,11 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
     def i32(a):
         return torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).to(dev)
 
+    # weights as a deployment loads them: LayerNorm affines folded into the QKV
+    # and fc1 weights once (dora_fold_block_weights), outside the step
     blocks = [P.BlockWeights({k: bf(v) for k, v in w.items()}, cfg.dim, cfg.heads, cfg.mlp_dim,
-                             cfg.ln_eps) for w in hw.weights]
+                             cfg.ln_eps).fold(stream) for w in hw.weights]
+    torch.cuda.synchronize()
     sets = [dict(x=bf(s["x"]), keeps=[i32(k) for k in s["keeps"]],
                  tables=[torch.from_numpy(t).to(dev) for t in s["tables"]]) for s in hw.sets]
     cu0, ids0 = i32(hw.cu0), i32(hw.ids0)
@@ -229,7 +232,7 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
                                     cu_out=cubuf[j % 2], ids_out=idbuf[j % 2], kept_idx=kept,
                                     stream=stream)
                 cu, ids = cubuf[j % 2], idbuf[j % 2]
-                n += 1 + 8
+                n += 1 + 9
             else:
                 P.dora_pruned_block(x, cu, blocks[l], cfg.n_tokens, out, ws, ids_in=ids,
                                     stream=stream)
@@ -414,8 +417,23 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
     launch with CUDA events on the launching stream.  Returns per-class times
     and algorithmic work."""
     d, m = cfg.dim, cfg.mlp_dim
-    bf16 = torch.bfloat16
-    xn = torch.zeros(t_cap, d, dtype=bf16, device=dev)
+    bf16, f32 = torch.bfloat16, torch.float32
+    sm = torch.zeros(d // 64, t_cap, 2, dtype=f32, device=dev)      # slice moments
+    mv = torch.zeros(t_cap, 2, dtype=f32, device=dev)               # row moments
+    mv2 = torch.zeros(t_cap, 2, dtype=f32, device=dev)              # after a deletion
+    # the folded QKV and fc1 weights, as dora_fold_block_weights makes them
+    folded = []
+    for blk in blocks:
+        w = blk.tensors
+        fl = {}
+        for name, n_out, g, be, b in (("qkv", 3 * d, "ln1_w", "ln1_b", "b_qkv"),
+                                      ("fc1", m, "ln2_w", "ln2_b", "b_fc1")):
+            fl[name] = (torch.zeros(n_out, d, dtype=bf16, device=dev),
+                        torch.zeros(n_out, dtype=f32, device=dev),
+                        torch.zeros(n_out, dtype=f32, device=dev))
+            P.dora_fold_ln_linear(w["w_" + name], w[g], w[be], *fl[name], bias=w[b], stream=stream)
+        folded.append(fl)
+    sb = 8.0 * d / 64          # slice-moment bytes per row
     qkv = torch.zeros(t_cap, 3 * d, dtype=bf16, device=dev)
     o = torch.zeros(t_cap, d, dtype=bf16, device=dev)
     hattn = torch.zeros(t_cap, d, dtype=bf16, device=dev)
@@ -455,20 +473,25 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
             n_in, n_out = lens[l]
             T, To = int(n_in.sum()), int(n_out.sum())
             rows = cu[B:]
-            launch("layernorm", lambda: P.dora_layernorm(x, w["ln1_w"], w["ln1_b"], cfg.ln_eps,
-                                                        xn, rows_dev=rows, stream=stream),
-                   dict(bytes=4.0 * T * d))
-            launch("gemm_qkv", lambda: P.dora_linear(xn, w["w_qkv"], qkv, bias=w["b_qkv"],
-                                                m_dev=rows, stream=stream),
-                   dict(flops=2.0 * T * 3 * d * d, bytes=2.0 * (T * d + 3 * d * d + 3 * T * d)))
+            fl = folded[l]
+            launch("row_stats", lambda: P.dora_row_stats(x, mv, rows_dev=rows, stream=stream),
+                   dict(bytes=2.0 * T * d + 8.0 * T))
+            launch("gemm_qkv", lambda: P.dora_linear_ln(x, mv, cfg.ln_eps, *fl["qkv"], qkv,
+                                                   m_dev=rows, stream=stream),
+                   dict(flops=2.0 * T * 3 * d * d,
+                        bytes=2.0 * (T * d + 3 * d * d + 3 * T * d) + 8.0 * T + 24.0 * d))
             launch("attention", lambda: P.dora_varlen_attn(qkv, cu, cfg.n_tokens, cfg.heads, o,
                                                           stream=stream),
                    dict(flops=A.attention_flops(n_in, cfg.heads), bytes=A.attention_bytes(T, d)))
-            launch("gemm_proj", lambda: P.dora_linear(o, w["w_proj"], hattn, bias=w["b_proj"],
-                                                residual=x, epilogue=P.EPI_BIAS_RESIDUAL,
-                                                m_dev=rows, stream=stream),
-                   dict(flops=2.0 * T * d * d, bytes=2.0 * (3 * T * d + d * d)))
             out = xb[l % 2]
+            launch("gemm_proj",
+                   lambda: P.dora_linear_residual_stats(o, w["w_proj"], x, hattn, sm,
+                                                        bias=w["b_proj"], m_dev=rows,
+                                                        stream=stream),
+                   dict(flops=2.0 * T * d * d, bytes=2.0 * (3 * T * d + d * d) + sb * T))
+            launch("merge_moments", lambda: P.dora_merge_moments(sm, mv, rows_dev=rows,
+                                                                stream=stream),
+                   dict(bytes=sb * T + 8.0 * T))
             if l in prune:
                 j = prune.index(l)
                 cuo, ido = cub[j % 2], idb[j % 2]
@@ -480,23 +503,19 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
                        lambda: P.dora_select_keep(scores, cu, inp["keeps"][j], cfg.n_tokens,
                                                   kept, cuo, stream=stream),
                        dict(bytes=4.0 * T + 4.0 * To + 8.0 * (B + 1) + 4.0 * B))
-                launch("compact_ln",
-                       lambda: P.dora_compact_ln(hattn, kept, cuo, w["ln2_w"], w["ln2_b"],
-                                                 cfg.ln_eps, hkeep, xn, ids_in=ids, ids_out=ido,
-                                                 stream=stream),
-                       dict(bytes=3.0 * 2 * To * d + 4.0 * To + 8.0 * To + 4.0 * (B + 1)))
-                hk, rows2 = hkeep, cuo[B:]
+                launch("compact",
+                       lambda: P.dora_compact_stats(hattn, kept, cuo, hkeep, mv, mv2, ids_in=ids,
+                                                    ids_out=ido, stream=stream),
+                       dict(bytes=2.0 * 2 * To * d + 16.0 * To + 4.0 * To + 8.0 * To
+                            + 4.0 * (B + 1)))
+                hk, rows2, mvk = hkeep, cuo[B:], mv2
                 cu, ids = cuo, ido
             else:
-                launch("layernorm", lambda: P.dora_layernorm(hattn, w["ln2_w"], w["ln2_b"],
-                                                            cfg.ln_eps, xn, rows_dev=rows,
-                                                            stream=stream),
-                       dict(bytes=4.0 * T * d))
-                hk, rows2 = hattn, rows
-            launch("gemm_fc1", lambda: P.dora_linear(xn, w["w_fc1"], u, bias=w["b_fc1"],
-                                                epilogue=P.EPI_BIAS_GELU, m_dev=rows2,
-                                                stream=stream),
-                   dict(flops=2.0 * To * d * m, bytes=2.0 * (To * d + d * m + To * m)))
+                hk, rows2, mvk = hattn, rows, mv
+            launch("gemm_fc1", lambda: P.dora_linear_ln(hk, mvk, cfg.ln_eps, *fl["fc1"], u,
+                                                   gelu=True, m_dev=rows2, stream=stream),
+                   dict(flops=2.0 * To * d * m,
+                        bytes=2.0 * (To * d + d * m + To * m) + 8.0 * To + 8.0 * m))
             launch("gemm_fc2", lambda: P.dora_linear(u, w["w_fc2"], out, bias=w["b_fc2"],
                                                 residual=hk, epilogue=P.EPI_BIAS_RESIDUAL,
                                                 m_dev=rows2, stream=stream),
@@ -551,12 +570,12 @@ def roofline_report(kern, peaks, peak_src):
         "peak_kind": f"bf16 burst ({tag})", "arith_intensity": round(ai, 1),
         "attainable_from_hbm": round(attain, 1), "frac_of_attainable": round(at_tf / attain, 4),
         "share_of_step": round(a["share"], 4)}
-    c = kern["compact_ln"]
+    c = kern["compact"]
     c_gbs = c["bytes"] / (c["ms"] * 1e-3) / 1e9
     s = kern["select_keep"]
     sel_gbs = s["bytes"] / (s["ms"] * 1e-3) / 1e9
     out["roofline_compact"] = {
-        "kernel": "compact_ln (compaction fused with LayerNorm')", "bound": "hbm",
+        "kernel": "compact (compaction with the row moments of LayerNorm')", "bound": "hbm",
         "achieved": round(c_gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
         "frac": round(c_gbs / peaks["hbm_gbs"], 4), "peak_kind": f"HBM copy ({tag})",
         "select_keep_gbs": round(sel_gbs, 1), "select_keep_us": round(1000 * s["ms"] / s["launches"], 2),

@@ -130,6 +130,18 @@ int dora_compact_ln(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
                     int32_t* status, dora_stream_t stream);
 
 /*
+ * dora_compact_stats -- dora_compact that also carries the row moments of
+ * every kept row (see "LayerNorm folded into the linear after it" below):
+ * mv_out[r] = mv_in[kept_idx[r]] (fp32 [t_in_cap, 2] each, 8-byte aligned),
+ * the input of the LayerNorm' folded into fc1, bit for bit what the rows had
+ * before the deletion.
+ */
+int dora_compact_stats(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
+                       const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
+                       const int32_t* ids_in, const float* mv_in, dora_bf16* packed,
+                       int32_t* ids_out, float* mv_out, int32_t* status, dora_stream_t stream);
+
+/*
  * dora_layernorm -- y = LayerNorm(x) row by row (the LayerNorm of Eq. 1),
  * biased variance, fp32 statistics, affine w, b (bf16 [dim]).
  * rows_cap   rows the buffers hold; rows_dev (nullable) points at the live row
@@ -156,6 +168,81 @@ int dora_layernorm(const dora_bf16* x, int32_t rows_cap, const int32_t* rows_dev
 int dora_linear(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
                 const dora_bf16* w, int32_t n, const dora_bf16* bias, const dora_bf16* residual,
                 int32_t epilogue, dora_bf16* y, int32_t* status, dora_stream_t stream);
+
+/*
+ * LayerNorm folded into the linear after it.  The LayerNorm of Eq. 1 before
+ * the QKV linear, and LayerNorm' before fc1, need only each row's mean and
+ * rstd = 1/sqrt(var + eps) once the affine is moved into the weights:
+ *     LayerNorm(x) W^T + b = rstd (x W'^T - mean c) + d,
+ *     W' = W diag(gamma) rounded to bf16,  c = W' 1,  d = W beta + b,
+ * exact algebra; the GEMM then reads the raw rows.  Two formats carry the row
+ * statistics (fp32, from the bf16 values):
+ *  - row moments mv [rows_cap, 2]: mv[2 r] = mean and mv[2 r + 1] = biased
+ *    variance of row r (what dora_linear_ln reads);
+ *  - slice moments sm [dim / 64, rows_cap, 2], slice-major: for row r and
+ *    64-column slice s, sm[2 (s rows_cap + r)] = the slice's mean and
+ *    sm[2 (s rows_cap + r) + 1] = the sum of squared deviations from it
+ *    (what a residual GEMM epilogue can write, a row being split over
+ *    several tiles).  dora_merge_moments turns them into row moments with the
+ *    pairwise update of Chan, Golub & LeVeque.
+ * rows_cap is the row capacity of the call that writes them (rows_cap, m_cap
+ * or t_in_cap).
+ */
+
+/*
+ * dora_row_stats -- row moments of bf16 rows x [rows_cap, dim] into mv
+ * (fp32 [rows_cap, 2], 8-byte aligned).  rows_dev (nullable) is the live row
+ * count on the device; rows beyond it are skipped.  dim % 8 == 0, dim <= 2048.
+ */
+int dora_row_stats(const dora_bf16* x, int32_t rows_cap, const int32_t* rows_dev, int32_t dim,
+                   float* mv, dora_stream_t stream);
+
+/*
+ * dora_merge_moments -- row moments mv (fp32 [rows_cap, 2]) of rows whose
+ * slice moments are sm (fp32 [slices, rows_cap, 2]): mean = (1/S) sum mean_s,
+ * var = (sum M2_s + 64 sum (mean_s - mean)^2) / (64 S).  rows_dev as in
+ * dora_row_stats.
+ */
+int dora_merge_moments(const float* sm, int32_t rows_cap, const int32_t* rows_dev,
+                       int32_t slices, float* mv, dora_stream_t stream);
+
+/*
+ * dora_fold_ln_linear -- moves a LayerNorm affine (gamma, beta: bf16 [k])
+ * into the linear W [n, k] (bias nullable bf16 [n]) that follows it:
+ * w_out [n, k] = bf16(W diag(gamma)) (one rounding: the product of two bf16
+ * values is exact in fp32), colsum fp32 [n] = row sums of w_out, colbias fp32
+ * [n] = W beta + bias.  Done once per set of weights.  k % 8 == 0; all
+ * pointers 16-byte aligned.
+ */
+int dora_fold_ln_linear(const dora_bf16* w, int32_t n, int32_t k, const dora_bf16* gamma,
+                        const dora_bf16* beta, const dora_bf16* bias, dora_bf16* w_out,
+                        float* colsum, float* colbias, dora_stream_t stream);
+
+/*
+ * dora_linear_ln -- y = LayerNorm(x) W^T + b, or its GELU when gelu != 0,
+ * computed as rstd (x W'^T - mean c) + d with W', c (colsum), d (colbias)
+ * from dora_fold_ln_linear and each row's mean and var from the row moments
+ * mv of x (fp32 [m_cap, 2]; dora_row_stats, dora_merge_moments or
+ * dora_compact_stats), rstd = 1/sqrt(var + eps).  eps is the LayerNorm
+ * epsilon.  x [m_cap, k] with
+ * k % 64 == 0, k <= 2048; n % 32 == 0; m_dev as in dora_linear.  fp32
+ * accumulation and epilogue, one rounding to bf16.
+ */
+int dora_linear_ln(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
+                   const float* mv, float eps, const dora_bf16* w_folded, int32_t n,
+                   const float* colsum, const float* colbias, int32_t gelu, dora_bf16* y,
+                   int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_linear_residual_stats -- dora_linear with DORA_EPI_BIAS_RESIDUAL that
+ * also writes the slice moments of the rounded output rows to stats_out (fp32
+ * [n / 64, m_cap, 2]; dora_merge_moments makes row moments of them), for the
+ * folded LayerNorm that reads them next.  n % 64 == 0; live rows only.
+ */
+int dora_linear_residual_stats(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
+                               const dora_bf16* w, int32_t n, const dora_bf16* bias,
+                               const dora_bf16* residual, dora_bf16* y, float* stats_out,
+                               int32_t* status, dora_stream_t stream);
 
 /*
  * dora_varlen_attn -- packed variable-length multi-head self-attention
@@ -207,16 +294,35 @@ typedef struct dora_block_weights {
   int32_t heads;
   int32_t mlp_dim;   /* multiple of 64 */
   float ln_eps;      /* LayerNorm epsilon, e.g. 1e-6 */
+  /* Nullable: these weights with both LayerNorms folded in, written by
+   * dora_fold_block_weights (256-byte aligned).  NULL = the block folds them
+   * into its workspace on every call (same result, more work per call). */
+  const void* folded;
 } dora_block_weights;
 
-/* Bytes of device workspace dora_pruned_block needs for t_cap rows. */
+/* Bytes of device workspace dora_pruned_block needs for t_cap rows (it
+ * includes room for the folded weights when w->folded is NULL). */
 size_t dora_workspace_size(int32_t t_cap, int32_t batch, const dora_block_weights* w);
+
+/* Bytes dora_fold_block_weights writes for these weights. */
+size_t dora_folded_weights_size(const dora_block_weights* w);
+
+/*
+ * dora_fold_block_weights -- folds LayerNorm (ln1_w, ln1_b) into the QKV
+ * linear and LayerNorm' (ln2_w, ln2_b) into fc1 (dora_fold_ln_linear on
+ * both), into `folded` (device, 256-byte aligned, folded_bytes >=
+ * dora_folded_weights_size(w)).  Call once after loading the weights and put
+ * the pointer in w->folded; refold whenever those weights change.
+ */
+int dora_fold_block_weights(const dora_block_weights* w, void* folded, size_t folded_bytes,
+                            dora_stream_t stream);
 
 /*
  * dora_pruned_block -- one block of Eq. 1 on the packed batch:
- *   LN1 -> QKV linear -> varlen attention -> projection + residual  (H_attn)
- *   [select_keep -> compaction fused with LN2]                       (H_keep)
- *   fc1 + GELU -> fc2 + residual                                     (H_next)
+ *   row moments -> QKV linear with LN1 folded in -> varlen attention
+ *     -> projection + residual (+ slice moments) -> merged moments  (H_attn)
+ *   [select_keep -> compaction carrying the row moments]            (H_keep)
+ *   fc1 with LN2 folded in + GELU -> fc2 + residual                 (H_next)
  * x_in      bf16 [t_cap, dim], rows [0, cu_in[batch]) live.
  * cu_in     int32 [batch+1]; ids_in int32 [t_cap] original token ids
  *           (nullable when scores is NULL).
@@ -265,8 +371,8 @@ int32_t* dora_workspace_status(void* workspace);
  *    that loads the library, for the life of the process.  A block whose
  *    dora_workspace_size(t_cap, batch, w) exceeds it is rejected with
  *    DORA_ERR_SCRATCH_TOO_SMALL before anything is launched (32 MiB fits e.g.
- *    a DeiT-Tiny-shape batch of 8 x 197 tokens, or about 1,900 token rows of
- *    a DeiT-Base-shape block).
+ *    a DeiT-Tiny-shape batch of 8 x 197 tokens, or about 2,100 token rows of
+ *    a DeiT-Base-shape block with pre-folded weights, 1,600 without).
  *  - The first call on a device looks up the device address of the scratch
  *    array (cudaGetSymbolAddress) with that device current; make that first
  *    call before any stream capture on the device.

@@ -19,7 +19,10 @@ __all__ = [
     "dora_select_keep", "dora_compact", "dora_compact_ln", "dora_layernorm", "dora_linear",
     "dora_varlen_attn", "dora_gather_scores", "BlockWeights", "dora_workspace_size",
     "dora_pruned_block", "dora_workspace_status", "dora_read_status", "alloc_workspace",
-    "dora_pruned_block_noalloc", "NOALLOC_SCRATCH_BYTES",
+    "dora_pruned_block_noalloc", "NOALLOC_SCRATCH_BYTES", "dora_row_stats",
+    "dora_fold_ln_linear", "dora_linear_ln", "dora_linear_residual_stats",
+    "dora_folded_weights_size", "dora_fold_block_weights", "dora_compact_stats",
+    "dora_merge_moments",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -50,6 +53,17 @@ _SIGS = {
     "dora_pruned_block_noalloc": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
                                                  _vp, _vp, _vp, _vp, _vp, _vp]),
     "dora_read_status": (ctypes.c_int, [_vp, _vp]),
+    "dora_row_stats": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _vp]),
+    "dora_fold_ln_linear": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
+    "dora_linear_ln": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _f32, _vp, _i32, _vp, _vp, _i32,
+                                      _vp, _vp, _vp]),
+    "dora_linear_residual_stats": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _i32, _vp, _vp, _vp,
+                                                  _vp, _vp, _vp]),
+    "dora_folded_weights_size": (_sz, [_vp]),
+    "dora_fold_block_weights": (ctypes.c_int, [_vp, _vp, _sz, _vp]),
+    "dora_compact_stats": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp,
+                                          _vp, _vp, _vp]),
+    "dora_merge_moments": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _vp]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -63,7 +77,7 @@ class DoraError(RuntimeError):
 class _BlockWeightsC(ctypes.Structure):
     _fields_ = [(n, _vp) for n in ("ln1_w", "ln1_b", "w_qkv", "b_qkv", "w_proj", "b_proj",
                                    "ln2_w", "ln2_b", "w_fc1", "b_fc1", "w_fc2", "b_fc2")] + [
-        ("dim", _i32), ("heads", _i32), ("mlp_dim", _i32), ("ln_eps", _f32)]
+        ("dim", _i32), ("heads", _i32), ("mlp_dim", _i32), ("ln_eps", _f32), ("folded", _vp)]
 
 
 def library_path() -> str:
@@ -157,6 +171,30 @@ def dora_compact(x, kept_idx, cu_out, packed, ids_in=None, ids_out=None, status=
            "dora_compact")
 
 
+def dora_compact_stats(x, kept_idx, cu_out, packed, mv_in, mv_out, ids_in=None, ids_out=None,
+                       status=None, stream=None):
+    """dora_compact that also carries the row moments: mv_out[r] = mv_in[kept_idx[r]]."""
+    _req(x, torch.bfloat16, "x")
+    _req(packed, torch.bfloat16, "packed")
+    _req(mv_in, torch.float32, "mv_in")
+    _req(mv_out, torch.float32, "mv_out")
+    _req(kept_idx, torch.int32, "kept_idx")
+    _req(cu_out, torch.int32, "cu_out")
+    _req(ids_in, torch.int32, "ids_in", optional=True)
+    _req(ids_out, torch.int32, "ids_out", optional=True)
+    _req(status, torch.int32, "status", optional=True)
+    t_in_cap, dim = x.shape
+    if packed.shape[0] < t_in_cap or packed.shape[1] != dim:
+        raise ValueError("packed must hold at least as many rows as x")
+    if mv_in.numel() < t_in_cap * 2 or mv_out.numel() < t_in_cap * 2:
+        raise ValueError("mv_in and mv_out must hold [t_in_cap, 2] floats")
+    _check(load_library().dora_compact_stats(_ptr(x), dim, _ptr(kept_idx), _ptr(cu_out),
+                                             cu_out.numel() - 1, t_in_cap, _ptr(ids_in),
+                                             _ptr(mv_in), _ptr(packed), _ptr(ids_out),
+                                             _ptr(mv_out), _ptr(status), _stream(stream)),
+           "dora_compact_stats")
+
+
 def dora_compact_ln(x, kept_idx, cu_out, ln_w, ln_b, eps, packed, ln_out, ids_in=None,
                     ids_out=None, status=None, stream=None):
     for n, t in (("x", x), ("packed", packed), ("ln_out", ln_out), ("ln_w", ln_w),
@@ -204,6 +242,88 @@ def dora_linear(x, w, y, bias=None, residual=None, epilogue=EPI_BIAS, m_dev=None
                                       _stream(stream)), "dora_linear")
 
 
+def dora_row_stats(x, mv, rows_dev=None, stream=None):
+    """Row moments (mean, biased variance) of the rows of x [rows, dim] into
+    mv (fp32 [rows, 2])."""
+    _req(x, torch.bfloat16, "x")
+    _req(mv, torch.float32, "mv")
+    _req(rows_dev, torch.int32, "rows_dev", optional=True)
+    rows, dim = x.shape
+    if mv.numel() < rows * 2:
+        raise ValueError("mv must hold [rows, 2] floats")
+    _check(load_library().dora_row_stats(_ptr(x), rows, _ptr(rows_dev), dim, _ptr(mv),
+                                         _stream(stream)), "dora_row_stats")
+
+
+def dora_merge_moments(sm, mv, rows_dev=None, stream=None):
+    """Row moments mv (fp32 [rows, 2]) from slice moments sm (fp32 [S, rows, 2])."""
+    _req(sm, torch.float32, "sm")
+    _req(mv, torch.float32, "mv")
+    _req(rows_dev, torch.int32, "rows_dev", optional=True)
+    slices, rows = sm.shape[0], sm.shape[1]
+    if mv.numel() < rows * 2:
+        raise ValueError("mv must hold [rows, 2] floats")
+    _check(load_library().dora_merge_moments(_ptr(sm), rows, _ptr(rows_dev), slices, _ptr(mv),
+                                             _stream(stream)), "dora_merge_moments")
+
+
+def dora_fold_ln_linear(w, gamma, beta, w_out, colsum, colbias, bias=None, stream=None):
+    """LayerNorm affine into the linear after it: w_out = bf16(w diag(gamma)),
+    colsum = w_out 1, colbias = w beta + bias."""
+    for n, t in (("w", w), ("gamma", gamma), ("beta", beta), ("w_out", w_out)):
+        _req(t, torch.bfloat16, n)
+    _req(bias, torch.bfloat16, "bias", optional=True)
+    _req(colsum, torch.float32, "colsum")
+    _req(colbias, torch.float32, "colbias")
+    n_out, k = w.shape
+    if tuple(w_out.shape) != (n_out, k) or colsum.numel() < n_out or colbias.numel() < n_out:
+        raise ValueError("shape mismatch: w, w_out [n,k]; colsum, colbias [n]")
+    _check(load_library().dora_fold_ln_linear(_ptr(w), n_out, k, _ptr(gamma), _ptr(beta),
+                                              _ptr(bias), _ptr(w_out), _ptr(colsum),
+                                              _ptr(colbias), _stream(stream)),
+           "dora_fold_ln_linear")
+
+
+def dora_linear_ln(x, mv, eps, w_folded, colsum, colbias, y, gelu=False, m_dev=None,
+                   status=None, stream=None):
+    """y = LayerNorm(x) W^T + b (GELU of it when gelu) from folded weights and
+    the row moments mv of x."""
+    _req(x, torch.bfloat16, "x")
+    _req(w_folded, torch.bfloat16, "w_folded")
+    _req(y, torch.bfloat16, "y")
+    _req(mv, torch.float32, "mv")
+    _req(colsum, torch.float32, "colsum")
+    _req(colbias, torch.float32, "colbias")
+    _req(m_dev, torch.int32, "m_dev", optional=True)
+    _req(status, torch.int32, "status", optional=True)
+    m_cap, k = x.shape
+    n = w_folded.shape[0]
+    if w_folded.shape[1] != k or tuple(y.shape) != (m_cap, n):
+        raise ValueError("shape mismatch: x [M,K], w_folded [N,K], y [M,N]")
+    _check(load_library().dora_linear_ln(_ptr(x), m_cap, _ptr(m_dev), k, _ptr(mv), float(eps),
+                                         _ptr(w_folded), n, _ptr(colsum), _ptr(colbias),
+                                         1 if gelu else 0, _ptr(y), _ptr(status),
+                                         _stream(stream)), "dora_linear_ln")
+
+
+def dora_linear_residual_stats(x, w, residual, y, stats_out, bias=None, m_dev=None, status=None,
+                               stream=None):
+    """y = residual + x W^T + b, plus the slice moments of y's rows."""
+    for n_, t in (("x", x), ("w", w), ("residual", residual), ("y", y)):
+        _req(t, torch.bfloat16, n_)
+    _req(bias, torch.bfloat16, "bias", optional=True)
+    _req(stats_out, torch.float32, "stats_out")
+    _req(m_dev, torch.int32, "m_dev", optional=True)
+    _req(status, torch.int32, "status", optional=True)
+    m_cap, k = x.shape
+    n = w.shape[0]
+    if w.shape[1] != k or tuple(y.shape) != (m_cap, n) or tuple(residual.shape) != (m_cap, n):
+        raise ValueError("shape mismatch: x [M,K], w [N,K], residual, y [M,N]")
+    _check(load_library().dora_linear_residual_stats(
+        _ptr(x), m_cap, _ptr(m_dev), k, _ptr(w), n, _ptr(bias), _ptr(residual), _ptr(y),
+        _ptr(stats_out), _ptr(status), _stream(stream)), "dora_linear_residual_stats")
+
+
 def dora_varlen_attn(qkv, cu_seqlens, max_seqlen, heads, out, head_dim=64, softmax_scale=0.0,
                      status=None, stream=None):
     _req(qkv, torch.bfloat16, "qkv")
@@ -245,8 +365,25 @@ class BlockWeights:
             _req(t, torch.bfloat16, n, optional=n.startswith("b_"))
             self.tensors[n] = t
         self.dim, self.heads, self.mlp_dim, self.ln_eps = dim, heads, mlp_dim, ln_eps
+        self.folded = None
         self.c = _BlockWeightsC(*[_ptr(self.tensors[n]) for n in self.NAMES], dim, heads, mlp_dim,
-                                float(ln_eps))
+                                float(ln_eps), None)
+
+    def fold(self, stream=None):
+        """Fold both LayerNorms into the QKV and fc1 weights once
+        (dora_fold_block_weights); later blocks run on the folded copy.
+        Call again after changing any of the weights."""
+        n = int(load_library().dora_folded_weights_size(ctypes.byref(self.c)))
+        buf = torch.empty(n + 256, dtype=torch.uint8, device=self.tensors["w_qkv"].device)
+        off = (-buf.data_ptr()) % 256
+        folded = buf[off:off + n]
+        self.c.folded = None
+        _check(load_library().dora_fold_block_weights(ctypes.byref(self.c), _ptr(folded), n,
+                                                      _stream(stream)),
+               "dora_fold_block_weights")
+        self.folded = folded
+        self.c.folded = _ptr(folded)
+        return self
 
 
 def dora_workspace_size(t_cap, batch, weights: BlockWeights) -> int:

@@ -39,6 +39,7 @@ int current_device_checked() {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+bool aligned8(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 7u) == 0; }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
@@ -130,7 +131,8 @@ static int compact_common(const dora_bf16* x, int32_t dim, const int32_t* kept_i
                           const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
                           const int32_t* ids_in, const dora_bf16* ln_w, const dora_bf16* ln_b,
                           float eps, dora_bf16* packed, int32_t* ids_out, dora_bf16* ln_out,
-                          int32_t* status, dora_stream_t stream) {
+                          const float* mv_in, float* mv_out, int32_t* status,
+                          dora_stream_t stream) {
   DORA_CHECK_ARG(batch >= 0 && t_in_cap >= 0);
   DORA_CHECK_ARG(dim > 0 && dim % 8 == 0 && dim <= kMaxDimRow);
   DORA_CHECK_ARG(cu_out != nullptr);
@@ -138,10 +140,11 @@ static int compact_common(const dora_bf16* x, int32_t dim, const int32_t* kept_i
   DORA_CHECK_ARG(aligned16(x) && aligned16(packed) && aligned16(ln_out));
   DORA_CHECK_ARG((ids_out == nullptr) || (ids_in != nullptr));
   if (ln_out) DORA_CHECK_ARG(ln_w && ln_b && aligned16(ln_w) && aligned16(ln_b) && eps >= 0.f);
+  if (mv_out) DORA_CHECK_ARG(mv_in && aligned8(mv_in) && aligned8(mv_out));
   DORA_CHECK_DEVICE();
   if (t_in_cap == 0) return DORA_OK;
   return cuda_status(launch_compact(x, dim, kept_idx, cu_out, batch, t_in_cap, ids_in, ln_w, ln_b,
-                                    eps, packed, ids_out, ln_out, status,
+                                    eps, packed, ids_out, ln_out, mv_in, mv_out, status,
                                     reinterpret_cast<cudaStream_t>(stream)));
 }
 
@@ -149,7 +152,16 @@ int dora_compact(const dora_bf16* x, int32_t dim, const int32_t* kept_idx, const
                  int32_t batch, int32_t t_in_cap, const int32_t* ids_in, dora_bf16* packed,
                  int32_t* ids_out, int32_t* status, dora_stream_t stream) {
   return compact_common(x, dim, kept_idx, cu_out, batch, t_in_cap, ids_in, nullptr, nullptr, 0.f,
-                        packed, ids_out, nullptr, status, stream);
+                        packed, ids_out, nullptr, nullptr, nullptr, status, stream);
+}
+
+int dora_compact_stats(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
+                       const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
+                       const int32_t* ids_in, const float* mv_in, dora_bf16* packed,
+                       int32_t* ids_out, float* mv_out, int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(mv_in != nullptr && mv_out != nullptr);
+  return compact_common(x, dim, kept_idx, cu_out, batch, t_in_cap, ids_in, nullptr, nullptr, 0.f,
+                        packed, ids_out, nullptr, mv_in, mv_out, status, stream);
 }
 
 int dora_compact_ln(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
@@ -159,7 +171,7 @@ int dora_compact_ln(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
                     int32_t* status, dora_stream_t stream) {
   DORA_CHECK_ARG(ln_out != nullptr);
   return compact_common(x, dim, kept_idx, cu_out, batch, t_in_cap, ids_in, ln_w, ln_b, eps,
-                        packed, ids_out, ln_out, status, stream);
+                        packed, ids_out, ln_out, nullptr, nullptr, status, stream);
 }
 
 int dora_layernorm(const dora_bf16* x, int32_t rows_cap, const int32_t* rows_dev, int32_t dim,
@@ -187,8 +199,85 @@ int dora_linear(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t
                  aligned16(residual));
   if (epilogue == DORA_EPI_BIAS_RESIDUAL) DORA_CHECK_ARG(residual && residual != y);
   DORA_CHECK_DEVICE();
-  return cuda_status(launch_linear(x, m_cap, m_dev, k, w, n, bias, residual, epilogue, y, status,
+  LinearEpi ep;
+  ep.bias = bias;
+  ep.residual = epilogue == DORA_EPI_BIAS_RESIDUAL ? residual : nullptr;
+  return cuda_status(launch_linear(x, m_cap, m_dev, k, w, n, epilogue, ep, y, status,
                                    reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_linear_residual_stats(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
+                               const dora_bf16* w, int32_t n, const dora_bf16* bias,
+                               const dora_bf16* residual, dora_bf16* y, float* stats_out,
+                               int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(m_cap >= 0 && m_cap <= (1 << 30));
+  DORA_CHECK_ARG(k > 0 && k % 64 == 0 && k <= (1 << 16));
+  DORA_CHECK_ARG(n > 0 && n % 64 == 0 && n <= (1 << 16));
+  DORA_CHECK_ARG(w && y && residual && stats_out && residual != y && (m_cap == 0 || x));
+  DORA_CHECK_ARG(aligned16(x) && aligned16(w) && aligned16(y) && aligned16(bias) &&
+                 aligned16(residual) && aligned8(stats_out));
+  DORA_CHECK_DEVICE();
+  LinearEpi ep;
+  ep.bias = bias;
+  ep.residual = residual;
+  ep.stats_out = stats_out;
+  ep.slices = n / kSliceCols;
+  return cuda_status(launch_linear(x, m_cap, m_dev, k, w, n, DORA_EPI_BIAS_RESIDUAL, ep, y, status,
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_row_stats(const dora_bf16* x, int32_t rows_cap, const int32_t* rows_dev, int32_t dim,
+                   float* mv, dora_stream_t stream) {
+  DORA_CHECK_ARG(rows_cap >= 0);
+  DORA_CHECK_ARG(dim > 0 && dim % 8 == 0 && dim <= kMaxDimRow);
+  DORA_CHECK_ARG(rows_cap == 0 || (x && mv));
+  DORA_CHECK_ARG(aligned16(x) && aligned8(mv));
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_row_stats(x, rows_cap, rows_dev, dim, mv,
+                                      reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_merge_moments(const float* sm, int32_t rows_cap, const int32_t* rows_dev,
+                       int32_t slices, float* mv, dora_stream_t stream) {
+  DORA_CHECK_ARG(rows_cap >= 0 && slices > 0 && slices <= (1 << 16) / kSliceCols);
+  DORA_CHECK_ARG(rows_cap == 0 || (sm && mv));
+  DORA_CHECK_ARG(aligned8(sm) && aligned8(mv));
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_merge_moments(sm, rows_cap, rows_dev, slices, mv,
+                                          reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_fold_ln_linear(const dora_bf16* w, int32_t n, int32_t k, const dora_bf16* gamma,
+                        const dora_bf16* beta, const dora_bf16* bias, dora_bf16* w_out,
+                        float* colsum, float* colbias, dora_stream_t stream) {
+  DORA_CHECK_ARG(n >= 0 && n <= (1 << 16) && k > 0 && k % 8 == 0 && k <= (1 << 16));
+  DORA_CHECK_ARG(n == 0 || (w && gamma && beta && w_out && colsum && colbias));
+  DORA_CHECK_ARG(aligned16(w) && aligned16(gamma) && aligned16(beta) && aligned16(w_out) &&
+                 aligned16(colsum) && aligned16(colbias));
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_fold_ln(w, n, k, gamma, beta, bias, w_out, colsum, colbias,
+                                    reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int dora_linear_ln(const dora_bf16* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
+                   const float* mv, float eps, const dora_bf16* w_folded, int32_t n,
+                   const float* colsum, const float* colbias, int32_t gelu, dora_bf16* y,
+                   int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(m_cap >= 0 && m_cap <= (1 << 30));
+  DORA_CHECK_ARG(k > 0 && k % 64 == 0 && k <= kMaxDimRow);
+  DORA_CHECK_ARG(n > 0 && n % 32 == 0 && n <= (1 << 16));
+  DORA_CHECK_ARG(eps >= 0.f && isfinite(eps));
+  DORA_CHECK_ARG(w_folded && y && colsum && colbias && (m_cap == 0 || (x && mv)));
+  DORA_CHECK_ARG(aligned16(x) && aligned16(w_folded) && aligned16(y) && aligned16(colsum) &&
+                 aligned16(colbias) && aligned8(mv));
+  DORA_CHECK_DEVICE();
+  LinearEpi ep;
+  ep.stats_in = mv;
+  ep.colsum = colsum;
+  ep.colbias = colbias;
+  ep.eps = eps;
+  return cuda_status(launch_linear(x, m_cap, m_dev, k, w_folded, n, gelu ? kEpiLnGelu : kEpiLn, ep,
+                                   y, status, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 int dora_varlen_attn(const dora_bf16* qkv, const int32_t* cu_seqlens, int32_t batch,
@@ -221,24 +310,61 @@ int dora_gather_scores(const float* table, int32_t table_stride, const int32_t* 
 // workspace and the pruned block
 // ---------------------------------------------------------------------------
 namespace {
-struct WsLayout {
-  size_t status, xn, qkv, o, hattn, hkeep, kept, u, total;
+size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+// The two linears with a LayerNorm folded in: W' = W diag(gamma) (bf16),
+// c = W' 1 and d = W beta + b (fp32).
+struct FoldLayout {
+  size_t wqkv, cqkv, dqkv, wfc1, cfc1, dfc1, total;
 };
 
-size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+FoldLayout fold_layout(const dora_block_weights* w) {
+  FoldLayout F{};
+  const size_t d = static_cast<size_t>(w->dim), f = static_cast<size_t>(w->mlp_dim);
+  size_t off = 0;
+  F.wqkv = off; off += up256(3 * d * d * 2);
+  F.cqkv = off; off += up256(3 * d * 4);
+  F.dqkv = off; off += up256(3 * d * 4);
+  F.wfc1 = off; off += up256(f * d * 2);
+  F.cfc1 = off; off += up256(f * 4);
+  F.dfc1 = off; off += up256(f * 4);
+  F.total = off;
+  return F;
+}
+
+cudaError_t fold_block(const dora_block_weights* w, uint8_t* fold, cudaStream_t stream) {
+  const FoldLayout F = fold_layout(w);
+  const int d = w->dim;
+  cudaError_t e = launch_fold_ln(w->w_qkv, 3 * d, d, w->ln1_w, w->ln1_b, w->b_qkv,
+                                 reinterpret_cast<uint16_t*>(fold + F.wqkv),
+                                 reinterpret_cast<float*>(fold + F.cqkv),
+                                 reinterpret_cast<float*>(fold + F.dqkv), stream);
+  if (e != cudaSuccess) return e;
+  return launch_fold_ln(w->w_fc1, w->mlp_dim, d, w->ln2_w, w->ln2_b, w->b_fc1,
+                        reinterpret_cast<uint16_t*>(fold + F.wfc1),
+                        reinterpret_cast<float*>(fold + F.cfc1),
+                        reinterpret_cast<float*>(fold + F.dfc1), stream);
+}
+
+struct WsLayout {
+  size_t status, sm, mv, mv2, qkv, o, hattn, hkeep, kept, u, fold, total;
+};
 
 WsLayout ws_layout(int32_t t_cap, const dora_block_weights* w) {
   WsLayout L{};
   const size_t t = static_cast<size_t>(t_cap), d = static_cast<size_t>(w->dim);
   size_t off = 0;
   L.status = off; off += 256;
-  L.xn = off;     off += up256(t * d * 2);
+  L.sm = off;     off += up256(t * (d / kSliceCols) * 8);
+  L.mv = off;     off += up256(t * 8);
+  L.mv2 = off;    off += up256(t * 8);
   L.qkv = off;    off += up256(t * 3 * d * 2);
   L.o = off;      off += up256(t * d * 2);
   L.hattn = off;  off += up256(t * d * 2);
   L.hkeep = off;  off += up256(t * d * 2);
   L.kept = off;   off += up256(t * 4);
   L.u = off;      off += up256(t * static_cast<size_t>(w->mlp_dim) * 2);
+  L.fold = off;   off += w->folded != nullptr ? 0 : fold_layout(w).total;
   L.total = off;
   return L;
 }
@@ -255,9 +381,25 @@ bool weights_ok(const dora_block_weights* w) {
   const void* opt[] = {w->b_qkv, w->b_proj, w->b_fc1, w->b_fc2};
   for (const void* p : opt)
     if (!aligned16(p)) return false;
+  if ((reinterpret_cast<uintptr_t>(w->folded) & 255u) != 0) return false;
   return true;
 }
 }  // namespace
+
+size_t dora_folded_weights_size(const dora_block_weights* w) {
+  if (!w || w->dim <= 0 || w->mlp_dim <= 0) return 0;
+  return fold_layout(w).total;
+}
+
+int dora_fold_block_weights(const dora_block_weights* w, void* folded, size_t folded_bytes,
+                            dora_stream_t stream) {
+  DORA_CHECK_ARG(weights_ok(w) && folded != nullptr);
+  DORA_CHECK_ARG((reinterpret_cast<uintptr_t>(folded) & 255u) == 0);
+  DORA_CHECK_ARG(folded_bytes >= fold_layout(w).total);
+  DORA_CHECK_DEVICE();
+  return cuda_status(fold_block(w, static_cast<uint8_t*>(folded),
+                                reinterpret_cast<cudaStream_t>(stream)));
+}
 
 size_t dora_workspace_size(int32_t t_cap, int32_t batch, const dora_block_weights* w) {
   (void)batch;
@@ -288,7 +430,9 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   int32_t* status = reinterpret_cast<int32_t*>(ws + L.status);
-  uint16_t* xn = reinterpret_cast<uint16_t*>(ws + L.xn);
+  float* sm = reinterpret_cast<float*>(ws + L.sm);
+  float* mv = reinterpret_cast<float*>(ws + L.mv);
+  float* mv2 = reinterpret_cast<float*>(ws + L.mv2);
   uint16_t* qkv = reinterpret_cast<uint16_t*>(ws + L.qkv);
   uint16_t* o = reinterpret_cast<uint16_t*>(ws + L.o);
   uint16_t* hattn = reinterpret_cast<uint16_t*>(ws + L.hattn);
@@ -298,41 +442,59 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
   const int d = w->dim;
   const int32_t* rows_in = cu_in + batch;
 
+  // LayerNorm and LayerNorm' ride in the QKV and fc1 linears (folded weights,
+  // made here unless the caller folded them once with dora_fold_block_weights)
+  uint8_t* fold = ws + L.fold;
+  if (w->folded != nullptr) fold = static_cast<uint8_t*>(const_cast<void*>(w->folded));
+  else if (fold_block(w, fold, stream) != cudaSuccess) return DORA_ERR_CUDA;
+  const FoldLayout F = fold_layout(w);
+  LinearEpi e_qkv, e_proj, e_fc1, e_fc2;
+  e_qkv.stats_in = mv;
+  e_fc1.stats_in = scores ? mv2 : mv;
+  e_qkv.eps = e_fc1.eps = w->ln_eps;
+  e_proj.slices = d / kSliceCols;
+  e_qkv.colsum = reinterpret_cast<const float*>(fold + F.cqkv);
+  e_qkv.colbias = reinterpret_cast<const float*>(fold + F.dqkv);
+  e_fc1.colsum = reinterpret_cast<const float*>(fold + F.cfc1);
+  e_fc1.colbias = reinterpret_cast<const float*>(fold + F.dfc1);
+  e_proj.bias = w->b_proj;
+  e_proj.residual = x_in;
+  e_proj.stats_out = sm;
+  e_fc2.bias = w->b_fc2;
+
   // H_attn = H + Attention(LayerNorm(H))
-  if ((launch_layernorm(x_in, t_cap, rows_in, d, w->ln1_w, w->ln1_b, w->ln_eps, xn, stream)) != cudaSuccess)
+  if (launch_row_stats(x_in, t_cap, rows_in, d, mv, stream) != cudaSuccess) return DORA_ERR_CUDA;
+  if (launch_linear(x_in, t_cap, rows_in, d, reinterpret_cast<const uint16_t*>(fold + F.wqkv),
+                    3 * d, kEpiLn, e_qkv, qkv, status, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
-  if ((launch_linear(xn, t_cap, rows_in, d, w->w_qkv, 3 * d, w->b_qkv, nullptr, DORA_EPI_BIAS,
-                         qkv, status, stream)) != cudaSuccess)
+  if (launch_varlen_attn(qkv, cu_in, batch, max_seqlen, t_cap, w->heads, 0.125f, o, status,
+                         stream) != cudaSuccess)
     return DORA_ERR_CUDA;
-  if ((launch_varlen_attn(qkv, cu_in, batch, max_seqlen, t_cap, w->heads, 0.125f, o, status,
-                              stream)) != cudaSuccess)
+  if (launch_linear(o, t_cap, rows_in, d, w->w_proj, d, DORA_EPI_BIAS_RESIDUAL, e_proj, hattn,
+                    status, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
-  if ((launch_linear(o, t_cap, rows_in, d, w->w_proj, d, w->b_proj, x_in,
-                         DORA_EPI_BIAS_RESIDUAL, hattn, status, stream)) != cudaSuccess)
+  if (launch_merge_moments(sm, t_cap, rows_in, d / kSliceCols, mv, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
-  // H_keep: delete, compact, LayerNorm' in one pass
+  // H_keep: delete and compact, carrying the row moments of LayerNorm'
   const uint16_t* hk = hattn;
   const int32_t* rows_mid = rows_in;
   if (scores) {
-    if ((launch_select_keep(scores, cu_in, keep_counts, batch, max_seqlen, kept, cu_out,
-                                status, stream)) != cudaSuccess)
+    if (launch_select_keep(scores, cu_in, keep_counts, batch, max_seqlen, kept, cu_out, status,
+                           stream) != cudaSuccess)
       return DORA_ERR_CUDA;
-    if ((launch_compact(hattn, d, kept, cu_out, batch, t_cap, ids_in, w->ln2_w, w->ln2_b,
-                            w->ln_eps, hkeep, ids_out, xn, status, stream)) != cudaSuccess)
+    if (launch_compact(hattn, d, kept, cu_out, batch, t_cap, ids_in, nullptr, nullptr, 0.f, hkeep,
+                       ids_out, nullptr, mv, mv2, status, stream) != cudaSuccess)
       return DORA_ERR_CUDA;
     hk = hkeep;
     rows_mid = cu_out + batch;
-  } else {
-    if ((launch_layernorm(hattn, t_cap, rows_in, d, w->ln2_w, w->ln2_b, w->ln_eps, xn,
-                              stream)) != cudaSuccess)
-      return DORA_ERR_CUDA;
   }
   // H_next = H_keep + MLP(LayerNorm'(H_keep))
-  if ((launch_linear(xn, t_cap, rows_mid, d, w->w_fc1, w->mlp_dim, w->b_fc1, nullptr,
-                         DORA_EPI_BIAS_GELU, u, status, stream)) != cudaSuccess)
+  e_fc2.residual = hk;
+  if (launch_linear(hk, t_cap, rows_mid, d, reinterpret_cast<const uint16_t*>(fold + F.wfc1),
+                    w->mlp_dim, kEpiLnGelu, e_fc1, u, status, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
-  if ((launch_linear(u, t_cap, rows_mid, w->mlp_dim, w->w_fc2, d, w->b_fc2, hk,
-                         DORA_EPI_BIAS_RESIDUAL, x_out, status, stream)) != cudaSuccess)
+  if (launch_linear(u, t_cap, rows_mid, w->mlp_dim, w->w_fc2, d, DORA_EPI_BIAS_RESIDUAL, e_fc2,
+                    x_out, status, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
   return DORA_OK;
 }

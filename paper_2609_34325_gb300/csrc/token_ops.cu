@@ -1,5 +1,7 @@
-// Token selection, stream compaction (optionally fused with LayerNorm'),
-// row LayerNorm and the synthetic score gather.  All are bandwidth- or
+// Token selection, stream compaction (optionally fused with LayerNorm', or
+// carrying the row moments of a LayerNorm folded into the next linear), row
+// LayerNorm, row moments and their merge from slice moments, the LayerNorm
+// fold of a linear's weights and the synthetic score gather.  All are bandwidth- or
 // latency-bound integer/copy work: no tensor cores.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -157,15 +159,16 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// K2: compaction (+ LayerNorm'), one warp per output row
+// K2: compaction (+ LayerNorm' or + row moments), one warp per output row
 // ---------------------------------------------------------------------------
-template <bool kLN>
+template <bool kLN, bool kStats>
 __global__ void __launch_bounds__(kRowThreads) compact_kernel(
     const uint4* __restrict__ x, int32_t chunks /* dim / 8 */, const int32_t* __restrict__ kept_idx,
     const int32_t* __restrict__ cu_out, int32_t batch, int32_t t_in_cap,
     const int32_t* __restrict__ ids_in, const uint4* __restrict__ ln_w,
     const uint4* __restrict__ ln_b, float eps, uint4* __restrict__ packed,
-    int32_t* __restrict__ ids_out, uint4* __restrict__ ln_out, int32_t* status) {
+    int32_t* __restrict__ ids_out, uint4* __restrict__ ln_out, const float2* __restrict__ mv_in,
+    float2* __restrict__ mv_out, int32_t* status) {
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
   int t_out = cu_out[batch];
@@ -180,7 +183,10 @@ __global__ void __launch_bounds__(kRowThreads) compact_kernel(
       if (lane == 0) record_status(status, DORA_ERR_DEVICE_SEQLEN);
       continue;
     }
-    if (ids_out != nullptr && lane == 0) ids_out[r] = ids_in[src];
+    if (lane == 0) {
+      if (ids_out != nullptr) ids_out[r] = ids_in[src];
+      if constexpr (kStats) mv_out[r] = mv_in[src];
+    }
     const uint4* srow = x + static_cast<size_t>(src) * chunks;
     uint4* drow = packed + static_cast<size_t>(r) * chunks;
     uint4 v[kMaxChunksPerLane];
@@ -334,6 +340,136 @@ __global__ void __launch_bounds__(kRowThreads) layernorm_kernel(
 }
 
 // ---------------------------------------------------------------------------
+// K6: row moments (mean, biased variance) for a folded LayerNorm, one warp
+// per row (two rows at a time), and their merge from slice moments
+// ---------------------------------------------------------------------------
+template <int CPL>
+__device__ __forceinline__ float2 row_moments(const uint4 (&v)[CPL], int lane, int chunks,
+                                              float inv_dim) {
+  float sum = 0.f;
+#pragma unroll
+  for (int q = 0; q < CPL; ++q) {
+    if (lane + 32 * q < chunks) {
+      const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) sum += bf16_lo(u[e]) + bf16_hi(u[e]);
+    }
+  }
+  const float mean = warp_sumf(sum) * inv_dim;
+  float sq = 0.f;
+#pragma unroll
+  for (int q = 0; q < CPL; ++q) {
+    if (lane + 32 * q < chunks) {
+      const uint32_t* u = reinterpret_cast<const uint32_t*>(&v[q]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a = bf16_lo(u[e]) - mean, c2 = bf16_hi(u[e]) - mean;
+        sq += a * a + c2 * c2;
+      }
+    }
+  }
+  return make_float2(mean, warp_sumf(sq) * inv_dim);
+}
+
+template <int CPL>
+__global__ void __launch_bounds__(kRowThreads) row_stats_kernel(
+    const uint4* __restrict__ x, int32_t rows_cap, const int32_t* __restrict__ rows_dev,
+    int32_t chunks, float2* __restrict__ mv) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  int rows = rows_cap;
+  if (rows_dev != nullptr) rows = min(rows_cap, max(0, *rows_dev));
+  const float inv_dim = 1.0f / static_cast<float>(chunks * 8);
+  for (int r = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < rows; r += 2 * warps) {
+    const int r2 = r + warps;                         // second row of this warp, if any
+    const bool two = r2 < rows;                       // warp-uniform
+    uint4 v[CPL], v2[CPL];
+#pragma unroll
+    for (int q = 0; q < CPL; ++q) {
+      const int c = lane + 32 * q;
+      if (c < chunks) {
+        v[q] = __ldg(x + static_cast<size_t>(r) * chunks + c);
+        if (two) v2[q] = __ldg(x + static_cast<size_t>(r2) * chunks + c);
+      }
+    }
+    const float2 a = row_moments<CPL>(v, lane, chunks, inv_dim);
+    if (lane == 0) mv[r] = a;
+    if (two) {
+      const float2 b = row_moments<CPL>(v2, lane, chunks, inv_dim);
+      if (lane == 0) mv[r2] = b;
+    }
+  }
+}
+
+// One thread per row: mean = (1/S) sum mean_s, M2 = sum (M2_s + 64 (mean_s -
+// mean)^2) over the row's S slices of 64 (the pairwise update of Chan, Golub
+// & LeVeque with equal counts), var = M2 / (64 S).
+__global__ void __launch_bounds__(256) merge_moments_kernel(const float2* __restrict__ sm,
+                                                            int32_t rows_cap,
+                                                            const int32_t* __restrict__ rows_dev,
+                                                            int32_t slices,
+                                                            float2* __restrict__ mv) {
+  int rows = rows_cap;
+  if (rows_dev != nullptr) rows = min(rows_cap, max(0, *rows_dev));
+  const size_t stride = static_cast<size_t>(rows_cap);
+  const float inv_s = 1.0f / static_cast<float>(slices);
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += gridDim.x * blockDim.x) {
+    const float2* p = sm + r;
+    float sum = 0.f;
+    for (int j = 0; j < slices; ++j) sum += p[j * stride].x;
+    const float mean = sum * inv_s;
+    float m2 = 0.f;
+    for (int j = 0; j < slices; ++j) {
+      const float2 t = p[j * stride];
+      const float d = t.x - mean;
+      m2 += t.y + static_cast<float>(kSliceCols) * d * d;
+    }
+    mv[r] = make_float2(mean, m2 * inv_s * (1.0f / kSliceCols));
+  }
+}
+
+// ---------------------------------------------------------------------------
+// K7: LayerNorm affine folded into the next linear, one warp per weight row
+// ---------------------------------------------------------------------------
+// w_out[n, :] = bf16(w[n, :] * gamma) (the product of two bf16 values is
+// exact in fp32, so this is one rounding), colsum[n] = sum of the rounded
+// w_out[n, :] (the values the GEMM multiplies), colbias[n] = w[n, :] . beta
+// + bias[n], both accumulated in fp32.
+__global__ void __launch_bounds__(kRowThreads) fold_ln_kernel(
+    const uint4* __restrict__ w, int32_t n, int32_t chunks, const uint4* __restrict__ gamma,
+    const uint4* __restrict__ beta, const uint16_t* __restrict__ bias, uint4* __restrict__ w_out,
+    float* __restrict__ colsum, float* __restrict__ colbias) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  for (int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < n; row += warps) {
+    float cs = 0.f, cb = 0.f;
+    for (int c = lane; c < chunks; c += 32) {
+      const uint4 wv = __ldg(w + static_cast<size_t>(row) * chunks + c);
+      const uint4 gv = __ldg(gamma + c), bv = __ldg(beta + c);
+      const uint32_t* wu = reinterpret_cast<const uint32_t*>(&wv);
+      const uint32_t* gu = reinterpret_cast<const uint32_t*>(&gv);
+      const uint32_t* bu = reinterpret_cast<const uint32_t*>(&bv);
+      uint4 o;
+      uint32_t* ou = reinterpret_cast<uint32_t*>(&o);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        ou[e] = pack_bf16x2(bf16_lo(wu[e]) * bf16_lo(gu[e]), bf16_hi(wu[e]) * bf16_hi(gu[e]));
+        cs += bf16_lo(ou[e]) + bf16_hi(ou[e]);
+        cb += bf16_lo(wu[e]) * bf16_lo(bu[e]) + bf16_hi(wu[e]) * bf16_hi(bu[e]);
+      }
+      w_out[static_cast<size_t>(row) * chunks + c] = o;
+    }
+    cs = warp_sumf(cs);
+    cb = warp_sumf(cb);
+    if (lane == 0) {
+      colsum[row] = cs;
+      colbias[row] = cb + (bias != nullptr ? __uint_as_float(static_cast<uint32_t>(bias[row]) << 16)
+                                           : 0.f);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // synthetic actor stand-in: row-aligned scores from per-image id tables
 // ---------------------------------------------------------------------------
 __global__ void gather_scores_kernel(const float* __restrict__ table, int32_t stride,
@@ -390,19 +526,29 @@ cudaError_t launch_compact(const uint16_t* x, int32_t dim, const int32_t* kept_i
                            const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
                            const int32_t* ids_in, const uint16_t* ln_w, const uint16_t* ln_b,
                            float eps, uint16_t* packed, int32_t* ids_out, uint16_t* ln_out,
-                           int32_t* status, cudaStream_t stream) {
+                           const float* mv_in, float* mv_out, int32_t* status,
+                           cudaStream_t stream) {
   const int grid = row_grid(t_in_cap);
   const int chunks = dim / 8;
-  if (ln_out != nullptr) {
-    compact_kernel<true><<<grid, kRowThreads, 0, stream>>>(
-        reinterpret_cast<const uint4*>(x), chunks, kept_idx, cu_out, batch, t_in_cap, ids_in,
-        reinterpret_cast<const uint4*>(ln_w), reinterpret_cast<const uint4*>(ln_b), eps,
-        reinterpret_cast<uint4*>(packed), ids_out, reinterpret_cast<uint4*>(ln_out), status);
-  } else {
-    compact_kernel<false><<<grid, kRowThreads, 0, stream>>>(
-        reinterpret_cast<const uint4*>(x), chunks, kept_idx, cu_out, batch, t_in_cap, ids_in,
-        nullptr, nullptr, 0.f, reinterpret_cast<uint4*>(packed), ids_out, nullptr, status);
-  }
+  const uint4* xx = reinterpret_cast<const uint4*>(x);
+  const uint4* ww = reinterpret_cast<const uint4*>(ln_w);
+  const uint4* bb = reinterpret_cast<const uint4*>(ln_b);
+  uint4* pp = reinterpret_cast<uint4*>(packed);
+  uint4* ll = reinterpret_cast<uint4*>(ln_out);
+  const float2* mi = reinterpret_cast<const float2*>(mv_in);
+  float2* mo = reinterpret_cast<float2*>(mv_out);
+  if (ln_out != nullptr)
+    compact_kernel<true, false><<<grid, kRowThreads, 0, stream>>>(
+        xx, chunks, kept_idx, cu_out, batch, t_in_cap, ids_in, ww, bb, eps, pp, ids_out, ll,
+        nullptr, nullptr, status);
+  else if (mv_out != nullptr)
+    compact_kernel<false, true><<<grid, kRowThreads, 0, stream>>>(
+        xx, chunks, kept_idx, cu_out, batch, t_in_cap, ids_in, nullptr, nullptr, 0.f, pp, ids_out,
+        nullptr, mi, mo, status);
+  else
+    compact_kernel<false, false><<<grid, kRowThreads, 0, stream>>>(
+        xx, chunks, kept_idx, cu_out, batch, t_in_cap, ids_in, nullptr, nullptr, 0.f, pp, ids_out,
+        nullptr, nullptr, nullptr, status);
   return cudaGetLastError();
 }
 
@@ -424,6 +570,44 @@ cudaError_t launch_layernorm(const uint16_t* x, int32_t rows_cap, const int32_t*
     case 4: layernorm_kernel<4><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
     default: layernorm_kernel<kMaxChunksPerLane><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_row_stats(const uint16_t* x, int32_t rows_cap, const int32_t* rows_dev,
+                             int32_t dim, float* mv, cudaStream_t stream) {
+  if (rows_cap == 0) return cudaSuccess;
+  const int chunks = dim / 8;
+  const int grid = row_grid((rows_cap + 1) / 2);
+  const uint4* xx = reinterpret_cast<const uint4*>(x);
+  float2* ss = reinterpret_cast<float2*>(mv);
+  switch ((chunks + 31) / 32) {
+    case 1: row_stats_kernel<1><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
+    case 2: row_stats_kernel<2><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
+    case 3: row_stats_kernel<3><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
+    case 4: row_stats_kernel<4><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
+    default: row_stats_kernel<kMaxChunksPerLane><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge_moments(const float* sm, int32_t rows_cap, const int32_t* rows_dev,
+                                 int32_t slices, float* mv, cudaStream_t stream) {
+  if (rows_cap == 0) return cudaSuccess;
+  int64_t g = (static_cast<int64_t>(rows_cap) + 255) / 256;
+  if (g > 152LL * 8) g = 152LL * 8;
+  merge_moments_kernel<<<static_cast<int>(g), 256, 0, stream>>>(
+      reinterpret_cast<const float2*>(sm), rows_cap, rows_dev, slices,
+      reinterpret_cast<float2*>(mv));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fold_ln(const uint16_t* w, int32_t n, int32_t k, const uint16_t* gamma,
+                           const uint16_t* beta, const uint16_t* bias, uint16_t* w_out,
+                           float* colsum, float* colbias, cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  fold_ln_kernel<<<row_grid(n), kRowThreads, 0, stream>>>(
+      reinterpret_cast<const uint4*>(w), n, k / 8, reinterpret_cast<const uint4*>(gamma),
+      reinterpret_cast<const uint4*>(beta), bias, reinterpret_cast<uint4*>(w_out), colsum, colbias);
   return cudaGetLastError();
 }
 

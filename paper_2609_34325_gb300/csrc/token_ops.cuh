@@ -17,11 +17,34 @@ cudaError_t launch_select_keep(const float* scores, const int32_t* cu_in,
                                int32_t* kept_idx, int32_t* cu_out, int32_t* status,
                                cudaStream_t stream);
 
+// ln_out (LayerNorm' of the kept rows) is nullable; so is mv_out, which
+// receives mv_in[kept_idx[r]] (row moments, below) for every packed row r.
 cudaError_t launch_compact(const uint16_t* x, int32_t dim, const int32_t* kept_idx,
                            const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
                            const int32_t* ids_in, const uint16_t* ln_w, const uint16_t* ln_b,
                            float eps, uint16_t* packed, int32_t* ids_out, uint16_t* ln_out,
-                           int32_t* status, cudaStream_t stream);
+                           const float* mv_in, float* mv_out, int32_t* status,
+                           cudaStream_t stream);
+
+// The input side of a LayerNorm folded into the next linear.
+// Row moments: mv[2 r] = mean and mv[2 r + 1] = biased variance of the bf16
+// values of row r.
+// Slice moments (written by the residual GEMM epilogue, where a row is split
+// over several CTAs), slice-major: for row r of a buffer of rows_cap rows and
+// 64-column slice s, sm[2 (s rows_cap + r)] is the slice's mean and
+// sm[2 (s rows_cap + r) + 1] the sum of squared deviations from it.
+constexpr int kSliceCols = 64;
+cudaError_t launch_row_stats(const uint16_t* x, int32_t rows_cap, const int32_t* rows_dev,
+                             int32_t dim, float* mv, cudaStream_t stream);
+// row moments from slice moments (Chan, Golub & LeVeque's pairwise update)
+cudaError_t launch_merge_moments(const float* sm, int32_t rows_cap, const int32_t* rows_dev,
+                                 int32_t slices, float* mv, cudaStream_t stream);
+
+// LayerNorm affine folded into a linear W [n, k]: w_out = bf16(W diag(gamma)),
+// colsum = w_out 1, colbias = W beta + bias (bias nullable).
+cudaError_t launch_fold_ln(const uint16_t* w, int32_t n, int32_t k, const uint16_t* gamma,
+                           const uint16_t* beta, const uint16_t* bias, uint16_t* w_out,
+                           float* colsum, float* colbias, cudaStream_t stream);
 
 cudaError_t launch_layernorm(const uint16_t* x, int32_t rows_cap, const int32_t* rows_dev,
                              int32_t dim, const uint16_t* w, const uint16_t* b, float eps,
@@ -31,11 +54,26 @@ cudaError_t launch_gather_scores(const float* table, int32_t stride, const int32
                                  const int32_t* cu, int32_t batch, float* scores, int32_t* status,
                                  cudaStream_t stream);
 
-// tcgen05 GEMM: y = epi(x w^T + b); tensor maps are built inside.
+// tcgen05 GEMM: y = epi(x w^T ...); tensor maps are built inside.  Besides
+// the public DORA_EPI_* epilogues, two with a LayerNorm folded in:
+//   kEpiLn      y = rstd_r (x w'^T - mean_r colsum) + colbias
+//   kEpiLnGelu  the same, then GELU
+// with rstd_r = 1/sqrt(var_r + eps) from the row moments (stats_in).
+constexpr int kEpiLn = 3;
+constexpr int kEpiLnGelu = 4;
+struct LinearEpi {
+  const uint16_t* bias = nullptr;       // bf16 [n], nullable (plain epilogues)
+  const uint16_t* residual = nullptr;   // bf16 [m, n] (residual epilogue)
+  const float* stats_in = nullptr;      // row moments of x, [m_cap][2] (LN epilogues)
+  const float* colsum = nullptr;        // fp32 [n] (LN epilogues)
+  const float* colbias = nullptr;       // fp32 [n] (LN epilogues)
+  float* stats_out = nullptr;           // slice moments of y, [n/64][m_cap], nullable
+  float eps = 0.f;                      // LayerNorm epsilon (LN epilogues)
+  int32_t slices = 0;                   // n / 64 (stats_out)
+};
 cudaError_t launch_linear(const uint16_t* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
-                          const uint16_t* w, int32_t n, const uint16_t* bias,
-                          const uint16_t* residual, int32_t epilogue, uint16_t* y,
-                          int32_t* status, cudaStream_t stream);
+                          const uint16_t* w, int32_t n, int32_t epilogue, const LinearEpi& ep,
+                          uint16_t* y, int32_t* status, cudaStream_t stream);
 
 // tcgen05 varlen attention.
 cudaError_t launch_varlen_attn(const uint16_t* qkv, const int32_t* cu, int32_t batch,

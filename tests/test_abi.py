@@ -61,19 +61,37 @@ def test_host_validation_without_gpu(lib):
     assert lib.dora_read_status(None, None) == 1
     assert lib.dora_pruned_block(None, None, None, 1, 197, 197, None, None, None, None, None,
                                  None, None, None, 0, None) == 1
+    assert lib.dora_row_stats(16, 4, None, 100, 16, None) == 1           # dim % 8
+    assert lib.dora_row_stats(16, 4, None, 128, 12, None) == 1            # mv alignment
+    assert lib.dora_merge_moments(16, 4, None, 0, 16, None) == 1          # no slices
+    assert lib.dora_compact_stats(16, 64, 16, 16, 1, 10, None, None, 16, None, 16, None,
+                                  None) == 1                              # mv_in missing
+    assert lib.dora_fold_ln_linear(16, 8, 12, 16, 16, None, 16, 16, 16, None) == 1   # k % 8
+    assert lib.dora_linear_ln(16, 128, None, 96, 16, 1e-6, 16, 128, 16, 16, 0, 16, None,
+                              None) == 1                                 # k % 64
+    assert lib.dora_linear_ln(16, 128, None, 128, 16, -1.0, 16, 128, 16, 16, 0, 16, None,
+                              None) == 1                                 # eps < 0
+    assert lib.dora_linear_residual_stats(16, 128, None, 128, 16, 96, None, 32, 16, 16, None,
+                                          None) == 1                     # n % 64
+    assert lib.dora_fold_block_weights(None, 256, 1 << 20, None) == 1
 
 
 def test_block_weights_struct_and_workspace(lib):
-    import torch
-    dims = dict(dim=768, heads=12, mlp_dim=3072)
-    w = P._BlockWeightsC(*([16] * 12), 768, 12, 3072, 1e-6)
-    n = lib.dora_workspace_size(50432, 256, ctypes.byref(w))
+    # per row: slice moments (dim/64 x 8 B), two row moments (8 B each), qkv,
+    # attention output, H_attn, H_keep, kept index, MLP hidden; plus the
+    # folded QKV and fc1 weights
+    # (bf16 W', fp32 c and d) when the caller has not folded them
     t, d, m = 50432, 768, 3072
-    assert n >= t * d * 2 * 7 + t * m * 2 + t * 4
-    assert n < t * d * 2 * 7 + t * m * 2 + t * 4 + 64 * 1024
+    w = P._BlockWeightsC(*([16] * 12), d, 12, m, 1e-6, None)
+    per_rows = t * (d // 64 * 8 + 16 + 3 * d * 2 + 3 * d * 2 + 4 + m * 2)
+    fold = (3 * d + m) * d * 2 + 2 * (3 * d + m) * 4
+    folded_size = lib.dora_folded_weights_size(ctypes.byref(w))
+    assert fold <= folded_size < fold + 8 * 256
+    n = lib.dora_workspace_size(t, 256, ctypes.byref(w))
+    assert per_rows + folded_size <= n < per_rows + folded_size + 16 * 256
+    w.folded = 256
+    assert lib.dora_workspace_size(t, 256, ctypes.byref(w)) == n - folded_size
     assert lib.dora_workspace_size(-1, 1, ctypes.byref(w)) == 0
-    assert dims["dim"] == dims["heads"] * 64
-    del torch
 
 
 def test_python_binding_rejects_cpu_tensors(lib):

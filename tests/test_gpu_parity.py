@@ -292,6 +292,179 @@ def test_linear_no_bias_full_rows():
 
 
 # ---------------------------------------------------------------------------
+# LayerNorm folded into the linear after it
+# ---------------------------------------------------------------------------
+
+def _row_moments_ref(x_bits):
+    """fp64 row moments (mean, biased variance) of bf16 rows."""
+    v = O.bf16_to_f64(x_bits)
+    mean = v.mean(axis=1)
+    return mean, ((v - mean[:, None]) ** 2).mean(axis=1)
+
+
+def _check_row_moments(got, x_bits, what):
+    """got [rows, 2] against fp64: fp32 sums of dim terms, a few roundings of
+    the largest partial sum."""
+    mean, var = _row_moments_ref(x_bits)
+    scale = np.abs(O.bf16_to_f64(x_bits)).max(axis=1)
+    assert np.all(np.abs(got[:, 0] - mean) <= 4e-6 * scale + 1e-30), what
+    assert np.all(np.abs(got[:, 1] - var) <= 1e-5 * var + 1e-6 * scale ** 2 + 1e-30), what
+
+
+def _ln_rows(rng, rows, dim):
+    """Rows with their own offset and spread, as a residual stream has."""
+    off = rng.uniform(-8, 8, (rows, 1))
+    sd = np.exp(rng.uniform(-1.5, 1.5, (rows, 1)))
+    return S.f32_to_bf16_bits(off + sd * rng.standard_normal((rows, dim)))
+
+
+@pytest.mark.parametrize("dim", [64, 192, 768, 1024, 2048])
+def test_row_stats(dim):
+    rng = np.random.default_rng(dim + 1)
+    rows_cap, rows = 1000, 777
+    x = _ln_rows(rng, rows_cap, dim)
+    mv = torch.full((rows_cap, 2), -3.0, dtype=torch.float32, device=dev())
+    P.dora_row_stats(bf(x), mv, rows_dev=i32([rows]))
+    torch.cuda.synchronize()
+    got = mv.cpu().numpy().astype(np.float64)
+    _check_row_moments(got[:rows], x[:rows], f"row_stats d={dim}")
+    assert np.all(got[rows:] == -3.0)
+
+
+@pytest.mark.parametrize("n,k", [(576, 192), (3072, 768), (32, 2048)])
+def test_fold_ln_linear(n, k):
+    rng = np.random.default_rng(n + k)
+    w = S.f32_to_bf16_bits(0.02 * rng.standard_normal((n, k)))
+    g = S.f32_to_bf16_bits(1 + 0.3 * rng.standard_normal(k))
+    be = S.f32_to_bf16_bits(0.1 * rng.standard_normal(k))
+    b = S.f32_to_bf16_bits(0.1 * rng.standard_normal(n))
+    w_out = torch.zeros(n, k, dtype=torch.bfloat16, device=dev())
+    cs = torch.zeros(n, dtype=torch.float32, device=dev())
+    cb = torch.zeros(n, dtype=torch.float32, device=dev())
+    P.dora_fold_ln_linear(bf(w), bf(g), bf(be), w_out, cs, cb, bias=bf(b))
+    torch.cuda.synchronize()
+    wf, gf, bef, bf_ = (O.bf16_to_f64(a) for a in (w, g, be, b))
+    # the product of two bf16 values is exact in fp32: one nearest-even rounding
+    want = S.f32_to_bf16_bits(wf * gf[None, :])
+    assert np.array_equal(bits(w_out), want)
+    c_ref = O.bf16_to_f64(want).sum(axis=1)
+    d_ref = wf @ bef + bf_
+    mag = np.abs(O.bf16_to_f64(want)).sum(axis=1)
+    # fp32 accumulation: k/32 terms per lane, then a 32-lane tree (a dropped
+    # term would be ~1/k of mag)
+    assert np.all(np.abs(cs.cpu().numpy() - c_ref) <= 8e-6 * mag + 1e-7)
+    mag_d = np.abs(wf) @ np.abs(bef) + np.abs(bf_)
+    assert np.all(np.abs(cb.cpu().numpy() - d_ref) <= 8e-6 * mag_d + 1e-7)
+
+
+@pytest.mark.parametrize("name", ["cfg1", "cfg3"])
+def test_compact_stats(name):
+    """Compaction carrying row moments: packed rows bit-exact (as
+    dora_compact) and mv_out[r] = mv_in[kept[r]] bit for bit."""
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    t_in = int(cu[-1])
+    rng = np.random.default_rng(5)
+    x = _ln_rows(rng, t_in, cfg.dim)
+    mv_in = rng.standard_normal((t_in, 2)).astype(np.float32)
+    keeps, _ = S.keep_schedule(cfg, 5)
+    scores = O.gather_scores(S.score_table(cfg, cfg.prune_blocks[0], 5), cu, ids)
+    rk, rcu, _ = O.select_keep(scores, cu, keeps[0])
+    t_out = int(rcu[-1])
+    packed = torch.zeros(t_in, cfg.dim, dtype=torch.bfloat16, device=dev())
+    mv_out = torch.full((t_in, 2), -3.0, dtype=torch.float32, device=dev())
+    ids_out = torch.full((t_in,), SENT, dtype=torch.int32, device=dev())
+    P.dora_compact_stats(bf(x), i32(rk), i32(rcu), packed, f32(mv_in), mv_out, ids_in=i32(ids),
+                         ids_out=ids_out)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits(packed[:t_out]), x[rk])
+    assert np.array_equal(ids_out.cpu().numpy()[:t_out], ids[rk])
+    got = mv_out.cpu().numpy()
+    assert np.array_equal(got[:t_out].view(np.uint32), mv_in[rk].view(np.uint32))
+    assert np.all(got[t_out:] == -3.0)
+
+
+LINEAR_LN_CASES = [
+    # m_cap, m_live, k, n, gelu
+    (300, 300, 64, 128, False),      # one slice, ragged M
+    (1576, 1576, 192, 576, False),   # cfg1 QKV
+    (1576, 1200, 192, 768, True),    # cfg1 fc1 after a deletion
+    (2000, 1999, 768, 2304, False),  # DeiT-B QKV
+    (2000, 1001, 768, 3072, True),   # DeiT-B fc1
+    (777, 640, 1024, 4096, True),
+    (129, 1, 2048, 32, False),
+    (256, 0, 768, 256, True),
+]
+
+
+@pytest.mark.parametrize("m_cap,m_live,k,n,gelu", LINEAR_LN_CASES)
+def test_linear_ln(m_cap, m_live, k, n, gelu):
+    """row moments -> fold -> GEMM with the folded LayerNorm, against the
+    oracle's LayerNorm then linear (then GELU) in fp64."""
+    rng = np.random.default_rng(m_cap + 3 * n + k)
+    eps = 1e-6
+    x = _ln_rows(rng, m_cap, k)
+    g = S.f32_to_bf16_bits(1 + 0.3 * rng.standard_normal(k))
+    be = S.f32_to_bf16_bits(0.2 * rng.standard_normal(k))
+    w = S.f32_to_bf16_bits(0.02 * rng.standard_normal((n, k)))
+    b = S.f32_to_bf16_bits(0.1 * rng.standard_normal(n))
+    mv = torch.zeros(m_cap, 2, dtype=torch.float32, device=dev())
+    w_out = torch.zeros(n, k, dtype=torch.bfloat16, device=dev())
+    cs = torch.zeros(n, dtype=torch.float32, device=dev())
+    cb = torch.zeros(n, dtype=torch.float32, device=dev())
+    y = torch.full((m_cap, n), 7.0, dtype=torch.bfloat16, device=dev())
+    st = _status()
+    m_dev = i32([m_live])
+    P.dora_row_stats(bf(x), mv, rows_dev=m_dev)
+    P.dora_fold_ln_linear(bf(w), bf(g), bf(be), w_out, cs, cb, bias=bf(b))
+    P.dora_linear_ln(bf(x), mv, eps, w_out, cs, cb, y, gelu=gelu, m_dev=m_dev, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    ref = O.linear(O.layernorm(O.bf16_to_f64(x[:m_live]), O.bf16_to_f64(g), O.bf16_to_f64(be),
+                               eps), O.bf16_to_f64(w), O.bf16_to_f64(b))
+    if gelu:
+        ref = O.gelu(ref)
+    assert_close(f64(y[:m_live]), ref, f"linear_ln {m_cap}x{n}x{k} gelu={gelu}")
+    assert torch.all(y[m_live:] == 7.0)
+
+
+@pytest.mark.parametrize("m_cap,m_live,k,n", [(1576, 1200, 768, 192), (2000, 1500, 3072, 768),
+                                              (129, 1, 64, 64), (777, 640, 4096, 1024)])
+def test_linear_residual_stats(m_cap, m_live, k, n):
+    """The residual epilogue's output equals dora_linear's bit for bit; its
+    slice moments match fp64 slice moments of that output, and merged they
+    match the fp64 row moments (and dora_row_stats) within fp32 rounding."""
+    rng = np.random.default_rng(m_cap + n)
+    x = S.f32_to_bf16_bits(rng.standard_normal((m_cap, k)))
+    w = S.f32_to_bf16_bits(0.02 * rng.standard_normal((n, k)))
+    b = S.f32_to_bf16_bits(0.1 * rng.standard_normal(n))
+    r = _ln_rows(rng, m_cap, n)
+    m_dev = i32([m_live])
+    y = torch.full((m_cap, n), 7.0, dtype=torch.bfloat16, device=dev())
+    y2 = torch.full((m_cap, n), 7.0, dtype=torch.bfloat16, device=dev())
+    sm = torch.full((n // 64, m_cap, 2), -3.0, dtype=torch.float32, device=dev())
+    mv = torch.full((m_cap, 2), -3.0, dtype=torch.float32, device=dev())
+    st = _status()
+    P.dora_linear_residual_stats(bf(x), bf(w), bf(r), y, sm, bias=bf(b), m_dev=m_dev, status=st)
+    P.dora_linear(bf(x), bf(w), y2, bias=bf(b), residual=bf(r), epilogue=P.EPI_BIAS_RESIDUAL,
+                  m_dev=m_dev)
+    P.dora_merge_moments(sm, mv, rows_dev=m_dev)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert torch.equal(y, y2)
+    yb = bits(y[:m_live])
+    got = sm.cpu().numpy().astype(np.float64).transpose(1, 0, 2)     # slice-major -> rows
+    assert np.all(got[m_live:] == -3.0)
+    v = O.bf16_to_f64(yb).reshape(m_live, n // 64, 64)
+    s_mean = v.mean(axis=2)
+    s_m2 = ((v - s_mean[..., None]) ** 2).sum(axis=2)
+    s_scale = np.abs(v).max(axis=2)
+    assert np.all(np.abs(got[:m_live, :, 0] - s_mean) <= 4e-6 * s_scale + 1e-30)
+    assert np.all(np.abs(got[:m_live, :, 1] - s_m2) <= 1e-5 * s_m2 + 64e-6 * s_scale ** 2 + 1e-30)
+    _check_row_moments(mv.cpu().numpy().astype(np.float64)[:m_live], yb, "merged moments")
+
+
+# ---------------------------------------------------------------------------
 # varlen attention (tcgen05)
 # ---------------------------------------------------------------------------
 
@@ -451,6 +624,26 @@ def test_block_full_oracle(name):
     assert_close(f64(r0["x_out"][:int(cu[-1])]), ref0["x_out"], f"dense block {name}")
     # pruned rows equal the dense block's rows at the kept positions (Eq. 1)
     assert np.array_equal(bits(r["x_out"][:t_out]), bits(r0["x_out"])[ref["kept_idx"]])
+
+
+def test_block_prefolded_weights_give_the_same_bits():
+    """Weights folded once (dora_fold_block_weights) and weights folded inside
+    every call produce the same block output bit for bit."""
+    cfg = S.get_config("cfg1")
+    cu, ids = S.initial_layout(cfg)
+    x = S.activations_bf16(cfg, 23)
+    wb = S.block_weights(cfg, 1, 23, random_affine=True)
+    keeps, _ = S.keep_schedule(cfg, 23)
+    scores = O.gather_scores(S.score_table(cfg, 1, 23), cu, ids)
+    w = _device_weights(cfg, wb)
+    wf = _device_weights(cfg, wb).fold()
+    assert P.dora_workspace_size(100, 1, wf) < P.dora_workspace_size(100, 1, w)
+    for sc, kp in ((scores, keeps[0]), (None, None)):
+        a = _run_block(cfg, x, cu, ids, w, sc, kp)
+        b = _run_block(cfg, x, cu, ids, wf, sc, kp)
+        assert a["status"] == 0 and b["status"] == 0
+        assert torch.equal(a["x_out"], b["x_out"])
+        assert np.array_equal(a["cu_out"], b["cu_out"])
 
 
 @pytest.mark.parametrize("name", ["cfg3", "cfg4", "cfg5"])
