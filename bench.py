@@ -213,31 +213,37 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
               for _ in range(2)]
     idbufs = [[torch.zeros(t_cap, dtype=torch.int32, device=dev) for _ in range(2)]
               for _ in range(2)]
+    # row moments handed from block to block (x_out_moments -> x_in_moments)
+    mvbufs = [[torch.zeros(t_cap, 2, dtype=torch.float32, device=dev) for _ in range(2)]
+              for _ in range(2)]
     scores = torch.zeros(t_cap, dtype=torch.float32, device=dev)
     kept = torch.zeros(t_cap, dtype=torch.int32, device=dev)
     prune = list(cfg.prune_blocks)
     launches_per_step = {True: 0, False: 0}
 
     def forward(inp, pruned=True, pair=0):
-        xbuf, cubuf, idbuf = xbufs[pair], cubufs[pair], idbufs[pair]
-        x, cu, ids = inp["x"], cu0, ids0
+        xbuf, cubuf, idbuf, mvbuf = xbufs[pair], cubufs[pair], idbufs[pair], mvbufs[pair]
+        x, cu, ids, mv_in = inp["x"], cu0, ids0, None
         n = 0
         for l in range(cfg.depth):
             out = xbuf[l % 2]
+            mv_out = mvbuf[l % 2] if l + 1 < cfg.depth else None
+            # QKV, attention, projection, merge, fc1, fc2 (+ row moments of the
+            # first input, + merge of the output's moments)
+            n += 6 + (mv_in is None) + (mv_out is not None)
             if pruned and l in prune:
                 j = prune.index(l)
                 P.dora_gather_scores(inp["tables"][j], ids, cu, scores, stream=stream)
                 P.dora_pruned_block(x, cu, blocks[l], cfg.n_tokens, out, ws, ids_in=ids,
                                     scores=scores, keep_counts=inp["keeps"][j],
                                     cu_out=cubuf[j % 2], ids_out=idbuf[j % 2], kept_idx=kept,
-                                    stream=stream)
+                                    x_in_moments=mv_in, x_out_moments=mv_out, stream=stream)
                 cu, ids = cubuf[j % 2], idbuf[j % 2]
-                n += 1 + 9
+                n += 3                                   # gather, select, compact
             else:
                 P.dora_pruned_block(x, cu, blocks[l], cfg.n_tokens, out, ws, ids_in=ids,
-                                    stream=stream)
-                n += 7
-            x = out
+                                    x_in_moments=mv_in, x_out_moments=mv_out, stream=stream)
+            x, mv_in = out, mv_out
         launches_per_step[pruned] = n
         return x, cu
 
@@ -421,6 +427,7 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
     sm = torch.zeros(d // 64, t_cap, 2, dtype=f32, device=dev)      # slice moments
     mv = torch.zeros(t_cap, 2, dtype=f32, device=dev)               # row moments
     mv2 = torch.zeros(t_cap, 2, dtype=f32, device=dev)              # after a deletion
+    mvx = [torch.zeros(t_cap, 2, dtype=f32, device=dev) for _ in range(2)]   # between blocks
     # the folded QKV and fc1 weights, as dora_fold_block_weights makes them
     folded = []
     for blk in blocks:
@@ -474,9 +481,12 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
             T, To = int(n_in.sum()), int(n_out.sum())
             rows = cu[B:]
             fl = folded[l]
-            launch("row_stats", lambda: P.dora_row_stats(x, mv, rows_dev=rows, stream=stream),
-                   dict(bytes=2.0 * T * d + 8.0 * T))
-            launch("gemm_qkv", lambda: P.dora_linear_ln(x, mv, cfg.ln_eps, *fl["qkv"], qkv,
+            mvi = mvx[(l + 1) % 2]                   # the previous block's output moments
+            if l == 0:
+                launch("row_stats", lambda: P.dora_row_stats(x, mvi, rows_dev=rows,
+                                                            stream=stream),
+                       dict(bytes=2.0 * T * d + 8.0 * T))
+            launch("gemm_qkv", lambda: P.dora_linear_ln(x, mvi, cfg.ln_eps, *fl["qkv"], qkv,
                                                    m_dev=rows, stream=stream),
                    dict(flops=2.0 * T * 3 * d * d,
                         bytes=2.0 * (T * d + 3 * d * d + 3 * T * d) + 8.0 * T + 24.0 * d))
@@ -516,10 +526,22 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
                                                    gelu=True, m_dev=rows2, stream=stream),
                    dict(flops=2.0 * To * d * m,
                         bytes=2.0 * (To * d + d * m + To * m) + 8.0 * To + 8.0 * m))
-            launch("gemm_fc2", lambda: P.dora_linear(u, w["w_fc2"], out, bias=w["b_fc2"],
-                                                residual=hk, epilogue=P.EPI_BIAS_RESIDUAL,
-                                                m_dev=rows2, stream=stream),
-                   dict(flops=2.0 * To * m * d, bytes=2.0 * (To * m + m * d + 2 * To * d)))
+            if l + 1 < cfg.depth:
+                launch("gemm_fc2",
+                       lambda: P.dora_linear_residual_stats(u, w["w_fc2"], hk, out, sm,
+                                                            bias=w["b_fc2"], m_dev=rows2,
+                                                            stream=stream),
+                       dict(flops=2.0 * To * m * d,
+                            bytes=2.0 * (To * m + m * d + 2 * To * d) + sb * To))
+                launch("merge_moments", lambda: P.dora_merge_moments(sm, mvx[l % 2],
+                                                                    rows_dev=rows2,
+                                                                    stream=stream),
+                       dict(bytes=sb * To + 8.0 * To))
+            else:
+                launch("gemm_fc2", lambda: P.dora_linear(u, w["w_fc2"], out, bias=w["b_fc2"],
+                                                    residual=hk, epilogue=P.EPI_BIAS_RESIDUAL,
+                                                    m_dev=rows2, stream=stream),
+                       dict(flops=2.0 * To * m * d, bytes=2.0 * (To * m + m * d + 2 * To * d)))
             x = out
     torch.cuda.synchronize()
     agg = {}

@@ -69,7 +69,7 @@ enum dora_epilogue {
 /* Human-readable name of a status code (static string). */
 const char* dora_status_string(int code);
 
-/* ABI version, currently 1. */
+/* ABI version, currently 2. */
 int dora_version(void);
 
 /*
@@ -334,6 +334,12 @@ int dora_fold_block_weights(const dora_block_weights* w, void* folded, size_t fo
  * x_out     out bf16 [t_cap, dim]; must not alias x_in.
  * cu_out    out int32 [batch+1]; ids_out out int32 [t_cap];
  * kept_idx  nullable out int32 [t_cap] (workspace is used when NULL).
+ * x_in_moments   nullable fp32 [t_cap, 2]: row moments (mean, var) of x_in's
+ *                live rows, e.g. the previous block's x_out_moments; NULL =
+ *                computed here (one more pass over x_in).
+ * x_out_moments  nullable out fp32 [t_cap, 2]: row moments of x_out's live
+ *                rows, from fc2's residual epilogue, for the next block's
+ *                x_in_moments.  May alias x_in_moments.
  * workspace device buffer of dora_workspace_size() bytes, 256-byte aligned;
  *           it also holds the status word read by dora_read_status.  It must
  *           be zero-filled once after allocation (rows past the live count
@@ -345,8 +351,9 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
                       int32_t batch, int32_t max_seqlen, int32_t t_cap,
                       const dora_block_weights* w, const float* scores,
                       const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
-                      int32_t* ids_out, int32_t* kept_idx, void* workspace,
-                      size_t workspace_bytes, dora_stream_t stream);
+                      int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
+                      float* x_out_moments, void* workspace, size_t workspace_bytes,
+                      dora_stream_t stream);
 
 /* Device address of the status word inside a dora_pruned_block workspace. */
 int32_t* dora_workspace_status(void* workspace);
@@ -389,8 +396,8 @@ int dora_pruned_block_noalloc(const dora_bf16* x_in, const int32_t* cu_in,
                               const int32_t* ids_in, int32_t batch, int32_t max_seqlen,
                               int32_t t_cap, const dora_block_weights* w, const float* scores,
                               const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
-                              int32_t* ids_out, int32_t* kept_idx, int32_t* status,
-                              dora_stream_t stream);
+                              int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
+                              float* x_out_moments, int32_t* status, dora_stream_t stream);
 
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug

@@ -48,10 +48,10 @@ _SIGS = {
     "dora_gather_scores": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _vp, _vp, _vp]),
     "dora_workspace_size": (_sz, [_i32, _i32, _vp]),
     "dora_pruned_block": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp, _vp,
-                                         _vp, _vp, _vp, _vp, _sz, _vp]),
+                                         _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "dora_workspace_status": (_vp, [_vp]),
     "dora_pruned_block_noalloc": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
-                                                 _vp, _vp, _vp, _vp, _vp, _vp]),
+                                                 _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
     "dora_read_status": (ctypes.c_int, [_vp, _vp]),
     "dora_row_stats": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _vp]),
     "dora_fold_ln_linear": (ctypes.c_int, [_vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -398,7 +398,10 @@ def alloc_workspace(t_cap, batch, weights: BlockWeights, device=None) -> torch.T
 
 def dora_pruned_block(x_in, cu_in, weights: BlockWeights, max_seqlen, x_out, workspace,
                       ids_in=None, scores=None, keep_counts=None, cu_out=None, ids_out=None,
-                      kept_idx=None, stream=None):
+                      kept_idx=None, x_in_moments=None, x_out_moments=None, stream=None):
+    """One block of Eq. 1 (dora_pruned_block).  x_in_moments / x_out_moments
+    (fp32 [t_cap, 2], optional) carry the row moments from block to block so
+    that the next block skips its pass over x_in."""
     _req(x_in, torch.bfloat16, "x_in")
     _req(x_out, torch.bfloat16, "x_out")
     _req(cu_in, torch.int32, "cu_in")
@@ -407,17 +410,24 @@ def dora_pruned_block(x_in, cu_in, weights: BlockWeights, max_seqlen, x_out, wor
                  ("ids_out", ids_out), ("kept_idx", kept_idx)):
         _req(t, torch.int32, n, optional=True)
     _req(scores, torch.float32, "scores", optional=True)
+    _req(x_in_moments, torch.float32, "x_in_moments", optional=True)
+    _req(x_out_moments, torch.float32, "x_out_moments", optional=True)
     t_cap = x_in.shape[0]
+    for t in (x_in_moments, x_out_moments):
+        if t is not None and t.numel() < 2 * t_cap:
+            raise ValueError("row moments must hold [t_cap, 2] floats")
     _check(load_library().dora_pruned_block(
         _ptr(x_in), _ptr(cu_in), _ptr(ids_in), cu_in.numel() - 1, int(max_seqlen), t_cap,
         ctypes.byref(weights.c), _ptr(scores), _ptr(keep_counts), _ptr(x_out), _ptr(cu_out),
-        _ptr(ids_out), _ptr(kept_idx), _ptr(workspace), workspace.numel(), _stream(stream)),
+        _ptr(ids_out), _ptr(kept_idx), _ptr(x_in_moments), _ptr(x_out_moments),
+        _ptr(workspace), workspace.numel(), _stream(stream)),
         "dora_pruned_block")
 
 
 def dora_pruned_block_noalloc(x_in, cu_in, weights: BlockWeights, max_seqlen, x_out,
                               ids_in=None, scores=None, keep_counts=None, cu_out=None,
-                              ids_out=None, kept_idx=None, status=None, stream=None):
+                              ids_out=None, kept_idx=None, x_in_moments=None,
+                              x_out_moments=None, status=None, stream=None):
     """dora_pruned_block without a workspace argument, for callers that cannot
     allocate device memory when they run the block: the intermediates live in
     a 32 MiB scratch array the library holds on each GPU.  Blocks needing more
@@ -431,11 +441,14 @@ def dora_pruned_block_noalloc(x_in, cu_in, weights: BlockWeights, max_seqlen, x_
                  ("ids_out", ids_out), ("kept_idx", kept_idx), ("status", status)):
         _req(t, torch.int32, n, optional=True)
     _req(scores, torch.float32, "scores", optional=True)
+    _req(x_in_moments, torch.float32, "x_in_moments", optional=True)
+    _req(x_out_moments, torch.float32, "x_out_moments", optional=True)
     t_cap = x_in.shape[0]
     _check(load_library().dora_pruned_block_noalloc(
         _ptr(x_in), _ptr(cu_in), _ptr(ids_in), cu_in.numel() - 1, int(max_seqlen), t_cap,
         ctypes.byref(weights.c), _ptr(scores), _ptr(keep_counts), _ptr(x_out), _ptr(cu_out),
-        _ptr(ids_out), _ptr(kept_idx), _ptr(status), _stream(stream)),
+        _ptr(ids_out), _ptr(kept_idx), _ptr(x_in_moments), _ptr(x_out_moments), _ptr(status),
+        _stream(stream)),
         "dora_pruned_block_noalloc")
 
 

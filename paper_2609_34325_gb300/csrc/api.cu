@@ -9,6 +9,8 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <stdlib.h>
+
 #include <mutex>
 
 #include "dora.h"
@@ -44,6 +46,11 @@ bool aligned8(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 7u) == 0
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 }  // namespace
+
+bool pdl_enabled() {
+  static const bool on = getenv("DORA_NO_PDL") == nullptr;
+  return on;
+}
 
 int num_sms() {
   int dev = 0;
@@ -113,7 +120,7 @@ const char* dora_status_string(int code) {
   }
 }
 
-int dora_version(void) { return 1; }
+int dora_version(void) { return 2; }
 
 int dora_select_keep(const float* scores, const int32_t* cu_in, const int32_t* keep_counts,
                      int32_t batch, int32_t max_seqlen, int32_t* kept_idx, int32_t* cu_out,
@@ -413,14 +420,16 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
                       int32_t batch, int32_t max_seqlen, int32_t t_cap,
                       const dora_block_weights* w, const float* scores,
                       const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
-                      int32_t* ids_out, int32_t* kept_idx, void* workspace,
-                      size_t workspace_bytes, dora_stream_t stream_) {
+                      int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
+                      float* x_out_moments, void* workspace, size_t workspace_bytes,
+                      dora_stream_t stream_) {
   DORA_CHECK_ARG(weights_ok(w));
   DORA_CHECK_ARG(batch >= 0 && batch <= 65535 && t_cap >= 0 && max_seqlen >= 0);
   DORA_CHECK_ARG(max_seqlen <= kMaxSeqlenSelect);
   DORA_CHECK_ARG(x_in && x_out && cu_in && workspace && x_in != x_out);
   DORA_CHECK_ARG(aligned16(x_in) && aligned16(x_out));
   DORA_CHECK_ARG((reinterpret_cast<uintptr_t>(workspace) & 255u) == 0);
+  DORA_CHECK_ARG(aligned8(x_in_moments) && aligned8(x_out_moments));
   if (scores) DORA_CHECK_ARG(keep_counts && cu_out && ids_in && ids_out);
   const WsLayout L = ws_layout(t_cap, w);
   DORA_CHECK_ARG(workspace_bytes >= L.total);
@@ -449,7 +458,7 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
   else if (fold_block(w, fold, stream) != cudaSuccess) return DORA_ERR_CUDA;
   const FoldLayout F = fold_layout(w);
   LinearEpi e_qkv, e_proj, e_fc1, e_fc2;
-  e_qkv.stats_in = mv;
+  e_qkv.stats_in = x_in_moments ? x_in_moments : mv;
   e_fc1.stats_in = scores ? mv2 : mv;
   e_qkv.eps = e_fc1.eps = w->ln_eps;
   e_proj.slices = d / kSliceCols;
@@ -461,9 +470,13 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
   e_proj.residual = x_in;
   e_proj.stats_out = sm;
   e_fc2.bias = w->b_fc2;
+  e_fc2.stats_out = x_out_moments ? sm : nullptr;   // merged into x_out_moments
+  e_fc2.slices = d / kSliceCols;
 
   // H_attn = H + Attention(LayerNorm(H))
-  if (launch_row_stats(x_in, t_cap, rows_in, d, mv, stream) != cudaSuccess) return DORA_ERR_CUDA;
+  if (x_in_moments == nullptr &&
+      launch_row_stats(x_in, t_cap, rows_in, d, mv, stream) != cudaSuccess)
+    return DORA_ERR_CUDA;
   if (launch_linear(x_in, t_cap, rows_in, d, reinterpret_cast<const uint16_t*>(fold + F.wqkv),
                     3 * d, kEpiLn, e_qkv, qkv, status, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
@@ -495,6 +508,10 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
     return DORA_ERR_CUDA;
   if (launch_linear(u, t_cap, rows_mid, w->mlp_dim, w->w_fc2, d, DORA_EPI_BIAS_RESIDUAL, e_fc2,
                     x_out, status, stream) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  if (x_out_moments != nullptr &&
+      launch_merge_moments(sm, t_cap, rows_mid, d / kSliceCols, x_out_moments, stream) !=
+          cudaSuccess)
     return DORA_ERR_CUDA;
   return DORA_OK;
 }

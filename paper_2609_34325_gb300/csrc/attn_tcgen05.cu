@@ -296,7 +296,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                        int batch, int max_seqlen, int t_cap, int heads, float scale_log2,
                        uint16_t* __restrict__ out, int32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
+  pdl_trigger();
   if (smem_u32(smem_raw) & 1023u) {
+    pdl_wait();
     if (threadIdx.x == 0) record_status(status, DORA_ERR_UNSUPPORTED);
     return;
   }
@@ -305,14 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = threadIdx.x & 31;
   const int dim = heads * HD;
 
-  if (warp == 0) {
-    long long b, e;
-    find_range(cu, batch, heads, t_cap, max_seqlen, status, b, e);
-    if (lane == 0) {
-      s.ih_begin = static_cast<int>(b);
-      s.ih_end = static_cast<int>(e);
-    }
-  } else if (threadIdx.x == 64) {
+  if (threadIdx.x == 64) {
     for (int b = 0; b < 2; ++b) {
       mbar_init(&s.q_full[b], 1);
       mbar_init(&s.q_empty[b], 1);
@@ -344,6 +339,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tm);
   }
   if (warp == 1) tmem_alloc(&s.tmem_base, kTmemCols);
+  // the set-up above overlaps the previous kernel; global memory waits for it
+  pdl_wait();
+  if (warp == 0) {
+    long long b, e;
+    find_range(cu, batch, heads, t_cap, max_seqlen, status, b, e);
+    if (lane == 0) {
+      s.ih_begin = static_cast<int>(b);
+      s.ih_end = static_cast<int>(e);
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -695,9 +700,8 @@ cudaError_t launch_varlen_attn(const uint16_t* qkv, const int32_t* cu, int32_t b
   const long long cap = num_sms();
   const int grid = static_cast<int>(ihs < cap ? ihs : cap);
   const float scale_log2 = scale * 1.4426950408889634f;
-  attn::varlen_attn_kernel<<<grid, attn::kThreads, smem, stream>>>(
-      tm, cu, batch, max_seqlen, t_cap, heads, scale_log2, out, status);
-  return cudaGetLastError();
+  return launch_pdl(attn::varlen_attn_kernel, dim3(grid), dim3(attn::kThreads), smem, stream, tm,
+                    cu, batch, max_seqlen, t_cap, heads, scale_log2, out, status);
 }
 
 }  // namespace dora

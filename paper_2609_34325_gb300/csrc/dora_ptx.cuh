@@ -165,6 +165,17 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// Programmatic dependent launch.  pdl_trigger lets the next kernel on the
+// stream be scheduled while this one runs (it starts as SMs free up);
+// pdl_wait blocks until the previous kernel has finished and its memory is
+// visible.  Every kernel of this library triggers at its start and waits
+// before its first global access that another kernel may have written or may
+// still read.  Without the launch attribute both return at once.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Contiguous copy of `bytes` (a multiple of 16; both addresses 16-byte
 // aligned) from global to this CTA's shared memory, completion signalled on
 // `bar` as transaction bytes.

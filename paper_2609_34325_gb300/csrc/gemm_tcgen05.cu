@@ -226,7 +226,9 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
                 uint16_t* __restrict__ Y, const LinearEpi ep, int m_cap,
                 const int32_t* __restrict__ m_dev, int N, int K, int32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
+  pdl_trigger();
   if (smem_u32(smem_raw) & 1023u) {           // swizzled tiles need 1 KB alignment
+    pdl_wait();
     if (threadIdx.x == 0) record_status(status, DORA_ERR_UNSUPPORTED);
     return;
   }
@@ -238,11 +240,6 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
   constexpr bool kPair = C::kPair;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  int M = m_cap;
-  if (m_dev != nullptr) {
-    const int v = *m_dev;
-    M = v < 0 ? 0 : (v > m_cap ? m_cap : v);
-  }
   // Work is a list of tile pairs: pair p covers M-tiles 2*(p / n_tiles) and
   // 2*(p / n_tiles) + 1 of N-tile p % n_tiles; CTA `rank` of cluster c takes
   // the M-tile 2*(p / n_tiles) + rank of pairs c, c + clusters, ...
@@ -251,8 +248,6 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
   const int cid = blockIdx.x / kCluster;
   const int n_clusters = gridDim.x / kCluster;
   const int n_tiles = (N + BN - 1) / BN;
-  const int m_pairs = (M + 2 * BM - 1) / (2 * BM);
-  const int num_pairs = m_pairs * n_tiles;
   const int kb_count = K / BK;
   constexpr uint32_t kTmemCols = 2 * BN;
   constexpr int kHalfB = BN / 2;
@@ -290,6 +285,15 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
   tc_fence_before();
   cluster_sync();              // peers' barriers are initialised before any multicast
   tc_fence_after();
+  // the set-up above overlaps the previous kernel; global memory waits for it
+  pdl_wait();
+  int M = m_cap;
+  if (m_dev != nullptr) {
+    const int v = *m_dev;
+    M = v < 0 ? 0 : (v > m_cap ? m_cap : v);
+  }
+  const int m_pairs = (M + 2 * BM - 1) / (2 * BM);
+  const int num_pairs = m_pairs * n_tiles;
   const uint32_t tmem = s.tmem_base;
   volatile int* abort = &s.abort_flag;
 
@@ -627,11 +631,13 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = kCluster;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.blockDim = dim3(Cfg<BN, EPI, PAIR>::kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
@@ -653,6 +659,7 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
       static_cast<long>((m_cap + 2 * BM - 1) / (2 * BM)) * ((n + BN - 1) / BN);
   const long clusters = pairs < max_clusters[dev] ? pairs : max_clusters[dev];
   cfg.gridDim = dim3(static_cast<unsigned>(kCluster * clusters));
+  cfg.numAttrs = pdl_enabled() ? 2 : 1;          // dependent launch (the kernel waits)
   return cudaLaunchKernelEx(&cfg, kern, ta, tb, ty, tr, y, ep, m_cap, m_dev, n, k, status);
 }
 

@@ -55,6 +55,7 @@ extern "C" int dora_pruned_block_noalloc(const dora_bf16* x_in, const int32_t* c
                                          const dora_block_weights* w, const float* scores,
                                          const int32_t* keep_counts, dora_bf16* x_out,
                                          int32_t* cu_out, int32_t* ids_out, int32_t* kept_idx,
+                                         const float* x_in_moments, float* x_out_moments,
                                          int32_t* status, dora_stream_t stream) {
   if (w == nullptr || t_cap < 0 || batch < 0) return DORA_ERR_INVALID_ARG;
   const size_t need = dora_workspace_size(t_cap, batch, w);
@@ -67,8 +68,8 @@ extern "C" int dora_pruned_block_noalloc(const dora_bf16* x_in, const int32_t* c
   // (first error wins); the rest is written before it is read.
   if (cudaMemsetAsync(scratch, 0, sizeof(int32_t), s) != cudaSuccess) return DORA_ERR_CUDA;
   const int rc = dora_pruned_block(x_in, cu_in, ids_in, batch, max_seqlen, t_cap, w, scores,
-                                   keep_counts, x_out, cu_out, ids_out, kept_idx, scratch,
-                                   kScratchBytes, stream);
+                                   keep_counts, x_out, cu_out, ids_out, kept_idx, x_in_moments,
+                                   x_out_moments, scratch, kScratchBytes, stream);
   if (rc != DORA_OK) return rc;
   if (status != nullptr &&
       cudaMemcpyAsync(status, dora_workspace_status(scratch), sizeof(int32_t),

@@ -99,6 +99,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
     const float* __restrict__ scores, const int32_t* __restrict__ cu_in,
     const int32_t* __restrict__ keep_counts, int32_t batch, int32_t max_seqlen,
     int32_t* __restrict__ kept_idx, int32_t* __restrict__ cu_out, int32_t* status) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ uint32_t keys[];            // [max_seqlen]
   __shared__ int scratch[33];
   const int i = blockIdx.x;
@@ -169,6 +171,8 @@ __global__ void __launch_bounds__(kRowThreads) compact_kernel(
     const uint4* __restrict__ ln_b, float eps, uint4* __restrict__ packed,
     int32_t* __restrict__ ids_out, uint4* __restrict__ ln_out, const float2* __restrict__ mv_in,
     float2* __restrict__ mv_out, int32_t* status) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
   int t_out = cu_out[batch];
@@ -312,6 +316,8 @@ __global__ void __launch_bounds__(kRowThreads) layernorm_kernel(
     const uint4* __restrict__ x, int32_t rows_cap, const int32_t* __restrict__ rows_dev,
     int32_t chunks, const uint4* __restrict__ w, const uint4* __restrict__ b, float eps,
     uint4* __restrict__ y) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
   int rows = rows_cap;
@@ -375,6 +381,8 @@ template <int CPL>
 __global__ void __launch_bounds__(kRowThreads) row_stats_kernel(
     const uint4* __restrict__ x, int32_t rows_cap, const int32_t* __restrict__ rows_dev,
     int32_t chunks, float2* __restrict__ mv) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
   int rows = rows_cap;
@@ -409,20 +417,41 @@ __global__ void __launch_bounds__(256) merge_moments_kernel(const float2* __rest
                                                             const int32_t* __restrict__ rows_dev,
                                                             int32_t slices,
                                                             float2* __restrict__ mv) {
+  pdl_trigger();
+  pdl_wait();
   int rows = rows_cap;
   if (rows_dev != nullptr) rows = min(rows_cap, max(0, *rows_dev));
   const size_t stride = static_cast<size_t>(rows_cap);
   const float inv_s = 1.0f / static_cast<float>(slices);
+  constexpr int kHeld = 16;     // slices held in registers (dim <= 1024): one round of loads
   for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += gridDim.x * blockDim.x) {
     const float2* p = sm + r;
-    float sum = 0.f;
-    for (int j = 0; j < slices; ++j) sum += p[j * stride].x;
-    const float mean = sum * inv_s;
-    float m2 = 0.f;
-    for (int j = 0; j < slices; ++j) {
-      const float2 t = p[j * stride];
-      const float d = t.x - mean;
-      m2 += t.y + static_cast<float>(kSliceCols) * d * d;
+    float mean, m2 = 0.f;
+    if (slices <= kHeld) {
+      float2 t[kHeld];
+#pragma unroll
+      for (int j = 0; j < kHeld; ++j)
+        if (j < slices) t[j] = __ldg(p + j * stride);
+      float sum = 0.f;
+#pragma unroll
+      for (int j = 0; j < kHeld; ++j)
+        if (j < slices) sum += t[j].x;
+      mean = sum * inv_s;
+#pragma unroll
+      for (int j = 0; j < kHeld; ++j)
+        if (j < slices) {
+          const float d = t[j].x - mean;
+          m2 += t[j].y + static_cast<float>(kSliceCols) * d * d;
+        }
+    } else {
+      float sum = 0.f;
+      for (int j = 0; j < slices; ++j) sum += __ldg(p + j * stride).x;
+      mean = sum * inv_s;
+      for (int j = 0; j < slices; ++j) {
+        const float2 t = __ldg(p + j * stride);
+        const float d = t.x - mean;
+        m2 += t.y + static_cast<float>(kSliceCols) * d * d;
+      }
     }
     mv[r] = make_float2(mean, m2 * inv_s * (1.0f / kSliceCols));
   }
@@ -439,6 +468,8 @@ __global__ void __launch_bounds__(kRowThreads) fold_ln_kernel(
     const uint4* __restrict__ w, int32_t n, int32_t chunks, const uint4* __restrict__ gamma,
     const uint4* __restrict__ beta, const uint16_t* __restrict__ bias, uint4* __restrict__ w_out,
     float* __restrict__ colsum, float* __restrict__ colbias) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
   for (int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < n; row += warps) {
@@ -476,6 +507,8 @@ __global__ void gather_scores_kernel(const float* __restrict__ table, int32_t st
                                      const int32_t* __restrict__ ids,
                                      const int32_t* __restrict__ cu, float* __restrict__ scores,
                                      int32_t* status) {
+  pdl_trigger();
+  pdl_wait();
   const int i = blockIdx.x;
   const int lo = cu[i], hi = cu[i + 1];
   const float* row = table + static_cast<size_t>(i) * stride;
@@ -516,10 +549,8 @@ cudaError_t launch_select_keep(const float* scores, const int32_t* cu_in,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
   }
-  select_keep_kernel<<<batch, kSelectThreads, smem, stream>>>(scores, cu_in, keep_counts, batch,
-                                                              max_seqlen, kept_idx, cu_out,
-                                                              status);
-  return cudaGetLastError();
+  return launch_pdl(select_keep_kernel, dim3(batch), dim3(kSelectThreads), smem, stream, scores,
+                    cu_in, keep_counts, batch, max_seqlen, kept_idx, cu_out, status);
 }
 
 cudaError_t launch_compact(const uint16_t* x, int32_t dim, const int32_t* kept_idx,
@@ -538,18 +569,16 @@ cudaError_t launch_compact(const uint16_t* x, int32_t dim, const int32_t* kept_i
   const float2* mi = reinterpret_cast<const float2*>(mv_in);
   float2* mo = reinterpret_cast<float2*>(mv_out);
   if (ln_out != nullptr)
-    compact_kernel<true, false><<<grid, kRowThreads, 0, stream>>>(
-        xx, chunks, kept_idx, cu_out, batch, t_in_cap, ids_in, ww, bb, eps, pp, ids_out, ll,
+    return launch_pdl(compact_kernel<true, false>, dim3(grid), dim3(kRowThreads), 0, stream,
+                      xx, chunks, kept_idx, cu_out, batch, t_in_cap, ids_in, ww, bb, eps, pp, ids_out, ll,
         nullptr, nullptr, status);
-  else if (mv_out != nullptr)
-    compact_kernel<false, true><<<grid, kRowThreads, 0, stream>>>(
+  if (mv_out != nullptr)
+    return launch_pdl(compact_kernel<false, true>, dim3(grid), dim3(kRowThreads), 0, stream,
         xx, chunks, kept_idx, cu_out, batch, t_in_cap, ids_in, nullptr, nullptr, 0.f, pp, ids_out,
         nullptr, mi, mo, status);
-  else
-    compact_kernel<false, false><<<grid, kRowThreads, 0, stream>>>(
+  return launch_pdl(compact_kernel<false, false>, dim3(grid), dim3(kRowThreads), 0, stream,
         xx, chunks, kept_idx, cu_out, batch, t_in_cap, ids_in, nullptr, nullptr, 0.f, pp, ids_out,
         nullptr, nullptr, nullptr, status);
-  return cudaGetLastError();
 }
 
 cudaError_t launch_layernorm(const uint16_t* x, int32_t rows_cap, const int32_t* rows_dev,
@@ -563,14 +592,15 @@ cudaError_t launch_layernorm(const uint16_t* x, int32_t rows_cap, const int32_t*
   const uint4* bb = reinterpret_cast<const uint4*>(b);
   uint4* yy = reinterpret_cast<uint4*>(y);
   // registers sized to the row: 16-byte chunks per lane
+  cudaError_t e;
   switch ((chunks + 31) / 32) {
-    case 1: layernorm_kernel<1><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
-    case 2: layernorm_kernel<2><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
-    case 3: layernorm_kernel<3><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
-    case 4: layernorm_kernel<4><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
-    default: layernorm_kernel<kMaxChunksPerLane><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    case 1: e = launch_pdl(layernorm_kernel<1>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    case 2: e = launch_pdl(layernorm_kernel<2>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    case 3: e = launch_pdl(layernorm_kernel<3>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    case 4: e = launch_pdl(layernorm_kernel<4>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
+    default: e = launch_pdl(layernorm_kernel<kMaxChunksPerLane>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ww, bb, eps, yy); break;
   }
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t launch_row_stats(const uint16_t* x, int32_t rows_cap, const int32_t* rows_dev,
@@ -580,14 +610,15 @@ cudaError_t launch_row_stats(const uint16_t* x, int32_t rows_cap, const int32_t*
   const int grid = row_grid((rows_cap + 1) / 2);
   const uint4* xx = reinterpret_cast<const uint4*>(x);
   float2* ss = reinterpret_cast<float2*>(mv);
+  cudaError_t e;
   switch ((chunks + 31) / 32) {
-    case 1: row_stats_kernel<1><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
-    case 2: row_stats_kernel<2><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
-    case 3: row_stats_kernel<3><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
-    case 4: row_stats_kernel<4><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
-    default: row_stats_kernel<kMaxChunksPerLane><<<grid, kRowThreads, 0, stream>>>(xx, rows_cap, rows_dev, chunks, ss); break;
+    case 1: e = launch_pdl(row_stats_kernel<1>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ss); break;
+    case 2: e = launch_pdl(row_stats_kernel<2>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ss); break;
+    case 3: e = launch_pdl(row_stats_kernel<3>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ss); break;
+    case 4: e = launch_pdl(row_stats_kernel<4>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ss); break;
+    default: e = launch_pdl(row_stats_kernel<kMaxChunksPerLane>, dim3(grid), dim3(kRowThreads), 0, stream, xx, rows_cap, rows_dev, chunks, ss); break;
   }
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t launch_merge_moments(const float* sm, int32_t rows_cap, const int32_t* rows_dev,
@@ -595,28 +626,27 @@ cudaError_t launch_merge_moments(const float* sm, int32_t rows_cap, const int32_
   if (rows_cap == 0) return cudaSuccess;
   int64_t g = (static_cast<int64_t>(rows_cap) + 255) / 256;
   if (g > 152LL * 8) g = 152LL * 8;
-  merge_moments_kernel<<<static_cast<int>(g), 256, 0, stream>>>(
-      reinterpret_cast<const float2*>(sm), rows_cap, rows_dev, slices,
-      reinterpret_cast<float2*>(mv));
-  return cudaGetLastError();
+  return launch_pdl(merge_moments_kernel, dim3(static_cast<unsigned>(g)), dim3(256), 0, stream,
+                    reinterpret_cast<const float2*>(sm), rows_cap, rows_dev, slices,
+                    reinterpret_cast<float2*>(mv));
 }
 
 cudaError_t launch_fold_ln(const uint16_t* w, int32_t n, int32_t k, const uint16_t* gamma,
                            const uint16_t* beta, const uint16_t* bias, uint16_t* w_out,
                            float* colsum, float* colbias, cudaStream_t stream) {
   if (n == 0) return cudaSuccess;
-  fold_ln_kernel<<<row_grid(n), kRowThreads, 0, stream>>>(
-      reinterpret_cast<const uint4*>(w), n, k / 8, reinterpret_cast<const uint4*>(gamma),
-      reinterpret_cast<const uint4*>(beta), bias, reinterpret_cast<uint4*>(w_out), colsum, colbias);
-  return cudaGetLastError();
+  return launch_pdl(fold_ln_kernel, dim3(row_grid(n)), dim3(kRowThreads), 0, stream,
+                    reinterpret_cast<const uint4*>(w), n, k / 8,
+                    reinterpret_cast<const uint4*>(gamma), reinterpret_cast<const uint4*>(beta),
+                    bias, reinterpret_cast<uint4*>(w_out), colsum, colbias);
 }
 
 cudaError_t launch_gather_scores(const float* table, int32_t stride, const int32_t* ids,
                                  const int32_t* cu, int32_t batch, float* scores, int32_t* status,
                                  cudaStream_t stream) {
   if (batch == 0) return cudaSuccess;
-  gather_scores_kernel<<<batch, 256, 0, stream>>>(table, stride, ids, cu, scores, status);
-  return cudaGetLastError();
+  return launch_pdl(gather_scores_kernel, dim3(batch), dim3(256), 0, stream, table, stride, ids, cu,
+                    scores, status);
 }
 
 }  // namespace dora

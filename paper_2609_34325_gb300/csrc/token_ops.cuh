@@ -6,6 +6,25 @@
 
 namespace dora {
 
+// Launch with programmatic stream serialization (dependent launch; the kernel
+// itself calls pdl_trigger / pdl_wait), unless DORA_NO_PDL is set.
+bool pdl_enabled();
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_enabled() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 constexpr int kSelectThreads = 256;
 constexpr int kRowThreads = 256;          // 8 rows per CTA, one warp per row
 constexpr int kMaxChunksPerLane = 8;      // 16-byte chunks per lane: dim <= 2048

@@ -38,7 +38,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_status_strings(lib):
-    assert P.dora_version() == 1
+    assert P.dora_version() == 2
     assert P.dora_status_string(0) == "ok"
     assert "timed out" in P.dora_status_string(4)
     assert P.dora_status_string(99) == "unknown status"
@@ -60,7 +60,7 @@ def test_host_validation_without_gpu(lib):
     assert lib.dora_gather_scores(16, 0, 16, 16, 1, 16, None, None) == 1
     assert lib.dora_read_status(None, None) == 1
     assert lib.dora_pruned_block(None, None, None, 1, 197, 197, None, None, None, None, None,
-                                 None, None, None, 0, None) == 1
+                                 None, None, None, None, None, 0, None) == 1
     assert lib.dora_row_stats(16, 4, None, 100, 16, None) == 1           # dim % 8
     assert lib.dora_row_stats(16, 4, None, 128, 12, None) == 1            # mv alignment
     assert lib.dora_merge_moments(16, 4, None, 0, 16, None) == 1          # no slices

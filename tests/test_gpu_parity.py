@@ -646,6 +646,47 @@ def test_block_prefolded_weights_give_the_same_bits():
         assert np.array_equal(a["cu_out"], b["cu_out"])
 
 
+def test_block_chained_row_moments():
+    """Two blocks chained through x_out_moments -> x_in_moments: the moments
+    each block hands on match the fp64 row moments of its output, and the
+    second block's output matches the oracle on its input (and the unchained
+    run within rounding)."""
+    cfg = S.get_config("cfg1")
+    cu, ids = S.initial_layout(cfg)
+    t_cap = int(cu[-1])
+    x = S.activations_bf16(cfg, 24)
+    keeps, _ = S.keep_schedule(cfg, 24)
+    wb = [S.block_weights(cfg, l, 24, random_affine=True) for l in range(2)]
+    ws_ = [_device_weights(cfg, w).fold() for w in wb]
+    ws = P.alloc_workspace(t_cap, cfg.batch, ws_[0])
+    scores = O.gather_scores(S.score_table(cfg, 1, 24), cu, ids)
+    x0 = bf(x)
+    mids = [torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev()) for _ in range(2)]
+    outs = [torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev()) for _ in range(2)]
+    m1 = torch.full((t_cap, 2), -3.0, dtype=torch.float32, device=dev())
+    m2 = torch.full((t_cap, 2), -3.0, dtype=torch.float32, device=dev())
+    cu_out = torch.zeros(len(cu), dtype=torch.int32, device=dev())
+    ids_out = torch.zeros(t_cap, dtype=torch.int32, device=dev())
+    for k, chained in enumerate((False, True)):
+        P.dora_pruned_block(x0, i32(cu), ws_[0], cfg.n_tokens, mids[k], ws, ids_in=i32(ids),
+                            x_out_moments=m1 if chained else None)
+        P.dora_pruned_block(mids[k], i32(cu), ws_[1], cfg.n_tokens, outs[k], ws, ids_in=i32(ids),
+                            scores=f32(scores), keep_counts=i32(keeps[0]), cu_out=cu_out,
+                            ids_out=ids_out, x_in_moments=m1 if chained else None,
+                            x_out_moments=m2 if chained else None)
+        torch.cuda.synchronize()
+        assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+    t_out = int(cu_out.cpu().numpy()[-1])
+    _check_row_moments(m1.cpu().numpy().astype(np.float64)[:t_cap], bits(mids[1]), "block 0 out")
+    _check_row_moments(m2.cpu().numpy().astype(np.float64)[:t_out], bits(outs[1][:t_out]),
+                       "block 1 out")
+    assert np.all(m2.cpu().numpy()[t_out:] == -3.0)
+    ref = O.pruned_block(O.bf16_to_f64(bits(mids[1])), cu, ids, O.decode_weights(wb[1]),
+                         cfg.heads, cfg.ln_eps, scores, keeps[0])
+    assert_close(f64(outs[1][:t_out]), ref["x_out"], "chained block")
+    assert_close(f64(outs[1][:t_out]), f64(outs[0][:t_out]), "chained vs unchained")
+
+
 @pytest.mark.parametrize("name", ["cfg3", "cfg4", "cfg5"])
 def test_block_full_size_sampled_images(name):
     cfg = S.get_config(name)

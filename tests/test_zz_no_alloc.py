@@ -95,7 +95,7 @@ def test_noalloc_rejects_blocks_larger_than_its_scratch():
     lib = P.load_library()
     rc = lib.dora_pruned_block_noalloc(x.data_ptr(), cu.data_ptr(), None, cfg.batch,
                                        cfg.n_tokens, t, ctypes.byref(w.c), None, None,
-                                       out.data_ptr(), None, None, None, None,
+                                       out.data_ptr(), None, None, None, None, None, None,
                                        torch.cuda.current_stream().cuda_stream)
     assert rc == 7 and P.dora_status_string(rc).startswith("block needs more scratch")
     torch.cuda.synchronize()
