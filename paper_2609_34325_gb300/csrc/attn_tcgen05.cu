@@ -12,8 +12,8 @@
 //                and publishes a descriptor per step and per unit.  No other
 //                role keeps unit bookkeeping.
 //   warps 1, 2   MMA issuers (one thread each): warp 1 issues S(j) = Q K^T
-//                (M=128, N=keys rounded to 16, K=64) into S/P buffer j mod 2,
-//                once PV(j-2) is done with that buffer; warp 2 issues O (+)= P(j) V
+//                (M=128, N=keys rounded to 16, K=64) into S/P buffer j mod 3,
+//                once PV(j-3) is done with that buffer; warp 2 issues O (+)= P(j) V
 //                with P read from the same buffer, into O buffer (unit mod 2).
 //                A single issuing thread could not keep up with 12 MMAs a step.
 //   warps 4-11   softmax, two threads per query row (TMEM lane), 64 of a step's
@@ -27,8 +27,9 @@
 //                chunk's last 16-key group that lie past the image.
 //   warps 12-15  epilogue: when a unit's last PV is done, O / row sum, staged
 //                through shared memory and stored four whole rows per store.
-// TMEM (512 columns): S/P buffers 0-127 and 128-255, O buffers 256-319 and
-// 320-383.  Rows past the image are computed but never stored; keys past it
+// TMEM (512 columns): S/P buffers 0-127, 128-255 and 256-383 (three, so
+// that the loop softmax(j) -> PV(j) -> S(j+3) spans three steps), O buffers
+// 384-447 and 448-511.  Rows past the image are computed but never stored; keys past it
 // are masked, and V rows past it are zeroed so stale data cannot leak through
 // 0 * NaN.
 #include <cuda.h>
@@ -55,8 +56,15 @@ constexpr int kEpiWarp0 = 12;   // epilogue warps 12-15
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleLog2 = 8.f;    // raise the reference maximum past 2^8
 constexpr uint32_t kSleepNs = 200000;  // waiting threads sleep instead of spinning
+#ifndef ATTN_SP_BUFS
+#define ATTN_SP_BUFS 3
+#endif
+constexpr int kSpBufs = ATTN_SP_BUFS;   // S/P buffers, used by steps in turn
 __device__ __forceinline__ uint32_t tmem_sp(int b) { return 128u * static_cast<uint32_t>(b); }
-__device__ __forceinline__ uint32_t tmem_o(int b) { return 256u + 64u * static_cast<uint32_t>(b); }
+__device__ __forceinline__ uint32_t tmem_o(int b) {
+  return 128u * kSpBufs + 64u * static_cast<uint32_t>(b);
+}
+static_assert(128 * kSpBufs + 2 * 64 <= 512, "TMEM columns");
 
 // Step descriptor (one 32-bit word).
 constexpr uint32_t kDStage = 0x3u;        // K/V stage
@@ -78,15 +86,15 @@ struct Smem {
   uint16_t v[kStages][KC * HD]; // 4 x 16 KB
   uint4 ostage[4][32 * 8];      // per epilogue warp: 32 output rows of 128 bytes
   float lsum[4][2][BQ];         // row sums of each column half, by unit mod 4
-  float mx[2][2][BQ];           // row maxima of each column half, by step parity
+  float mx[kSpBufs][2][BQ];     // row maxima of each column half, by S/P buffer
   uint64_t q_full[2];
   uint64_t q_empty[2];
   uint64_t kv_full[kStages];
   uint64_t kv_empty[kStages];
-  uint64_t s_full[2];           // S of a step in S/P buffer b
-  uint64_t p_full[2];           // P written over it (one arrival per softmax warp)
-  uint64_t xbar[2][4];          // the two halves of a lane quarter exchanged their maxima
-  uint64_t p_free[2];           // PV of buffer b done
+  uint64_t s_full[kSpBufs];     // S of a step in S/P buffer b
+  uint64_t p_full[kSpBufs];     // P written over it (one arrival per softmax warp)
+  uint64_t xbar[kSpBufs][4];    // the two halves of a lane quarter exchanged their maxima
+  uint64_t p_free[kSpBufs];     // PV of buffer b done
   uint64_t o_done[2];           // last PV of a unit in O buffer b done
   uint64_t o_free[2];           // O buffer b read out (one arrival per epilogue warp)
   uint64_t l_full[4];           // row sums of a unit (one arrival per softmax warp)
@@ -311,12 +319,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(&s.q_full[b], 1);
       mbar_init(&s.q_empty[b], 1);
+      mbar_init(&s.o_done[b], 1);
+      mbar_init(&s.o_free[b], 4);
+    }
+    for (int b = 0; b < kSpBufs; ++b) {
       mbar_init(&s.s_full[b], 1);
       mbar_init(&s.p_full[b], 8);
       for (int q = 0; q < 4; ++q) mbar_init(&s.xbar[b][q], 2);
       mbar_init(&s.p_free[b], 1);
-      mbar_init(&s.o_done[b], 1);
-      mbar_init(&s.o_free[b], 4);
     }
     for (int i = 0; i < 4; ++i) mbar_init(&s.l_full[i], 8);
     for (int i = 0; i < kStages; ++i) {
@@ -445,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1 || warp == 2) {
     // ---------------- MMA issuers: warp 1 issues S, warp 2 issues PV (lane 0) ----------------
     // Each reads every step descriptor.  The only order between the two is
-    // explicit: S(j+2) waits until PV(j) has read S/P buffer j mod 2.
+    // explicit: S(j + kSpBufs) waits until PV(j) has read S/P buffer j mod kSpBufs.
     if (lane == 0) {
       for (int j = 0;; ++j) {
         const int i = j % kDescRing;
@@ -455,16 +465,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (d & kDEnd) break;
         const int stg = static_cast<int>(d & kDStage);
         const int up = (d & kDUPar) ? 1 : 0;
-        const int b = j & 1;
+        const int b = j % kSpBufs;
+        const uint32_t bph = static_cast<uint32_t>(j / kSpBufs) & 1u;   // buffer use parity
         if (warp == 1) {
           // S(j) = Q K^T into S/P buffer b
           if ((d & kDFirst) &&
               !mbar_wait_sleep(&s.q_full[up], (d & kDQPar) ? 1u : 0u, abort, kSleepNs))
             break;
           if (!mbar_wait_sleep(&s.kv_full[stg], (d & kDKvPar) ? 1u : 0u, abort, kSleepNs)) break;
-          // the buffer's previous P has been read by its PV (step j - 2)
-          if (j >= 2 && !mbar_wait_sleep(&s.p_free[b], ((j - 2) >> 1) & 1, abort, kSleepNs))
-            break;
+          // the buffer's previous P has been read by its PV (step j - kSpBufs)
+          if (j >= kSpBufs && !mbar_wait_sleep(&s.p_free[b], bph ^ 1u, abort, kSleepNs)) break;
           tc_fence_after();
           const uint64_t qd = sdesc_sw128(smem_u32(s.q[up]), 16, 1024);
           const uint64_t kd = sdesc_sw128(smem_u32(s.k[stg]), 16, 1024);
@@ -483,7 +493,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (first && (d & kDOWait) &&
               !mbar_wait_sleep(&s.o_free[up], (d & kDOPar) ? 1u : 0u, abort, kSleepNs))
             break;
-          if (!mbar_wait_sleep(&s.p_full[b], (j >> 1) & 1, abort, kSleepNs)) break;
+          if (!mbar_wait_sleep(&s.p_full[b], bph, abort, kSleepNs)) break;
           tc_fence_after();
           const int nk = (d_kc(d) + 15) >> 4;
           const uint64_t vd = sdesc_sw128(smem_u32(s.v[stg]), 1024, 1024);
@@ -512,9 +522,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int kc = d_kc(d), kc16 = (kc + 15) & ~15;
       const int kh = min(max(kc - 64 * half, 0), 64);    // keys in this thread's half
       const bool live = quarter * 32 < d_rows(d);        // warp-uniform
-      const int b = j & 1;
+      const int b = j % kSpBufs;
+      const uint32_t bph = static_cast<uint32_t>(j / kSpBufs) & 1u;   // buffer use parity
       const uint32_t tsp = tmem + lane_sel + tmem_sp(b);
-      if (!mbar_wait_warp_sleep(&s.s_full[b], (j >> 1) & 1, abort, kSleepNs)) return false;
+      if (!mbar_wait_warp_sleep(&s.s_full[b], bph, abort, kSleepNs)) return false;
       tc_fence_after();
       // S is done, so the K/V load landed: zero V rows [kc, kc16) (whole 128-byte rows)
       if (kc < kc16) {
@@ -539,7 +550,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       s.mx[b][half][r] = mloc;
       __syncwarp();
       if (lane == 0) mbar_arrive(&s.xbar[b][quarter]);
-      if (!mbar_wait_warp_sleep(&s.xbar[b][quarter], (j >> 1) & 1, abort, kSleepNs)) return false;
+      if (!mbar_wait_warp_sleep(&s.xbar[b][quarter], bph, abort, kSleepNs)) return false;
       const float mc = fmaxf(mloc, s.mx[b][half ^ 1][r]) * scale_log2;
       if (live) {
         // reference maximum: set on a unit's first chunk, raised past 2^8
@@ -569,7 +580,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (rescale) {
           // O holds the chunks before this one once their PV is done: bring this
           // half's 32 columns to the raised reference before this chunk's PV
-          if (!mbar_wait_warp_sleep(&s.p_free[b ^ 1], ((j - 1) >> 1) & 1, abort, kSleepNs))
+          const int pb = (j - 1) % kSpBufs;              // the previous step's buffer
+          if (!mbar_wait_warp_sleep(&s.p_free[pb], static_cast<uint32_t>((j - 1) / kSpBufs) & 1u,
+                                    abort, kSleepNs))
             return false;
           tc_fence_after();
           const uint32_t to = tmem + lane_sel + tmem_o((d & kDUPar) ? 1 : 0) +
