@@ -56,7 +56,7 @@ def parse_args():
     ap.add_argument("--config", default="cfg3")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--input-sets", type=int, default=3)
-    ap.add_argument("--cpu-images", type=int, default=2)
+    ap.add_argument("--cpu-images", type=int, default=20)
     ap.add_argument("--no-extras", action="store_true",
                     help="headline loop only (no dense, e2e, per-kernel or CPU legs)")
     ap.add_argument("--graph", action="store_true", help="replay the step as a CUDA graph")
