@@ -275,15 +275,18 @@ __device__ __forceinline__ float max32(const uint32_t (&a)[32], float m) {
 // place: pair (2k, 2k+1) lands in a[k], whose S value is already consumed.
 __device__ __forceinline__ void exp32_pack(uint32_t (&a)[32], float scale_log2, float neg_m,
                                            float& l) {
-  float l0 = 0.f, l1 = 0.f;
+  const uint64_t sc = f2_pack(scale_log2, scale_log2), nm = f2_pack(neg_m, neg_m);
+  uint64_t acc = f2_pack(0.f, 0.f);
 #pragma unroll
   for (int e = 0; e < 32; e += 2) {
-    const float p0 = ex2_approx(fmaf(__uint_as_float(a[e]), scale_log2, neg_m));
-    const float p1 = ex2_approx(fmaf(__uint_as_float(a[e + 1]), scale_log2, neg_m));
-    l0 += p0;
-    l1 += p1;
+    float x0, x1;
+    f2_unpack(f2_fma(f2_pack(__uint_as_float(a[e]), __uint_as_float(a[e + 1])), sc, nm), x0, x1);
+    const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+    acc = f2_add(acc, f2_pack(p0, p1));
     a[e >> 1] = pack_bf16x2(p0, p1);
   }
+  float l0, l1;
+  f2_unpack(acc, l0, l1);
   l += l0 + l1;
 }
 

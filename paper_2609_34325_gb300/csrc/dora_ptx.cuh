@@ -124,7 +124,7 @@ __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity,
 // spinning, leaving the issue slots to the other warps of its SM sub-partition.
 __device__ __forceinline__ bool mbar_wait_sleep(uint64_t* bar, uint32_t parity,
                                                 volatile int* abort, uint32_t hint_ns) {
-  if (mbar_try_wait(bar, parity)) return true;   // cheaper when already complete
+  if (mbar_test(bar, parity)) return true;   // cheaper when already complete
   const uint64_t t0 = globaltimer_ns();
   while (true) {
     if (mbar_try_wait_hint(bar, parity, hint_ns)) return true;

@@ -646,6 +646,82 @@ def test_block_prefolded_weights_give_the_same_bits():
         assert np.array_equal(a["cu_out"], b["cu_out"])
 
 
+@pytest.mark.parametrize("name,scored", [("cfg1", False), ("cfg1", True), ("cfg2", True)])
+def test_block_equals_its_public_entry_points(name, scored):
+    """The block gives the same bits as its steps run one by one through the
+    public entries: row moments, QKV linear with LayerNorm folded in, varlen
+    attention, projection + residual with slice moments, their merge,
+    [selection, compaction carrying the moments,] fc1 with LayerNorm' folded
+    in + GELU, fc2 + residual with slice moments, their merge.  The block
+    runs twice on one workspace and gives the same bits both times."""
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    t = int(cu[-1])
+    d, m, h = cfg.dim, cfg.mlp_dim, cfg.heads
+    x = S.activations_bf16(cfg, 26)
+    wb = S.block_weights(cfg, 2, 26, random_affine=True)
+    W = {k: bf(v) for k, v in wb.items()}
+    wf = _device_weights(cfg, wb).fold()
+    ws = P.alloc_workspace(t, cfg.batch, wf)
+    keeps, _ = S.keep_schedule(cfg, 26)
+    scores = O.gather_scores(S.score_table(cfg, 0, 26), cu, ids) if scored else None
+    f32t = lambda *shape, v=0.0: torch.full(shape, v, dtype=torch.float32, device=dev())
+    bf16t = lambda *shape: torch.zeros(*shape, dtype=torch.bfloat16, device=dev())
+    xin = bf(x)
+    outs = []
+    for _ in range(2):
+        x_out, mo = bf16t(t, d), f32t(t, 2, v=-3.0)
+        cu_out = torch.zeros(len(cu), dtype=torch.int32, device=dev())
+        ids_out = torch.zeros(t, dtype=torch.int32, device=dev())
+        P.dora_pruned_block(xin, i32(cu), wf, cfg.n_tokens, x_out, ws, ids_in=i32(ids),
+                            scores=None if scores is None else f32(scores),
+                            keep_counts=i32(keeps[0]) if scored else None, cu_out=cu_out,
+                            ids_out=ids_out, x_out_moments=mo)
+        torch.cuda.synchronize()
+        assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+        outs.append((x_out, mo, cu_out))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+
+    def fold(wname, g, b, bias, n):
+        w_, c_, d_ = bf16t(n, d), f32t(n), f32t(n)
+        P.dora_fold_ln_linear(W[wname], W[g], W[b], w_, c_, d_, bias=W[bias])
+        return w_, c_, d_
+    st = _status()
+    rows = i32([t])
+    mv = f32t(t, 2)
+    P.dora_row_stats(xin, mv, rows_dev=rows)
+    qkv = bf16t(t, 3 * d)
+    P.dora_linear_ln(xin, mv, cfg.ln_eps, *fold("w_qkv", "ln1_w", "ln1_b", "b_qkv", 3 * d), qkv,
+                     m_dev=rows, status=st)
+    o = bf16t(t, d)
+    P.dora_varlen_attn(qkv, i32(cu), cfg.n_tokens, h, o, status=st)
+    hattn, sm = bf16t(t, d), f32t(d // 64, t, 2)
+    P.dora_linear_residual_stats(o, W["w_proj"], xin, hattn, sm, bias=W["b_proj"], m_dev=rows,
+                                 status=st)
+    P.dora_merge_moments(sm, mv, rows_dev=rows)
+    hk, mv2, rows2 = hattn, mv, rows
+    if scored:
+        kept = torch.zeros(t, dtype=torch.int32, device=dev())
+        cu2 = torch.zeros(len(cu), dtype=torch.int32, device=dev())
+        P.dora_select_keep(f32(scores), i32(cu), i32(keeps[0]), cfg.n_tokens, kept, cu2, status=st)
+        hk, mv2 = bf16t(t, d), f32t(t, 2)
+        P.dora_compact_stats(hattn, kept, cu2, hk, mv, mv2, ids_in=i32(ids),
+                             ids_out=torch.zeros(t, dtype=torch.int32, device=dev()), status=st)
+        rows2 = cu2[-1:].contiguous()
+    u = bf16t(t, m)
+    P.dora_linear_ln(hk, mv2, cfg.ln_eps, *fold("w_fc1", "ln2_w", "ln2_b", "b_fc1", m), u,
+                     gelu=True, m_dev=rows2, status=st)
+    y, sm2, mo = bf16t(t, d), f32t(d // 64, t, 2), f32t(t, 2, v=-3.0)
+    P.dora_linear_residual_stats(u, W["w_fc2"], hk, y, sm2, bias=W["b_fc2"], m_dev=rows2,
+                                 status=st)
+    P.dora_merge_moments(sm2, mo, rows_dev=rows2)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    t_out = int(rows2.item())
+    assert torch.equal(outs[0][0][:t_out], y[:t_out])
+    assert torch.equal(outs[0][1], mo)
+
+
 def test_block_chained_row_moments():
     """Two blocks chained through x_out_moments -> x_in_moments: the moments
     each block hands on match the fp64 row moments of its output, and the
