@@ -40,7 +40,7 @@ __all__ = [
     "Config", "CONFIGS", "get_config", "splitmix64", "hash_u64", "uniform_f64",
     "uniform_f32", "normal_f64", "f32_to_bf16_bits", "bf16_bits_to_f32",
     "activations_bf16", "block_weights", "score_table", "keep_schedule",
-    "initial_layout", "compression_from_counts",
+    "initial_layout", "compression_from_counts", "actor_weights", "ACTOR_SHAPES",
 ]
 
 _M64 = np.uint64(0xFFFFFFFFFFFFFFFF)
@@ -55,6 +55,7 @@ TAG_SCORE = 3      # + (block << 8)
 TAG_KEEP = 4       # per-image budget law draws
 TAG_BUMP = 5       # cfg5 bump centre / width
 TAG_LNAFF = 6      # optional random LayerNorm affine (tests)
+TAG_ACTOR = 7      # + (which << 8): actor weights
 
 
 def splitmix64(x: np.ndarray) -> np.ndarray:
@@ -321,3 +322,48 @@ def compression_from_counts(cfg: Config, keeps, befores) -> np.ndarray:
             post = sched[l].astype(np.float64) - 1.0
         total += n0 - post
     return total / (L * n0)
+
+
+# ---------------------------------------------------------------------------
+# actor weights (random init): shapes of Appendix A.1, nn.Linear layout
+# ---------------------------------------------------------------------------
+
+def ACTOR_SHAPES(dim: int, depth: int, n0: int) -> dict:
+    """Tensor shapes of the actor's parameters for a backbone of width ``dim``,
+    ``depth`` blocks and ``n0`` visual tokens: budget head outputs
+    M = (n0 - 4) / 2."""
+    m = (n0 - 4) // 2
+    return {
+        "gate_w1": (64, dim + 19), "gate_b1": (64,), "gate_w2": (1, 64), "gate_b2": (1,),
+        "gate_emb": (depth, 16),
+        "enc_w_in": (128, dim), "enc_b_in": (128,), "enc_emb": (depth, 128), "enc_w_h": (128, 3),
+        "enc_ln1_w": (128,), "enc_ln1_b": (128,), "enc_w_qkv": (384, 128), "enc_b_qkv": (384,),
+        "enc_w_o": (128, 128), "enc_b_o": (128,), "enc_ln2_w": (128,), "enc_ln2_b": (128,),
+        "enc_w_fc1": (256, 128), "enc_b_fc1": (256,), "enc_w_fc2": (128, 256),
+        "enc_b_fc2": (128,),
+        "bud_ln_w": (128,), "bud_ln_b": (128,), "bud_w1": (128, 128), "bud_b1": (128,),
+        "bud_w2": (m, 128), "bud_b2": (m,),
+        "sel_w_k": (128,), "sel_w1": (64, 128), "sel_b1": (64,), "sel_w2": (1, 64),
+        "sel_b2": (1,),
+    }
+
+
+def actor_weights(dim: int, depth: int, n0: int, seed: int = 0, gate_bias: float = 0.0) -> dict:
+    """bf16 bit patterns of a randomly initialised actor.  Matrices ~
+    N(0, 1/fan_in), biases and embeddings ~ N(0, 0.1^2), LayerNorm gains
+    1 + N(0, 0.1^2) and shifts N(0, 0.1^2); ``gate_bias`` is added to the
+    gate's output bias (tests use it to keep gate decisions clear of 0.5)."""
+    out = {}
+    for which, (name, shape) in enumerate(ACTOR_SHAPES(dim, depth, n0).items()):
+        count = int(np.prod(shape))
+        tag = TAG_ACTOR + (which << 8)
+        if name.endswith("_emb") or len(shape) == 1 or name in ("gate_b2", "sel_b2"):
+            v = normal_f64(seed, tag, np.arange(count, dtype=np.uint64)) * 0.1
+            if name.endswith("ln1_w") or name.endswith("ln2_w") or name == "bud_ln_w":
+                v = v + 1.0
+            if name == "gate_b2":
+                v = v + gate_bias
+            out[name] = f32_to_bf16_bits(v).reshape(shape)
+        else:
+            out[name] = _normal_bf16(seed, tag, count, 1.0 / np.sqrt(shape[1])).reshape(shape)
+    return out

@@ -22,6 +22,10 @@ block of Eq. 1 (Sec. 3.1), in float64, from bf16/fp32 inputs decoded exactly:
 * ``pruned_block``  Eq. 1: attention over all N_l+1 tokens, residual, delete,
                     LayerNorm', MLP on survivors, residual.
 * ``forward``       Eq. 1 applied block after block.
+* ``actor_gate``, ``actor_encoder``, ``actor_budget``, ``actor_selector``,
+  ``actor_block``   the deterministic actor that produces each block's gate,
+                    removal count and deletion scores (Sec. 3.2 "The actor";
+                    Appendix A.1-A.3).
 
 Readings where the paper is silent (all listed in the design doc):
 
@@ -32,6 +36,10 @@ Readings where the paper is silent (all listed in the design doc):
   is reported.
 * LayerNorm uses the biased variance; GELU is the exact erf form; the qkv row
   layout is [3][H][head_dim]; the default softmax scale is 1/sqrt(head_dim).
+* Actor: LayerNorm epsilon 1e-5; W_k and W_h carry no bias; budget ties go to
+  the smaller removal count; the encoder's attention scale is 1/sqrt(32);
+  every image gets a budget and selector scores (the gate only decides
+  whether they are used); E_<l / (L - 1) divides by 1 when L = 1.
 
 Parity pins: every function here is checked in ``tests/test_oracle_pins.py``
 against brute force, closed forms, invariants the paper fixes, or an
@@ -320,3 +328,131 @@ def forward(x: np.ndarray, cu: np.ndarray, ids: np.ndarray, blocks: list, heads:
         x, cu, ids = r["x_out"], r["cu_out"], r["ids_out"]
         kept_hist.append(r["kept_idx"])
     return dict(x=x, cu=cu, ids=ids, kept=kept_hist)
+
+
+# ----------------------------------------------------------------------------
+# O6: the deployment actor (Sec. 3.2 "The actor"; Appendix A.1-A.3)
+# ----------------------------------------------------------------------------
+# Widths fixed by Appendix A.1.
+ACTOR_WIDTH = 128          # shared encoder width (four heads of 32)
+ACTOR_HEADS = 4
+ACTOR_FF = 256             # encoder feed-forward 128 -> 256 -> 128
+ACTOR_GATE_HIDDEN = 64     # gate (d + 19) -> 64 -> 1
+ACTOR_GATE_EMB = 16        # gate block embedding
+ACTOR_SEL_HIDDEN = 64      # selector 128 -> 64 -> 1
+ACTOR_EPS = 1e-5           # the actor's LayerNorm epsilon (paper silent: PyTorch default)
+
+
+def sigmoid(x):
+    """Logistic function, written through tanh so that it never overflows:
+    1 / (1 + e^-x) = (1 + tanh(x / 2)) / 2."""
+    return 0.5 * (1.0 + np.tanh(0.5 * np.asarray(x, dtype=np.float64)))
+
+
+def silu(x):
+    """SiLU, x * sigmoid(x)."""
+    x = np.asarray(x, dtype=np.float64)
+    return x * sigmoid(x)
+
+
+def budget_grid(n0: int) -> np.ndarray:
+    """Candidate removal counts B = {2, 4, ..., N0 - 4} (Appendix A.2)."""
+    return np.arange(2, n0 - 4 + 1, 2, dtype=np.int64)
+
+
+def actor_history(n_l: int, n0: int, rho: float, interventions: int, depth: int) -> np.ndarray:
+    """h_l = [N_l / N0, rho_l, E_<l / (L - 1)] (Appendix A.1, history vector);
+    for a single-block model (L = 1) the last entry divides by 1."""
+    return np.array([n_l / n0, rho, interventions / max(depth - 1, 1)], dtype=np.float64)
+
+
+def actor_gate(k_cls: np.ndarray, e_gate: np.ndarray, h: np.ndarray, w: dict) -> float:
+    """p^G = sigmoid(MLP([K_CLS, e^G_l, h_l])): a (d + 19) -> 64 -> 1 MLP with
+    a SiLU hidden layer (Appendix A.1, gate)."""
+    z = np.concatenate([np.asarray(k_cls, np.float64), e_gate, h])
+    hid = silu(w["gate_w1"] @ z + w["gate_b1"])
+    return float(sigmoid(w["gate_w2"][0] @ hid + w["gate_b2"][0]))
+
+
+def actor_encoder(keys: np.ndarray, e_enc: np.ndarray, h: np.ndarray, w: dict,
+                  eps: float = ACTOR_EPS) -> np.ndarray:
+    """Z_l for one image (Appendix A.1, shared encoder).  ``keys`` [N_l + 1, d]
+    with row 0 the CLS key.  X_j = W_in K_j + b_in + e^C_l, plus W_h h_l on CLS
+    only; then one pre-LayerNorm Transformer block of width 128 with four
+    attention heads and a 128 -> 256 -> 128 GELU feed-forward sublayer."""
+    x = linear(keys, w["enc_w_in"], w["enc_b_in"]) + e_enc
+    x[0] += w["enc_w_h"] @ h
+    n = x.shape[0]
+    qkv = linear(layernorm(x, w["enc_ln1_w"], w["enc_ln1_b"], eps), w["enc_w_qkv"],
+                 w["enc_b_qkv"])
+    o = varlen_attention(qkv, np.array([0, n]), ACTOR_HEADS, ACTOR_WIDTH // ACTOR_HEADS)
+    z1 = x + linear(o, w["enc_w_o"], w["enc_b_o"])
+    f = linear(layernorm(z1, w["enc_ln2_w"], w["enc_ln2_b"], eps), w["enc_w_fc1"],
+               w["enc_b_fc1"])
+    return z1 + linear(gelu(f), w["enc_w_fc2"], w["enc_b_fc2"])
+
+
+def actor_budget(z_cls: np.ndarray, n_l: int, n0: int, w: dict, eps: float = ACTOR_EPS):
+    """Deployment budget (Sec. 3.2; Appendix A.3): LayerNorm(Z_CLS) then a
+    128 -> 128 -> M GELU MLP gives one logit per grid entry; budgets that would
+    leave fewer than four visual tokens (k > N_l - 4) are masked; the highest
+    remaining logit wins (ties: the smaller budget).  Returns (k, logits);
+    k = 0 when no budget is feasible."""
+    u = layernorm(np.asarray(z_cls, np.float64)[None], w["bud_ln_w"], w["bud_ln_b"], eps)[0]
+    logits = w["bud_w2"] @ gelu(w["bud_w1"] @ u + w["bud_b1"]) + w["bud_b2"]
+    grid = budget_grid(n0)
+    feasible = grid <= n_l - 4
+    if not feasible.any():
+        return 0, logits
+    masked = np.where(feasible, logits, -np.inf)
+    return int(grid[int(np.argmax(masked))]), logits
+
+
+def actor_selector(z_vis: np.ndarray, k: int, n_l: int, w: dict) -> np.ndarray:
+    """Eq. 2: s_j = MLP_S(Z_j + W_k k / N_l), a shared 128 -> 64 -> 1 SiLU MLP
+    over the visual tokens; higher means remove first."""
+    u = np.asarray(z_vis, np.float64) + w["sel_w_k"] * (k / n_l)
+    return silu(u @ w["sel_w1"].T + w["sel_b1"]) @ w["sel_w2"][0] + w["sel_b2"][0]
+
+
+def actor_block(keys: np.ndarray, cu: np.ndarray, block: int, n0: int, depth: int,
+                rho: np.ndarray, interventions: np.ndarray, w: dict,
+                eps: float = ACTOR_EPS) -> dict:
+    """The deterministic actor at one block for every image of a packed batch
+    (Sec. 3.2 "Sampling and deployment"; Appendix A.3).
+
+    ``keys`` [T, d] are the block's keys (heads concatenated), row-aligned with
+    the packed tokens; ``rho`` and ``interventions`` hold each image's rho_l
+    and E_<l.  Every image gets a gate probability, a budget (argmax over its
+    feasible grid) and selector scores computed with that budget; the gate
+    opens when p >= 0.5 and a budget is feasible, and then k_l = the budget,
+    otherwise k_l = 0.  Returns p, gate, budget, k, keep_counts (N_l + 1 - k_l,
+    CLS included), scores [T] (CLS rows 0), z [T, 128], logits [B, M], and the
+    next block's rho and interventions."""
+    keys = bf16_to_f64(keys) if np.asarray(keys).dtype == np.uint16 else np.asarray(keys,
+                                                                                   np.float64)
+    cu = np.asarray(cu, dtype=np.int64)
+    b = len(cu) - 1
+    p = np.zeros(b)
+    gate = np.zeros(b, dtype=np.int32)
+    budget = np.zeros(b, dtype=np.int32)
+    k = np.zeros(b, dtype=np.int32)
+    scores = np.zeros(int(cu[-1]))
+    z = np.zeros((int(cu[-1]), ACTOR_WIDTH))
+    logits = np.zeros((b, len(budget_grid(n0))))
+    for i in range(b):
+        lo, hi = int(cu[i]), int(cu[i + 1])
+        n_l = hi - lo - 1
+        h = actor_history(n_l, n0, float(rho[i]), int(interventions[i]), depth)
+        p[i] = actor_gate(keys[lo], w["gate_emb"][block], h, w)
+        zi = actor_encoder(keys[lo:hi], w["enc_emb"][block], h, w, eps)
+        z[lo:hi] = zi
+        budget[i], logits[i] = actor_budget(zi[0], n_l, n0, w, eps)
+        scores[lo + 1:hi] = actor_selector(zi[1:], int(budget[i]), n_l, w)
+        gate[i] = int(p[i] >= 0.5 and budget[i] > 0)
+        k[i] = budget[i] if gate[i] else 0
+    n_vis = np.diff(cu) - 1
+    return dict(p=p, gate=gate, budget=budget, k=k, keep_counts=(n_vis + 1 - k).astype(np.int32),
+                scores=scores, z=z, logits=logits,
+                rho_next=np.where(gate == 1, k / np.maximum(n_vis, 1), 0.0),
+                interventions_next=np.asarray(interventions) + gate)

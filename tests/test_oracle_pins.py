@@ -410,3 +410,161 @@ def test_compression_identity_and_calibration():
         c = S.compression_from_counts(cfg, *S.keep_schedule(cfg, seed))
         assert abs(c.mean() - 0.38) <= 0.01
         assert c.min() < 0.30 and c.max() > 0.45          # per-image spread
+
+
+# ---------------------------------------------------------------------------
+# the deployment actor (Sec. 3.2 "The actor"; Appendix A.1-A.3)
+# ---------------------------------------------------------------------------
+
+def _actor_w(d=64, depth=4, n0=20, seed=3, **kw):
+    return {k: O.bf16_to_f64(v) for k, v in S.actor_weights(d, depth, n0, seed, **kw).items()}
+
+
+def test_actor_sigmoid_and_silu_closed_forms():
+    assert O.sigmoid(0.0) == 0.5
+    for x in (-40.0, -2.5, -1e-3, 0.7, 4.0, 40.0):
+        ref = 1.0 / (1.0 + math.exp(-x))
+        assert abs(O.sigmoid(x) - ref) <= 1e-15 + 1e-14 * ref
+        assert abs(O.silu(x) - x * ref) <= 1e-14 * (1 + abs(x))
+
+
+def test_actor_gate_closed_forms():
+    """p = 0.5 exactly with a zero output layer; one-hot first layers read the
+    block embedding and the history at the positions Appendix A.1 gives them
+    ([K_CLS (d), e^G (16), h (3)])."""
+    d = 64
+    w = _actor_w(d)
+    k_cls = np.linspace(-1, 1, d)
+    e_g = w["gate_emb"][2]
+    h = O.actor_history(10, 20, 0.25, 2, 4)
+    assert np.allclose(h, [0.5, 0.25, 2 / 3], rtol=0, atol=1e-15)
+    w0 = dict(w, gate_w2=np.zeros((1, 64)), gate_b2=np.zeros(1))
+    assert O.actor_gate(k_cls, e_g, h, w0) == 0.5
+    for col, val in ((d, e_g[0]), (d + 15, e_g[15]), (d + 16, h[0]), (d + 18, h[2]), (3, k_cls[3])):
+        w1 = np.zeros((64, d + 19))
+        w1[0, col] = 1.0
+        wv = dict(w, gate_w1=w1, gate_b1=np.zeros(64), gate_w2=np.eye(1, 64), gate_b2=np.array([0.5]))
+        silu_v = val / (1 + math.exp(-val))
+        assert abs(O.actor_gate(k_cls, e_g, h, wv) - 1 / (1 + math.exp(-(silu_v + 0.5)))) < 1e-14
+
+
+def test_actor_encoder_reduces_to_its_input_projection():
+    """With the attention output and feed-forward output layers zeroed the
+    block is the identity, so Z = W_in K + b_in + e^C (+ W_h h on CLS),
+    summed out element by element."""
+    d, n = 64, 7
+    w = _actor_w(d)
+    for nm in ("enc_w_o", "enc_b_o", "enc_w_fc2", "enc_b_fc2"):
+        w[nm] = np.zeros_like(w[nm])
+    rng = np.random.default_rng(1)
+    keys = rng.standard_normal((n + 1, d))
+    h = np.array([0.3, 0.1, 0.5])
+    e_c = w["enc_emb"][1]
+    z = O.actor_encoder(keys, e_c, h, w)
+    for j in range(n + 1):
+        for c in (0, 17, 127):
+            ref = sum(w["enc_w_in"][c, t] * keys[j, t] for t in range(d)) + w["enc_b_in"][c] + e_c[c]
+            if j == 0:
+                ref += sum(w["enc_w_h"][c, t] * h[t] for t in range(3))
+            assert abs(z[j, c] - ref) < 1e-12
+
+
+def test_actor_encoder_is_permutation_equivariant_over_visual_tokens():
+    """No positional term enters the encoder (Appendix A.1): permuting the
+    visual tokens permutes their outputs and leaves Z_CLS unchanged."""
+    d, n = 64, 9
+    w = _actor_w(d)
+    rng = np.random.default_rng(2)
+    keys = rng.standard_normal((n + 1, d))
+    h = np.array([0.9, 0.2, 0.0])
+    perm = np.concatenate([[0], 1 + rng.permutation(n)])
+    z = O.actor_encoder(keys, w["enc_emb"][0], h, w)
+    zp = O.actor_encoder(keys[perm], w["enc_emb"][0], h, w)
+    assert np.allclose(zp, z[perm], rtol=0, atol=1e-12)
+
+
+def test_actor_encoder_equal_keys_average_the_values():
+    """Equal attention keys (key weights zero) make every head average its
+    values uniformly: Z1 = X + W_o mean_j(V_j) + b_o for every token."""
+    d, n = 64, 6
+    w = _actor_w(d)
+    w["enc_w_qkv"] = w["enc_w_qkv"].copy()
+    w["enc_w_qkv"][128:256] = 0.0
+    for nm in ("enc_w_fc2", "enc_b_fc2"):
+        w[nm] = np.zeros_like(w[nm])
+    rng = np.random.default_rng(4)
+    keys = rng.standard_normal((n + 1, d))
+    h = np.array([0.5, 0.0, 0.0])
+    e_c = w["enc_emb"][3]
+    x = keys @ w["enc_w_in"].T + w["enc_b_in"] + e_c
+    x[0] += w["enc_w_h"] @ h
+    mu = x.mean(axis=1, keepdims=True)
+    xn = (x - mu) / np.sqrt(((x - mu) ** 2).mean(axis=1, keepdims=True) + O.ACTOR_EPS)
+    xn = xn * w["enc_ln1_w"] + w["enc_ln1_b"]
+    v = xn @ w["enc_w_qkv"][256:].T + w["enc_b_qkv"][256:]
+    ref = x + (w["enc_w_o"] @ v.mean(axis=0) + w["enc_b_o"])[None, :]
+    assert np.allclose(O.actor_encoder(keys, e_c, h, w), ref, rtol=0, atol=1e-12)
+
+
+def test_actor_budget_masked_argmax_brute_force():
+    """Appendix A.2/A.3: the highest logit among budgets k <= N_l - 4 (at least
+    four visual tokens survive), none when N_l < 6; equal logits pick the
+    smallest budget."""
+    n0 = 196
+    w = _actor_w(64, n0=n0)
+    grid = list(range(2, n0 - 4 + 1, 2))
+    rng = np.random.default_rng(5)
+    for n_l in (3, 5, 6, 7, 10, 33, 100, 196):
+        z = rng.standard_normal(128)
+        k, logits = O.actor_budget(z, n_l, n0, w)
+        best = None
+        for idx, kk in enumerate(grid):
+            if kk <= n_l - 4 and (best is None or logits[idx] > logits[best]):
+                best = idx
+        assert k == (0 if best is None else grid[best])
+        assert k == 0 or n_l - k >= 4
+    wt = dict(w, bud_w2=np.zeros_like(w["bud_w2"]), bud_b2=np.full(len(grid), 0.3))
+    assert O.actor_budget(rng.standard_normal(128), 50, n0, wt)[0] == 2
+
+
+def test_actor_selector_closed_form():
+    """Eq. 2 with a one-hot first layer: s_j = silu(Z_j[0] + 2 k / N_l) + 0.25."""
+    w = _actor_w(64)
+    w1 = np.zeros((64, 128))
+    w1[0, 0] = 1.0
+    wk = np.zeros(128)
+    wk[0] = 2.0
+    ws = dict(w, sel_w1=w1, sel_b1=np.zeros(64), sel_w2=np.eye(1, 64), sel_b2=np.array([0.25]),
+              sel_w_k=wk)
+    rng = np.random.default_rng(6)
+    z = rng.standard_normal((5, 128))
+    s = O.actor_selector(z, 8, 40, ws)
+    for j in range(5):
+        a = z[j, 0] + 2 * 8 / 40
+        assert abs(s[j] - (a / (1 + math.exp(-a)) + 0.25)) < 1e-14
+
+
+def test_actor_block_decisions_and_history():
+    """Deployment rules (Appendix A.3): the gate opens when p >= 0.5 and a
+    budget is feasible; k_l = the budget then, 0 otherwise; keep = N_l + 1 -
+    k_l; rho_{l+1} = k_l / N_l and E counts the interventions."""
+    d, n0, depth = 64, 20, 4
+    lens = np.array([21, 5, 9, 13, 21])             # N_l + 1 tokens; 5 -> N_l = 4: no budget
+    cu = O.cu_from_counts(lens)
+    rng = np.random.default_rng(7)
+    keys = rng.standard_normal((int(cu[-1]), d))
+    rho = np.array([0.0, 0.1, 0.2, 0.0, 0.3])
+    e_prev = np.array([0, 1, 2, 0, 1])
+    for gb, want in ((9.0, 1), (-9.0, 0)):
+        w = _actor_w(d, depth, n0, gate_bias=gb)
+        r = O.actor_block(keys, cu, 2, n0, depth, rho, e_prev, w)
+        n_vis = lens - 1
+        feasible = n_vis >= 6
+        assert np.array_equal(r["gate"], (want * feasible).astype(np.int32))
+        assert np.array_equal(r["gate"], ((r["p"] >= 0.5) & (r["budget"] > 0)).astype(np.int32))
+        assert np.array_equal(r["k"], r["budget"] * r["gate"])
+        assert np.array_equal(r["keep_counts"], lens - r["k"])
+        assert np.all((r["k"] == 0) | (r["keep_counts"] - 1 >= 4))
+        assert np.allclose(r["rho_next"], r["k"] / n_vis)
+        assert np.array_equal(r["interventions_next"], e_prev + r["gate"])
+        assert np.all(r["scores"][cu[:-1]] == 0.0)
