@@ -399,6 +399,85 @@ int dora_pruned_block_noalloc(const dora_bf16* x_in, const int32_t* cu_in,
                               int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
                               float* x_out_moments, int32_t* status, dora_stream_t stream);
 
+/*
+ * The deterministic actor (Sec. 3.2 "The actor"; Appendix A.1-A.3): at a
+ * block it reads the block's keys and produces, for every image, the gate
+ * decision, the removal count k_l and the deletion scores that
+ * dora_select_keep consumes.
+ *
+ * dora_actor_weights -- bf16 device tensors of the actor, nn.Linear layout
+ * [out, in], the shapes of Appendix A.1 (d = backbone width, L = depth,
+ * M = (n0 - 4) / 2 budget-head outputs):
+ *   gate: gate_w1 [64, d + 19], gate_b1 [64], gate_w2 [1, 64], gate_b2 [1],
+ *         gate_emb [L, 16]  -- input order [K_CLS, e^G_l, h_l];
+ *   encoder: enc_w_in [128, d], enc_b_in [128], enc_emb [L, 128],
+ *         enc_w_h [128, 3], enc_ln1_w/b [128], enc_w_qkv [384, 128] (rows
+ *         q, k, v, each four heads of 32), enc_b_qkv [384], enc_w_o [128, 128],
+ *         enc_b_o [128], enc_ln2_w/b [128], enc_w_fc1 [256, 128],
+ *         enc_b_fc1 [256], enc_w_fc2 [128, 256], enc_b_fc2 [128];
+ *   budget head: bud_ln_w/b [128], bud_w1 [128, 128], bud_b1 [128],
+ *         bud_w2 [M, 128], bud_b2 [M];
+ *   selector: sel_w_k [128], sel_w1 [64, 128], sel_b1 [64], sel_w2 [1, 64],
+ *         sel_b2 [1].
+ * dim % 64 == 0, dim <= 2048; 6 <= n0 <= 1028; eps = the actor's LayerNorm
+ * epsilon; prepared = NULL or the buffer dora_actor_prepare filled (the
+ * encoder's folded and padded weights; without it every call rebuilds them
+ * in its workspace).  Every pointer 16-byte aligned.
+ */
+typedef struct {
+  const dora_bf16 *gate_w1, *gate_b1, *gate_w2, *gate_b2, *gate_emb;
+  const dora_bf16 *enc_w_in, *enc_b_in, *enc_emb, *enc_w_h;
+  const dora_bf16 *enc_ln1_w, *enc_ln1_b, *enc_w_qkv, *enc_b_qkv, *enc_w_o, *enc_b_o;
+  const dora_bf16 *enc_ln2_w, *enc_ln2_b, *enc_w_fc1, *enc_b_fc1, *enc_w_fc2, *enc_b_fc2;
+  const dora_bf16 *bud_ln_w, *bud_ln_b, *bud_w1, *bud_b1, *bud_w2, *bud_b2;
+  const dora_bf16 *sel_w_k, *sel_w1, *sel_b1, *sel_w2, *sel_b2;
+  int32_t dim, depth, n0;
+  float eps;
+  const void* prepared;
+} dora_actor_weights;
+
+/* Bytes dora_actor_prepare writes; bytes of workspace dora_actor needs for
+ * t_cap rows and `batch` images (it includes the prepared weights when
+ * w->prepared is NULL). */
+size_t dora_actor_prepared_size(const dora_actor_weights* w);
+size_t dora_actor_workspace_size(int32_t t_cap, int32_t batch, const dora_actor_weights* w);
+
+/* Builds the encoder's device-side weights once: the per-block input bias
+ * b_in + e^C_l (bf16), the QKV and feed-forward weights with their
+ * LayerNorms folded in (as dora_fold_ln_linear), and the QKV rows and W_o
+ * columns zero-padded from heads of 32 to heads of 64. */
+int dora_actor_prepare(const dora_actor_weights* w, void* prepared, size_t prepared_bytes,
+                       dora_stream_t stream);
+
+/*
+ * dora_actor -- the actor at block `block` (0 <= block < L) for the packed
+ * batch.  qkv bf16 [t_cap, 3 dim] is the block's QKV output (its keys are
+ * columns [dim, 2 dim), heads concatenated); cu int32 [batch + 1] the image
+ * boundaries (row cu[i] is image i's CLS).  rho fp32 [batch] and
+ * interventions int32 [batch] are each image's rho_l and E_<l (zeros at
+ * block 0); n_l = cu[i+1] - cu[i] - 1 visual tokens.
+ * Outputs per image: p_gate fp32 (nullable; the gate probability), gate
+ * int32 (1 when p >= 0.5 and a budget is feasible), budget int32 (the
+ * highest-logit budget with k <= n_l - 4, ties to the smaller, 0 if none),
+ * k int32 (budget when the gate is open, else 0), keep_counts int32
+ * (n_l + 1 - k, CLS included), rho_next fp32 and interventions_next int32
+ * (nullable; the next block's history: k / n_l and E_<l + gate; may alias
+ * rho and interventions).  scores fp32 [t_cap]: the selector's deletion
+ * score of every visual row, computed with the image's budget (CLS rows 0).
+ * z_out nullable bf16 [t_cap, 128]: the encoder output Z_l.
+ * The encoder runs on bf16 GEMMs with fp32 accumulation (heads of 32
+ * padded to the attention kernel's 64); gate, budget head and selector in
+ * fp32.  The gate decision is the sign of the gate logit (p >= 0.5).
+ * workspace: dora_actor_workspace_size bytes, 256-byte aligned; its first
+ * word is the status word (dora_workspace_status).
+ */
+int dora_actor(const dora_bf16* qkv, const int32_t* cu, int32_t batch, int32_t max_seqlen,
+               int32_t t_cap, int32_t block, const dora_actor_weights* w, const float* rho,
+               const int32_t* interventions, float* p_gate, int32_t* gate, int32_t* budget,
+               int32_t* k, int32_t* keep_counts, float* scores, float* rho_next,
+               int32_t* interventions_next, dora_bf16* z_out, void* workspace,
+               size_t workspace_bytes, dora_stream_t stream);
+
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug
  * only: it blocks the host. */

@@ -448,7 +448,8 @@ def actor_block(keys: np.ndarray, cu: np.ndarray, block: int, n0: int, depth: in
         zi = actor_encoder(keys[lo:hi], w["enc_emb"][block], h, w, eps)
         z[lo:hi] = zi
         budget[i], logits[i] = actor_budget(zi[0], n_l, n0, w, eps)
-        scores[lo + 1:hi] = actor_selector(zi[1:], int(budget[i]), n_l, w)
+        if n_l > 0:                                   # an image of CLS alone has nothing to score
+            scores[lo + 1:hi] = actor_selector(zi[1:], int(budget[i]), n_l, w)
         gate[i] = int(p[i] >= 0.5 and budget[i] > 0)
         k[i] = budget[i] if gate[i] else 0
     n_vis = np.diff(cu) - 1

@@ -22,7 +22,8 @@ __all__ = [
     "dora_pruned_block_noalloc", "NOALLOC_SCRATCH_BYTES", "dora_row_stats",
     "dora_fold_ln_linear", "dora_linear_ln", "dora_linear_residual_stats",
     "dora_folded_weights_size", "dora_fold_block_weights", "dora_compact_stats",
-    "dora_merge_moments",
+    "dora_merge_moments", "ActorWeights", "dora_actor", "dora_actor_workspace_size",
+    "alloc_actor_workspace",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -64,6 +65,11 @@ _SIGS = {
     "dora_compact_stats": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp,
                                           _vp, _vp, _vp]),
     "dora_merge_moments": (ctypes.c_int, [_vp, _i32, _vp, _i32, _vp, _vp]),
+    "dora_actor_prepared_size": (_sz, [_vp]),
+    "dora_actor_workspace_size": (_sz, [_i32, _i32, _vp]),
+    "dora_actor_prepare": (ctypes.c_int, [_vp, _vp, _sz, _vp]),
+    "dora_actor": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp,
+                                  _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -462,3 +468,90 @@ def dora_read_status(status) -> int:
     code = ctypes.c_int32(0)
     _check(load_library().dora_read_status(_ptr(status), ctypes.byref(code)), "dora_read_status")
     return int(code.value)
+
+
+# ---------------------------------------------------------------------------
+# the deployment actor
+# ---------------------------------------------------------------------------
+_ACTOR_NAMES = ("gate_w1", "gate_b1", "gate_w2", "gate_b2", "gate_emb", "enc_w_in", "enc_b_in",
+                "enc_emb", "enc_w_h", "enc_ln1_w", "enc_ln1_b", "enc_w_qkv", "enc_b_qkv",
+                "enc_w_o", "enc_b_o", "enc_ln2_w", "enc_ln2_b", "enc_w_fc1", "enc_b_fc1",
+                "enc_w_fc2", "enc_b_fc2", "bud_ln_w", "bud_ln_b", "bud_w1", "bud_b1", "bud_w2",
+                "bud_b2", "sel_w_k", "sel_w1", "sel_b1", "sel_w2", "sel_b2")
+
+
+class _ActorWeightsC(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in _ACTOR_NAMES] + [
+        ("dim", _i32), ("depth", _i32), ("n0", _i32), ("eps", _f32), ("prepared", _vp)]
+
+
+class ActorWeights:
+    """Device weights of the actor (dora_actor_weights) plus the C struct that
+    points at them.  ``tensors`` maps the struct's names to bf16 CUDA tensors;
+    ``prepare()`` builds the encoder's folded and padded weights once."""
+
+    NAMES = _ACTOR_NAMES
+
+    def __init__(self, tensors: dict, dim: int, depth: int, n0: int, eps: float = 1e-5):
+        self.tensors = {}
+        for n in self.NAMES:
+            t = tensors.get(n)
+            _req(t, torch.bfloat16, n)
+            self.tensors[n] = t.contiguous()
+        self.dim, self.depth, self.n0, self.eps = dim, depth, n0, eps
+        self.prepared = None
+        self.c = _ActorWeightsC(*[_ptr(self.tensors[n]) for n in self.NAMES], dim, depth, n0,
+                                float(eps), None)
+
+    def prepare(self, stream=None):
+        n = int(load_library().dora_actor_prepared_size(ctypes.byref(self.c)))
+        buf = torch.empty(n + 256, dtype=torch.uint8, device=self.tensors["enc_w_in"].device)
+        off = (-buf.data_ptr()) % 256
+        prep = buf[off:off + n]
+        self.c.prepared = None
+        _check(load_library().dora_actor_prepare(ctypes.byref(self.c), _ptr(prep), n,
+                                                 _stream(stream)), "dora_actor_prepare")
+        self.prepared = buf
+        self.c.prepared = _ptr(prep)
+        return self
+
+
+def dora_actor_workspace_size(t_cap, batch, weights: ActorWeights) -> int:
+    return int(load_library().dora_actor_workspace_size(int(t_cap), int(batch),
+                                                        ctypes.byref(weights.c)))
+
+
+def alloc_actor_workspace(t_cap, batch, weights: ActorWeights, device=None) -> torch.Tensor:
+    n = dora_actor_workspace_size(t_cap, batch, weights)
+    return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def dora_actor(qkv, cu, weights: ActorWeights, block, max_seqlen, rho, interventions, gate,
+               budget, k, keep_counts, scores, workspace, p_gate=None, rho_next=None,
+               interventions_next=None, z_out=None, stream=None):
+    """The deterministic actor at one block (dora_actor): gate, budget, k,
+    keep counts and deletion scores for every image of the packed batch."""
+    _req(qkv, torch.bfloat16, "qkv")
+    _req(cu, torch.int32, "cu")
+    _req(workspace, torch.uint8, "workspace")
+    for n, t, dt, opt in (("rho", rho, torch.float32, False),
+                          ("interventions", interventions, torch.int32, False),
+                          ("gate", gate, torch.int32, False), ("budget", budget, torch.int32, False),
+                          ("k", k, torch.int32, False), ("keep_counts", keep_counts, torch.int32, False),
+                          ("scores", scores, torch.float32, False),
+                          ("p_gate", p_gate, torch.float32, True),
+                          ("rho_next", rho_next, torch.float32, True),
+                          ("interventions_next", interventions_next, torch.int32, True),
+                          ("z_out", z_out, torch.bfloat16, True)):
+        _req(t, dt, n, optional=opt)
+    t_cap = qkv.shape[0]
+    batch = cu.numel() - 1
+    if qkv.shape[1] != 3 * weights.dim or scores.numel() < t_cap:
+        raise ValueError("qkv must be [t_cap, 3 dim] and scores hold t_cap floats")
+    if z_out is not None and tuple(z_out.shape) != (t_cap, 128):
+        raise ValueError("z_out must be [t_cap, 128]")
+    _check(load_library().dora_actor(
+        _ptr(qkv), _ptr(cu), batch, int(max_seqlen), t_cap, int(block), ctypes.byref(weights.c),
+        _ptr(rho), _ptr(interventions), _ptr(p_gate), _ptr(gate), _ptr(budget), _ptr(k),
+        _ptr(keep_counts), _ptr(scores), _ptr(rho_next), _ptr(interventions_next), _ptr(z_out),
+        _ptr(workspace), workspace.numel(), _stream(stream)), "dora_actor")

@@ -1,0 +1,483 @@
+// The deterministic actor of DORA at deployment (Sec. 3.2 "The actor";
+// Appendix A.1-A.3), at one block, for every image of a packed batch:
+//   gate      p = sigmoid(MLP_G([K_CLS, e^G_l, h_l])), a (d + 19) -> 64 -> 1
+//             SiLU MLP: one CTA per image;
+//   encoder   X = W_in K + b_in + e^C_l (+ W_h h_l on the CLS row), then one
+//             pre-LayerNorm Transformer block of width 128 (four heads of 32,
+//             GELU feed-forward 128 -> 256 -> 128), run on the library's
+//             tcgen05 GEMMs (LayerNorms folded in) and varlen attention;
+//   budget    the highest logit of MLP_B(LayerNorm(Z_CLS)) among the budgets
+//             k <= N_l - 4 (ties to the smaller), and
+//   selector  s_j = MLP_S(Z_j + W_k k / N_l), a 128 -> 64 -> 1 SiLU MLP:
+//             one CTA per image.
+// The attention kernel works on heads of 64 lanes.  The encoder's heads of 32
+// are zero-padded to 64: the padded QKV rows and W_o columns are zero, so
+// every score, softmax weight and head output equals that of the 32-wide head
+// (the softmax scale stays 1/sqrt(32)).
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "dora.h"
+#include "dora_ptx.cuh"
+#include "token_ops.cuh"
+
+namespace dora {
+namespace actor {
+
+constexpr int W = 128;          // encoder width
+constexpr int HEADS = 4;
+constexpr int HD = 32;          // encoder head width
+constexpr int HDP = 64;         // padded head width
+constexpr int FF = 256;         // feed-forward width
+constexpr int GH = 64;          // gate hidden units
+constexpr int GE = 16;          // gate block embedding
+constexpr int SH = 64;          // selector hidden units
+constexpr int kMaxDim = 2048;
+constexpr int kMaxN0 = 1028;    // budget-head outputs (n0 - 4) / 2 <= 512
+constexpr int kMaxBudgets = (kMaxN0 - 4) / 2;
+constexpr int kSelWarps = 8;
+
+__device__ __forceinline__ float ld(const uint16_t* __restrict__ p, size_t i) {
+  return __uint_as_float(static_cast<uint32_t>(p[i]) << 16);
+}
+__device__ __forceinline__ uint16_t to_bf16(float v) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(v);
+  return *reinterpret_cast<const uint16_t*>(&h);
+}
+__device__ __forceinline__ float silu(float x) { return x / (1.f + expf(-x)); }
+__device__ __forceinline__ float gelu(float x) {
+  return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// ---------------------------------------------------------------------------
+// preparation (once per set of weights)
+// ---------------------------------------------------------------------------
+// Padded QKV [768, 128]: row part * 256 + head * 64 + j takes folded row
+// part * 128 + head * 32 + j for j < 32 and is zero otherwise (so are its c, d).
+__global__ void pad_qkv_kernel(const uint16_t* __restrict__ wf, const float* __restrict__ cf,
+                               const float* __restrict__ df, uint16_t* __restrict__ wp,
+                               float* __restrict__ cp, float* __restrict__ dp) {
+  const int p = blockIdx.x;
+  const int part = p / (HEADS * HDP), head = (p / HDP) % HEADS, j = p % HDP;
+  const bool live = j < HD;
+  const int src = part * W + head * HD + j;
+  for (int c = threadIdx.x; c < W; c += blockDim.x)
+    wp[static_cast<size_t>(p) * W + c] = live ? wf[static_cast<size_t>(src) * W + c] : 0;
+  if (threadIdx.x == 0) {
+    cp[p] = live ? cf[src] : 0.f;
+    dp[p] = live ? df[src] : 0.f;
+  }
+}
+
+// Padded W_o [128, 256]: column head * 64 + j takes column head * 32 + j for
+// j < 32 and is zero otherwise.
+__global__ void pad_wo_kernel(const uint16_t* __restrict__ wo, uint16_t* __restrict__ wp) {
+  const int r = blockIdx.x;
+  for (int c = threadIdx.x; c < HEADS * HDP; c += blockDim.x) {
+    const int head = c / HDP, j = c % HDP;
+    wp[static_cast<size_t>(r) * HEADS * HDP + c] =
+        j < HD ? wo[static_cast<size_t>(r) * W + head * HD + j] : 0;
+  }
+}
+
+// The input projection's bias at every block: bf16(b_in + e^C_l).
+__global__ void bias_in_kernel(const uint16_t* __restrict__ b_in, const uint16_t* __restrict__ emb,
+                               uint16_t* __restrict__ out) {
+  const int l = blockIdx.x;
+  for (int c = threadIdx.x; c < W; c += blockDim.x)
+    out[static_cast<size_t>(l) * W + c] = to_bf16(ld(b_in, c) + ld(emb, static_cast<size_t>(l) * W + c));
+}
+
+// ---------------------------------------------------------------------------
+// gate (Appendix A.1): one CTA of 128 threads per image
+// ---------------------------------------------------------------------------
+// h_l = [N_l / N0, rho_l, E_<l / (L - 1)]; the gate logit and p^G; and W_h h_l
+// added to the image's CLS row of the encoder input x [rows, 128].
+__global__ void __launch_bounds__(128) gate_kernel(
+    const uint16_t* __restrict__ qkv, int dim, const int32_t* __restrict__ cu, int t_cap, int block,
+    int depth, int n0, const float* __restrict__ rho, const int32_t* __restrict__ interventions,
+    const uint16_t* __restrict__ w1, const uint16_t* __restrict__ b1,
+    const uint16_t* __restrict__ w2, const uint16_t* __restrict__ b2,
+    const uint16_t* __restrict__ emb, const uint16_t* __restrict__ w_h,
+    uint16_t* __restrict__ x, float* __restrict__ glogit, float* __restrict__ p_gate) {
+  __shared__ float z[kMaxDim + GE + 3];
+  __shared__ float hid[GH];
+  const int i = blockIdx.x, t = threadIdx.x;
+  const int lo = cu[i], hi = cu[i + 1];
+  const int n = (lo < 0 || hi > t_cap) ? -1 : hi - lo - 1;   // visual tokens
+  if (n < 0) {                                       // empty (or outside the buffer): closed
+    if (t == 0) {
+      glogit[i] = -INFINITY;
+      if (p_gate != nullptr) p_gate[i] = 0.f;
+    }
+    return;
+  }
+  const float h0 = static_cast<float>(n) / static_cast<float>(n0);
+  const float h1 = rho[i];
+  const float h2 = static_cast<float>(interventions[i]) / static_cast<float>(max(depth - 1, 1));
+  const size_t krow = static_cast<size_t>(lo) * 3 * dim + dim;   // the CLS key
+  for (int c = t; c < dim; c += blockDim.x) z[c] = ld(qkv, krow + c);
+  if (t < GE) z[dim + t] = ld(emb, static_cast<size_t>(block) * GE + t);
+  if (t == 0) {
+    z[dim + GE] = h0;
+    z[dim + GE + 1] = h1;
+    z[dim + GE + 2] = h2;
+  }
+  __syncthreads();
+  const int kin = dim + GE + 3;
+  if (t < GH) {
+    const uint16_t* wr = w1 + static_cast<size_t>(t) * kin;
+    float a = ld(b1, t);
+    for (int c = 0; c < kin; ++c) a = fmaf(ld(wr, c), z[c], a);
+    hid[t] = silu(a);
+  }
+  __syncthreads();
+  if (t < 32) {
+    const float s = warp_sum(ld(w2, t) * hid[t] + ld(w2, t + 32) * hid[t + 32]);
+    if (t == 0) {
+      const float lg = s + ld(b2, 0);
+      glogit[i] = lg;
+      if (p_gate != nullptr) p_gate[i] = 1.f / (1.f + expf(-lg));
+    }
+  }
+  // the history enters the encoder on the CLS token only
+  uint16_t* xr = x + static_cast<size_t>(lo) * W;
+  const float v = ld(w_h, t * 3) * h0 + ld(w_h, t * 3 + 1) * h1 + ld(w_h, t * 3 + 2) * h2;
+  xr[t] = to_bf16(ld(xr, t) + v);
+}
+
+// ---------------------------------------------------------------------------
+// budget head and selector (Sec. 3.2, Eq. 2; Appendix A.1-A.3): one CTA of
+// 256 threads per image
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) budget_select_kernel(
+    const uint16_t* __restrict__ z, const int32_t* __restrict__ cu, int t_cap, int n0, float eps,
+    const uint16_t* __restrict__ ln_w, const uint16_t* __restrict__ ln_b,
+    const uint16_t* __restrict__ bw1, const uint16_t* __restrict__ bb1,
+    const uint16_t* __restrict__ bw2, const uint16_t* __restrict__ bb2,
+    const uint16_t* __restrict__ w_k, const uint16_t* __restrict__ sw1,
+    const uint16_t* __restrict__ sb1, const uint16_t* __restrict__ sw2,
+    const uint16_t* __restrict__ sb2, const float* __restrict__ glogit,
+    const int32_t* __restrict__ interventions, int32_t* __restrict__ gate,
+    int32_t* __restrict__ budget, int32_t* __restrict__ k_out, int32_t* __restrict__ keep,
+    float* __restrict__ rho_next, int32_t* __restrict__ e_next, float* __restrict__ scores) {
+  __shared__ float u[W], hb[W], logit[kMaxBudgets];
+  __shared__ float su[kSelWarps][W];
+  __shared__ int s_budget;
+  const int i = blockIdx.x, t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int lo = cu[i], hi = cu[i + 1];
+  const int n = (lo < 0 || hi > t_cap) ? -1 : hi - lo - 1;
+  const int m_out = (n0 - 4) / 2;
+  if (n < 0) {
+    if (t == 0) {
+      gate[i] = budget[i] = k_out[i] = keep[i] = 0;
+      if (rho_next != nullptr) rho_next[i] = 0.f;
+      if (e_next != nullptr) e_next[i] = interventions[i];
+    }
+    return;
+  }
+  const size_t zc = static_cast<size_t>(lo) * W;
+  if (warp == 0) {                                   // LayerNorm(Z_CLS)
+    float v[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) v[q] = ld(z, zc + lane + 32 * q);
+    const float mean = warp_sum(v[0] + v[1] + v[2] + v[3]) * (1.f / W);
+    float d2 = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) d2 += (v[q] - mean) * (v[q] - mean);
+    const float rstd = rsqrtf(warp_sum(d2) * (1.f / W) + eps);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int c = lane + 32 * q;
+      u[c] = (v[q] - mean) * rstd * ld(ln_w, c) + ld(ln_b, c);
+    }
+  }
+  __syncthreads();
+  if (t < W) {
+    float a = ld(bb1, t);
+    for (int c = 0; c < W; ++c) a = fmaf(ld(bw1, static_cast<size_t>(t) * W + c), u[c], a);
+    hb[t] = gelu(a);
+  }
+  __syncthreads();
+  for (int m = t; m < m_out; m += blockDim.x) {
+    float a = ld(bb2, m);
+    for (int c = 0; c < W; ++c) a = fmaf(ld(bw2, static_cast<size_t>(m) * W + c), hb[c], a);
+    logit[m] = a;
+  }
+  __syncthreads();
+  if (t == 0) {
+    int best = -1;
+    float bv = 0.f;
+    for (int m = 0; m < m_out; ++m)
+      if (2 * (m + 1) <= n - 4 && (best < 0 || logit[m] > bv)) {
+        best = m;
+        bv = logit[m];
+      }
+    const int bud = best < 0 ? 0 : 2 * (best + 1);
+    const int g = (glogit[i] >= 0.f && bud > 0) ? 1 : 0;
+    const int kk = g ? bud : 0;
+    budget[i] = bud;
+    gate[i] = g;
+    k_out[i] = kk;
+    keep[i] = n + 1 - kk;
+    if (rho_next != nullptr) rho_next[i] = n > 0 ? static_cast<float>(kk) / n : 0.f;
+    if (e_next != nullptr) e_next[i] = interventions[i] + g;
+    s_budget = bud;
+    scores[lo] = 0.f;
+  }
+  __syncthreads();
+  // selector: warp w scores visual tokens 1 + w, 1 + w + 8, ...; each lane
+  // owns two of the 64 hidden units
+  const float kr = n > 0 ? static_cast<float>(s_budget) / n : 0.f;
+  for (int j = 1 + warp; j <= n; j += kSelWarps) {
+    const size_t zr = static_cast<size_t>(lo + j) * W;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int c = lane + 32 * q;
+      su[warp][c] = ld(z, zr + c) + ld(w_k, c) * kr;
+    }
+    __syncwarp();
+    float part = 0.f;
+#pragma unroll
+    for (int q = 0; q < SH / 32; ++q) {
+      const int hh = lane + 32 * q;
+      float a = ld(sb1, hh);
+      for (int c = 0; c < W; ++c) a = fmaf(ld(sw1, static_cast<size_t>(hh) * W + c), su[warp][c], a);
+      part += ld(sw2, hh) * silu(a);
+    }
+    part = warp_sum(part);
+    if (lane == 0) scores[lo + j] = part + ld(sb2, 0);
+    __syncwarp();
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side: layouts
+// ---------------------------------------------------------------------------
+size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+struct Prep {
+  size_t bias_in, wqkv_f, cqkv_f, dqkv_f, wqkv_p, cqkv_p, dqkv_p, wo_p, wfc1, cfc1, dfc1, total;
+};
+
+Prep prep_layout(const dora_actor_weights* w) {
+  Prep P{};
+  size_t off = 0;
+  P.bias_in = off; off += up256(static_cast<size_t>(w->depth) * W * 2);
+  P.wqkv_f = off;  off += up256(3 * W * W * 2);
+  P.cqkv_f = off;  off += up256(3 * W * 4);
+  P.dqkv_f = off;  off += up256(3 * W * 4);
+  P.wqkv_p = off;  off += up256(3 * HEADS * HDP * W * 2);
+  P.cqkv_p = off;  off += up256(3 * HEADS * HDP * 4);
+  P.dqkv_p = off;  off += up256(3 * HEADS * HDP * 4);
+  P.wo_p = off;    off += up256(W * HEADS * HDP * 2);
+  P.wfc1 = off;    off += up256(FF * W * 2);
+  P.cfc1 = off;    off += up256(FF * 4);
+  P.dfc1 = off;    off += up256(FF * 4);
+  P.total = off;
+  return P;
+}
+
+struct Ws {
+  size_t status, x, mv, qkv, o, z1, sm, f, z, glogit, prep, total;
+};
+
+Ws ws_layout(int32_t t_cap, int32_t batch, const dora_actor_weights* w) {
+  Ws L{};
+  const size_t t = static_cast<size_t>(t_cap), b = static_cast<size_t>(batch);
+  size_t off = 0;
+  L.status = off; off += 256;
+  L.x = off;      off += up256(t * W * 2);
+  L.mv = off;     off += up256(t * 8);
+  L.qkv = off;    off += up256(t * 3 * HEADS * HDP * 2);
+  L.o = off;      off += up256(t * HEADS * HDP * 2);
+  L.z1 = off;     off += up256(t * W * 2);
+  L.sm = off;     off += up256(t * 2 * 8);
+  L.f = off;      off += up256(t * FF * 2);
+  L.z = off;      off += up256(t * W * 2);
+  L.glogit = off; off += up256(b * 4);
+  L.prep = off;   off += w->prepared != nullptr ? 0 : prep_layout(w).total;
+  L.total = off;
+  return L;
+}
+
+bool weights_ok(const dora_actor_weights* w) {
+  if (w == nullptr) return false;
+  if (w->dim <= 0 || w->dim % 64 != 0 || w->dim > kMaxDim) return false;
+  if (w->depth <= 0 || w->n0 < 6 || w->n0 > kMaxN0) return false;
+  if (!(w->eps >= 0.f) || !isfinite(w->eps)) return false;
+  const void* req[] = {w->gate_w1, w->gate_b1, w->gate_w2, w->gate_b2, w->gate_emb,
+                       w->enc_w_in, w->enc_b_in, w->enc_emb, w->enc_w_h, w->enc_ln1_w,
+                       w->enc_ln1_b, w->enc_w_qkv, w->enc_b_qkv, w->enc_w_o, w->enc_b_o,
+                       w->enc_ln2_w, w->enc_ln2_b, w->enc_w_fc1, w->enc_b_fc1, w->enc_w_fc2,
+                       w->enc_b_fc2, w->bud_ln_w, w->bud_ln_b, w->bud_w1, w->bud_b1,
+                       w->bud_w2, w->bud_b2, w->sel_w_k, w->sel_w1, w->sel_b1, w->sel_w2,
+                       w->sel_b2};
+  for (const void* p : req)
+    if (p == nullptr || (reinterpret_cast<uintptr_t>(p) & 15u) != 0) return false;
+  return (reinterpret_cast<uintptr_t>(w->prepared) & 255u) == 0;
+}
+
+cudaError_t prepare(const dora_actor_weights* w, uint8_t* prep, cudaStream_t stream) {
+  const Prep P = prep_layout(w);
+  cudaError_t e = launch_fold_ln(w->enc_w_qkv, 3 * W, W, w->enc_ln1_w, w->enc_ln1_b,
+                                 w->enc_b_qkv, reinterpret_cast<uint16_t*>(prep + P.wqkv_f),
+                                 reinterpret_cast<float*>(prep + P.cqkv_f),
+                                 reinterpret_cast<float*>(prep + P.dqkv_f), stream);
+  if (e != cudaSuccess) return e;
+  pad_qkv_kernel<<<3 * HEADS * HDP, 128, 0, stream>>>(
+      reinterpret_cast<const uint16_t*>(prep + P.wqkv_f),
+      reinterpret_cast<const float*>(prep + P.cqkv_f),
+      reinterpret_cast<const float*>(prep + P.dqkv_f), reinterpret_cast<uint16_t*>(prep + P.wqkv_p),
+      reinterpret_cast<float*>(prep + P.cqkv_p), reinterpret_cast<float*>(prep + P.dqkv_p));
+  pad_wo_kernel<<<W, 256, 0, stream>>>(w->enc_w_o, reinterpret_cast<uint16_t*>(prep + P.wo_p));
+  bias_in_kernel<<<w->depth, W, 0, stream>>>(w->enc_b_in, w->enc_emb,
+                                             reinterpret_cast<uint16_t*>(prep + P.bias_in));
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_fold_ln(w->enc_w_fc1, FF, W, w->enc_ln2_w, w->enc_ln2_b, w->enc_b_fc1,
+                        reinterpret_cast<uint16_t*>(prep + P.wfc1),
+                        reinterpret_cast<float*>(prep + P.cfc1),
+                        reinterpret_cast<float*>(prep + P.dfc1), stream);
+}
+
+}  // namespace actor
+}  // namespace dora
+
+using namespace dora;
+
+extern "C" {
+
+size_t dora_actor_prepared_size(const dora_actor_weights* w) {
+  if (w == nullptr || w->depth <= 0) return 0;
+  return actor::prep_layout(w).total;
+}
+
+size_t dora_actor_workspace_size(int32_t t_cap, int32_t batch, const dora_actor_weights* w) {
+  if (w == nullptr || t_cap < 0 || batch < 0 || w->depth <= 0) return 0;
+  return actor::ws_layout(t_cap, batch, w).total;
+}
+
+int dora_actor_prepare(const dora_actor_weights* w, void* prepared, size_t prepared_bytes,
+                       dora_stream_t stream) {
+  if (!actor::weights_ok(w) || prepared == nullptr ||
+      (reinterpret_cast<uintptr_t>(prepared) & 255u) != 0 ||
+      prepared_bytes < actor::prep_layout(w).total)
+    return DORA_ERR_INVALID_ARG;
+  const int dev = checked_device();
+  if (dev == -1) return DORA_ERR_CUDA;
+  if (dev < 0) return DORA_ERR_UNSUPPORTED;
+  return actor::prepare(w, static_cast<uint8_t*>(prepared),
+                        reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? DORA_OK
+             : DORA_ERR_CUDA;
+}
+
+int dora_actor(const dora_bf16* qkv, const int32_t* cu, int32_t batch, int32_t max_seqlen,
+               int32_t t_cap, int32_t block, const dora_actor_weights* w, const float* rho,
+               const int32_t* interventions, float* p_gate, int32_t* gate, int32_t* budget,
+               int32_t* k, int32_t* keep_counts, float* scores, float* rho_next,
+               int32_t* interventions_next, dora_bf16* z_out, void* workspace,
+               size_t workspace_bytes, dora_stream_t stream_) {
+  using namespace actor;
+  if (!weights_ok(w)) return DORA_ERR_INVALID_ARG;
+  if (batch < 0 || batch > 65535 || t_cap < 0 || max_seqlen < 0 || max_seqlen > 65535)
+    return DORA_ERR_INVALID_ARG;
+  if (block < 0 || block >= w->depth) return DORA_ERR_INVALID_ARG;
+  if (cu == nullptr || workspace == nullptr ||
+      (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return DORA_ERR_INVALID_ARG;
+  if (batch > 0 && (qkv == nullptr || rho == nullptr || interventions == nullptr ||
+                    gate == nullptr || budget == nullptr || k == nullptr ||
+                    keep_counts == nullptr || scores == nullptr))
+    return DORA_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(qkv) & 15u) != 0 ||
+      (reinterpret_cast<uintptr_t>(z_out) & 15u) != 0)
+    return DORA_ERR_INVALID_ARG;
+  const Ws L = ws_layout(t_cap, batch, w);
+  if (workspace_bytes < L.total) return DORA_ERR_INVALID_ARG;
+  const int dev = checked_device();
+  if (dev == -1) return DORA_ERR_CUDA;
+  if (dev < 0) return DORA_ERR_UNSUPPORTED;
+  if (t_cap == 0 || batch == 0) return DORA_OK;
+
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  int32_t* status = reinterpret_cast<int32_t*>(ws + L.status);
+  uint16_t* x = reinterpret_cast<uint16_t*>(ws + L.x);
+  float* mv = reinterpret_cast<float*>(ws + L.mv);
+  uint16_t* qkv_e = reinterpret_cast<uint16_t*>(ws + L.qkv);
+  uint16_t* o_e = reinterpret_cast<uint16_t*>(ws + L.o);
+  uint16_t* z1 = reinterpret_cast<uint16_t*>(ws + L.z1);
+  float* sm = reinterpret_cast<float*>(ws + L.sm);
+  uint16_t* f = reinterpret_cast<uint16_t*>(ws + L.f);
+  uint16_t* z = z_out != nullptr ? z_out : reinterpret_cast<uint16_t*>(ws + L.z);
+  float* glogit = reinterpret_cast<float*>(ws + L.glogit);
+  uint8_t* prep = ws + L.prep;
+  if (w->prepared != nullptr) prep = static_cast<uint8_t*>(const_cast<void*>(w->prepared));
+  else if (prepare(w, prep, stream) != cudaSuccess) return DORA_ERR_CUDA;
+  const Prep P = prep_layout(w);
+  const int32_t* rows = cu + batch;
+  const int d = w->dim;
+
+  // X = W_in K + (b_in + e^C_l), K read in place from the block's qkv rows
+  LinearEpi e_in;
+  e_in.bias = reinterpret_cast<const uint16_t*>(prep + P.bias_in) + static_cast<size_t>(block) * W;
+  if (launch_linear(qkv + d, t_cap, rows, d, w->enc_w_in, W, DORA_EPI_BIAS, e_in, x, status,
+                    stream, 3 * d) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  // gate, and the history term on every CLS row
+  gate_kernel<<<batch, 128, 0, stream>>>(qkv, d, cu, t_cap, block, w->depth, w->n0, rho, interventions,
+                                         w->gate_w1, w->gate_b1, w->gate_w2, w->gate_b2,
+                                         w->gate_emb, w->enc_w_h, x, glogit, p_gate);
+  if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
+  // Z1 = X + W_o Attention(LayerNorm1(X)) + b_o
+  LinearEpi e_q;
+  e_q.stats_in = mv;
+  e_q.colsum = reinterpret_cast<const float*>(prep + P.cqkv_p);
+  e_q.colbias = reinterpret_cast<const float*>(prep + P.dqkv_p);
+  e_q.eps = w->eps;
+  LinearEpi e_o;
+  e_o.bias = w->enc_b_o;
+  e_o.residual = x;
+  e_o.stats_out = sm;
+  e_o.slices = W / kSliceCols;
+  if (launch_row_stats(x, t_cap, rows, W, mv, stream) != cudaSuccess ||
+      launch_linear(x, t_cap, rows, W, reinterpret_cast<const uint16_t*>(prep + P.wqkv_p),
+                    3 * HEADS * HDP, kEpiLn, e_q, qkv_e, status, stream) != cudaSuccess ||
+      launch_varlen_attn(qkv_e, cu, batch, max_seqlen, t_cap, HEADS, 0.17677669529663688f, o_e,
+                         status, stream) != cudaSuccess ||
+      launch_linear(o_e, t_cap, rows, HEADS * HDP, reinterpret_cast<const uint16_t*>(prep + P.wo_p),
+                    W, DORA_EPI_BIAS_RESIDUAL, e_o, z1, status, stream) != cudaSuccess ||
+      launch_merge_moments(sm, t_cap, rows, W / kSliceCols, mv, stream) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  // Z = Z1 + W_2 GELU(W_1 LayerNorm2(Z1) + b_1) + b_2
+  LinearEpi e_f1;
+  e_f1.stats_in = mv;
+  e_f1.colsum = reinterpret_cast<const float*>(prep + P.cfc1);
+  e_f1.colbias = reinterpret_cast<const float*>(prep + P.dfc1);
+  e_f1.eps = w->eps;
+  LinearEpi e_f2;
+  e_f2.bias = w->enc_b_fc2;
+  e_f2.residual = z1;
+  if (launch_linear(z1, t_cap, rows, W, reinterpret_cast<const uint16_t*>(prep + P.wfc1), FF,
+                    kEpiLnGelu, e_f1, f, status, stream) != cudaSuccess ||
+      launch_linear(f, t_cap, rows, FF, w->enc_w_fc2, W, DORA_EPI_BIAS_RESIDUAL, e_f2, z, status,
+                    stream) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  // budget and selector
+  budget_select_kernel<<<batch, 256, 0, stream>>>(
+      z, cu, t_cap, w->n0, w->eps, w->bud_ln_w, w->bud_ln_b, w->bud_w1, w->bud_b1, w->bud_w2,
+      w->bud_b2, w->sel_w_k, w->sel_w1, w->sel_b1, w->sel_w2, w->sel_b2, glogit, interventions,
+      gate, budget, k, keep_counts, rho_next, interventions_next, scores);
+  return cudaGetLastError() == cudaSuccess ? DORA_OK : DORA_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -47,6 +47,8 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 }  // namespace
 
+int checked_device() { return current_device_checked(); }
+
 bool pdl_enabled() {
   static const bool on = getenv("DORA_NO_PDL") == nullptr;
   return on;

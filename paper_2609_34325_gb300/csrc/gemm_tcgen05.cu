@@ -693,12 +693,13 @@ static cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const
 
 cudaError_t launch_linear(const uint16_t* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
                           const uint16_t* w, int32_t n, int32_t epilogue, const LinearEpi& ep,
-                          uint16_t* y, int32_t* status, cudaStream_t stream) {
+                          uint16_t* y, int32_t* status, cudaStream_t stream, int32_t lda) {
   if (m_cap == 0) return cudaSuccess;
   const int bn = (n % 256 == 0) ? 256 : 128;
   CUtensorMap ta, tb, ty, tr;
+  if (lda != 0 && (lda < k || lda % 8 != 0)) return cudaErrorInvalidValue;
   if (encode_tmap_2d_bf16(&ta, x, static_cast<uint64_t>(k), static_cast<uint64_t>(m_cap),
-                          static_cast<uint64_t>(k) * 2, gemm::BK, gemm::BM) != 0)
+                          static_cast<uint64_t>(lda != 0 ? lda : k) * 2, gemm::BK, gemm::BM) != 0)
     return cudaErrorInvalidValue;
   if (encode_tmap_2d_bf16(&tb, w, static_cast<uint64_t>(k), static_cast<uint64_t>(n),
                           static_cast<uint64_t>(k) * 2, gemm::BK, static_cast<uint32_t>(bn / 2)) != 0)

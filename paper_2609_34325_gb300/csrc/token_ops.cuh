@@ -6,6 +6,10 @@
 
 namespace dora {
 
+// The current device if it is an sm_103 part; -1 when the query fails, -2
+// for another architecture.
+int checked_device();
+
 // Launch with programmatic stream serialization (dependent launch; the kernel
 // itself calls pdl_trigger / pdl_wait), unless DORA_NO_PDL is set.
 bool pdl_enabled();
@@ -90,9 +94,10 @@ struct LinearEpi {
   float eps = 0.f;                      // LayerNorm epsilon (LN epilogues)
   int32_t slices = 0;                   // n / 64 (stats_out)
 };
+// lda: row pitch of x in elements (0 = k; a multiple of 8).
 cudaError_t launch_linear(const uint16_t* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
                           const uint16_t* w, int32_t n, int32_t epilogue, const LinearEpi& ep,
-                          uint16_t* y, int32_t* status, cudaStream_t stream);
+                          uint16_t* y, int32_t* status, cudaStream_t stream, int32_t lda = 0);
 
 // tcgen05 varlen attention.
 cudaError_t launch_varlen_attn(const uint16_t* qkv, const int32_t* cu, int32_t batch,

@@ -99,3 +99,35 @@ def test_python_binding_rejects_cpu_tensors(lib):
     x = torch.zeros(4, 8, dtype=torch.bfloat16)
     with pytest.raises(TypeError):
         P.dora_layernorm(x, x[0], x[0], 1e-6, x)
+
+
+def test_actor_struct_sizes_and_host_checks(lib):
+    w = P._ActorWeightsC(*([16] * len(P.ActorWeights.NAMES)), 768, 12, 196, 1e-5, None)
+    prep = lib.dora_actor_prepared_size(ctypes.byref(w))
+    assert prep > 0
+    # per row: X, Z1, Z (128 bf16 each), padded qkv (768), attention out (256),
+    # feed-forward (256), row moments and two slice moments; per image the gate logit
+    t, b = 50000, 256
+    per_rows = t * (3 * 256 + 1536 + 512 + 512 + 8 + 16) + 4 * b
+    n = lib.dora_actor_workspace_size(t, b, ctypes.byref(w))
+    assert per_rows + prep <= n < per_rows + prep + 16 * 256
+    w.prepared = 256
+    assert lib.dora_actor_workspace_size(t, b, ctypes.byref(w)) == n - prep
+    w.prepared = None
+    n = lib.dora_actor_workspace_size(1000, 4, ctypes.byref(w))
+    args = [16, 16, 4, 197, 1000, 0, ctypes.byref(w), 16, 16, None, 16, 16, 16, 16, 16, None, None,
+            None, 256, n, None]
+    bad = []
+    for i, v in ((5, 12),):                       # block >= depth
+        a = list(args); a[i] = v; bad.append(a)
+    a = list(args); a[6] = None; bad.append(a)    # no weights
+    a = list(args); a[18] = 264; bad.append(a)    # misaligned workspace
+    a = list(args); a[19] = n - 1; bad.append(a)  # workspace too small
+    for a in bad:
+        assert lib.dora_actor(*a) == 1
+    for field, v in (("dim", 100), ("n0", 4), ("n0", 2000), ("depth", 0)):
+        w2 = P._ActorWeightsC(*([16] * len(P.ActorWeights.NAMES)), 768, 12, 196, 1e-5, None)
+        setattr(w2, field, v)
+        a = list(args); a[6] = ctypes.byref(w2)
+        assert lib.dora_actor(*a) == 1
+        assert lib.dora_actor_prepare(ctypes.byref(w2), 256, 1 << 20, None) == 1

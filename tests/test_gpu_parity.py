@@ -833,3 +833,121 @@ def test_forward_deit_b_shape_per_block():
             cu_d, ids_d = cu_o, ids_o
         cur = nxt
     assert np.array_equal(np.diff(host_cu), keeps[-1])
+
+
+# ---------------------------------------------------------------------------
+# the deployment actor (Sec. 3.2 "The actor"; Appendix A.1-A.3)
+# ---------------------------------------------------------------------------
+
+def _actor_case(cfg, seed, gate_bias=0.0, lens=None):
+    """Packed qkv rows with the given image lengths, per-image history, and the
+    actor's weights (host bits and prepared device copy)."""
+    rng = np.random.default_rng(seed)
+    if lens is None:
+        lens = np.full(cfg.batch, cfg.n_tokens)
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    qkv = S.f32_to_bf16_bits(rng.standard_normal((t, 3 * cfg.dim)))
+    rho = rng.uniform(0, 0.5, len(lens)).astype(np.float32)
+    e_prev = rng.integers(0, 3, len(lens)).astype(np.int32)
+    wa = S.actor_weights(cfg.dim, cfg.depth, cfg.n_vis0, seed, gate_bias=gate_bias)
+    aw = P.ActorWeights({k_: bf(v) for k_, v in wa.items()}, cfg.dim, cfg.depth, cfg.n_vis0)
+    return cu, qkv, rho, e_prev, wa, aw.prepare()
+
+
+def _run_actor(cfg, cu, qkv, rho, e_prev, aw, block, max_seqlen):
+    b, t = len(cu) - 1, int(cu[-1])
+    out = {n: torch.full((b,), -7, dtype=torch.int32, device=dev())
+           for n in ("gate", "budget", "k", "keep", "e_next")}
+    p = torch.zeros(b, dtype=torch.float32, device=dev())
+    rho_next = torch.zeros(b, dtype=torch.float32, device=dev())
+    scores = torch.full((t,), 5.0, dtype=torch.float32, device=dev())
+    z = torch.zeros(t, 128, dtype=torch.bfloat16, device=dev())
+    ws = P.alloc_actor_workspace(t, b, aw)
+    P.dora_actor(bf(qkv), i32(cu), aw, block, max_seqlen, f32(rho), i32(e_prev), out["gate"],
+                 out["budget"], out["k"], out["keep"], scores, ws, p_gate=p, rho_next=rho_next,
+                 interventions_next=out["e_next"], z_out=z)
+    torch.cuda.synchronize()
+    assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+    r = {n: v.cpu().numpy() for n, v in out.items()}
+    r.update(p=p.cpu().numpy(), rho_next=rho_next.cpu().numpy(), scores=scores.cpu().numpy(),
+             z=f64(z))
+    return r
+
+
+# The encoder's residual stream is rounded to bf16 three times (X, Z1, Z),
+# each by at most 2^-9 of the value, before the GEMM and attention errors the
+# block tolerance already allows for: 3e-2 absolute or 2e-2 relative.
+ACTOR_ATOL, ACTOR_RTOL = 3e-2, 2e-2
+
+
+def _check_actor(cfg, cu, qkv, rho, e_prev, wa, got, block, images):
+    """Oracle on a sub-batch of images (the actor treats images independently)."""
+    wf = O.decode_weights(wa)
+    rows, lcu = sub_batch(cu, images)
+    ref = O.actor_block(qkv[rows][:, cfg.dim:2 * cfg.dim], lcu, block, cfg.n_vis0, cfg.depth,
+                        rho[images], e_prev[images], wf)
+    n_vis = np.diff(cu)[images] - 1
+    # encoder output within the block tolerance; gate probability in fp32
+    assert_close(got["z"][rows], ref["z"], "actor Z", atol=ACTOR_ATOL, rtol=ACTOR_RTOL)
+    assert np.all(np.abs(got["p"][images] - ref["p"]) <= 1e-4)
+    # decisions agree wherever the oracle's margin exceeds the arithmetic's error
+    clear = np.abs(ref["p"] - 0.5) > 1e-4
+    assert np.array_equal((got["p"][images] >= 0.5)[clear], (ref["p"] >= 0.5)[clear])
+    grid = O.budget_grid(cfg.n_vis0)
+    for j, i in enumerate(images):
+        bud = int(got["budget"][i])
+        feas = grid <= n_vis[j] - 4
+        if not feas.any():
+            assert bud == 0
+            continue
+        assert bud in grid[feas]
+        best = ref["logits"][j][feas].max()
+        assert ref["logits"][j][list(grid).index(bud)] >= best - 0.05, (i, bud, ref["budget"][j])
+    # the integer bookkeeping is exact given the GPU's own decisions
+    g, bud = got["gate"][images], got["budget"][images]
+    assert np.array_equal(g, ((got["p"][images] >= 0.5) & (bud > 0)).astype(np.int32))
+    assert np.array_equal(got["k"][images], bud * g)
+    assert np.array_equal(got["keep"][images], n_vis + 1 - bud * g)
+    assert np.array_equal(got["e_next"][images], e_prev[images] + g)
+    assert np.allclose(got["rho_next"][images], bud * g / np.maximum(n_vis, 1), rtol=1e-6)
+    # selector scores: the oracle's selector on the oracle's Z with the GPU's budget
+    for j, i in enumerate(images):
+        lo, hi = int(lcu[j]), int(lcu[j + 1])
+        assert got["scores"][cu[i]] == 0.0
+        if n_vis[j] == 0:
+            continue
+        ref_s = O.actor_selector(ref["z"][lo + 1:hi], int(got["budget"][i]), int(n_vis[j]), wf)
+        assert_close(got["scores"][cu[i] + 1:cu[i + 1]], ref_s, f"actor scores image {i}",
+                     atol=ACTOR_ATOL, rtol=ACTOR_RTOL)
+
+
+@pytest.mark.parametrize("name,block,seed", [("cfg1", 0, 31), ("cfg2", 0, 32), ("cfg3", 5, 33)])
+def test_actor_matches_oracle(name, block, seed):
+    cfg = S.get_config(name)
+    lens = None
+    if name == "cfg3":
+        keeps, _ = S.keep_schedule(cfg, seed)
+        lens = keeps[1]                              # token counts after two deletions
+    cu, qkv, rho, e_prev, wa, aw = _actor_case(cfg, seed, lens=lens)
+    got = _run_actor(cfg, cu, qkv, rho, e_prev, aw, block, int(np.diff(cu).max()))
+    b = len(cu) - 1
+    images = list(range(b)) if b <= 64 else [0, 1, 77, 128, b - 2, b - 1]
+    _check_actor(cfg, cu, qkv, rho, e_prev, wa, got, block, images)
+
+
+def test_actor_edges_short_images_and_gate_bias():
+    """Images too short for any budget (N_l < 6) keep everything; an empty
+    image is skipped; a strongly positive or negative gate bias opens or
+    closes every feasible gate."""
+    cfg = S.get_config("cfg1")
+    lens = np.array([197, 6, 7, 1, 10, 0, 150, 3])
+    for gb, want in ((8.0, 1), (-8.0, 0)):
+        cu, qkv, rho, e_prev, wa, aw = _actor_case(cfg, 41, gate_bias=gb, lens=lens)
+        got = _run_actor(cfg, cu, qkv, rho, e_prev, aw, 0, int(lens.max()))
+        n_vis = lens - 1
+        feasible = n_vis >= 6
+        assert np.array_equal(got["gate"], (want * feasible).astype(np.int32))
+        assert np.array_equal(got["keep"], lens - got["k"])
+        assert np.all(got["k"][~feasible] == 0)
+        _check_actor(cfg, cu, qkv, rho, e_prev, wa, got, 0, [0, 1, 2, 3, 4, 6, 7])
