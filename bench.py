@@ -238,9 +238,24 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
         lanes.append(L)
     ws = lanes[0]["ws"]
     prune = list(cfg.prune_blocks)
+    # the deployment actor at random init (Sec. 3.2), for the leg whose
+    # deletion scores come from the actor (the configured keep counts stay)
+    actor = None
+    if not args.no_extras:
+        wa = S.actor_weights(cfg.dim, cfg.depth, cfg.n_vis0, args.seed)
+        actor = P.ActorWeights({k: bf(v) for k, v in wa.items()}, cfg.dim, cfg.depth,
+                               cfg.n_vis0).prepare(stream)
+        for L in lanes:
+            nb, tc = L["nb"], L["tcap"]
+            L["actor"] = dict(
+                ws=P.alloc_actor_workspace(tc, nb, actor, dev),
+                rho=torch.zeros(nb, dtype=torch.float32, device=dev),
+                e=torch.zeros(nb, dtype=torch.int32, device=dev),
+                out=[torch.zeros(nb, dtype=torch.int32, device=dev) for _ in range(4)],
+                scores=torch.zeros(tc, dtype=torch.float32, device=dev))
     launches_per_step = {True: 0, False: 0}
 
-    def forward(inp, pruned=True, pair=0):
+    def forward(inp, pruned=True, pair=0, with_actor=False):
         """One forward step: every lane through the 12 blocks, block launches
         interleaved across lanes; the main stream joins the others at the end.
         Returns [(x_out, cu_out)] per lane."""
@@ -263,7 +278,22 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
                 # first input, + merge of the output's moments)
                 n += 6 + (c["mv"] is None) + (mv_out is not None)
                 sl = L["stream"]
-                if pruned and l in prune:
+                if pruned and l in prune and with_actor:
+                    j = prune.index(l)
+                    A_ = L["actor"]
+                    P.dora_pruned_block_actor(c["x"], c["cu"], blocks[l], cfg.n_tokens, out,
+                                              L["ws"], actor, l, A_["rho"], A_["e"], *A_["out"],
+                                              A_["scores"], A_["ws"], c["ids"], cubuf[j % 2],
+                                              idbuf[j % 2],
+                                              keep_counts=inp["keeps"][j][L["i0"]:L["i1"]],
+                                              kept_idx=L["kept"], x_in_moments=c["mv"],
+                                              x_out_moments=mv_out, stream=sl)
+                    c["cu"], c["ids"] = cubuf[j % 2], idbuf[j % 2]
+                    # actor: input projection, gate, LayerNorm statistics, QKV,
+                    # attention, output projection, moment merge, two
+                    # feed-forward linears, budget and selector; then select, compact
+                    n += 10 + 2
+                elif pruned and l in prune:
                     j = prune.index(l)
                     P.dora_gather_scores(inp["tables"][j][L["i0"]:L["i1"]], c["ids"], c["cu"],
                                          L["scores"], stream=sl)
@@ -378,6 +408,20 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
     result["dense"] = {"value": round(cfg.batch * args.steps * world / dsecs, 1), "unit": UNIT,
                        "ms_per_step": round(1000 * dsecs / args.steps, 4)}
     result["speedup_vs_dense"] = round(dsecs / secs, 4)
+
+    # the same pruned forward with the actor producing the deletion scores at
+    # the pruning blocks (its cost included, as the paper's timing does)
+    asecs, _ = timed(lambda i: forward(sets[i % nsets], True, with_actor=True), args.steps,
+                     max(args.warmup, 3))
+    ast = max(P.dora_read_status(P.dora_workspace_status(L["actor"]["ws"])) for L in lanes)
+    result["with_actor"] = {
+        "value": round(cfg.batch * args.steps * world / asecs, 1), "unit": UNIT,
+        "ms_per_step": round(1000 * asecs / args.steps, 4),
+        "actor_ms_per_step": round(1000 * (asecs - secs) / args.steps, 4),
+        "device_status": ast,
+        "what": "actor at random init (gate, width-128 encoder, budget head, selector) on each "
+                "pruning block's keys; its scores choose the deleted tokens, the configured keep "
+                "counts stay"}
 
     # the same pruned step replayed as CUDA graphs (one per input set)
     try:

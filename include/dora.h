@@ -478,6 +478,30 @@ int dora_actor(const dora_bf16* qkv, const int32_t* cu, int32_t batch, int32_t m
                int32_t* interventions_next, dora_bf16* z_out, void* workspace,
                size_t workspace_bytes, dora_stream_t stream);
 
+/*
+ * dora_pruned_block_actor -- dora_pruned_block at block `block` with the
+ * actor deciding the deletion (Sec. 3.2; Eq. 1): after the attention
+ * residual, dora_actor runs on this block's own keys (the QKV linear's
+ * output inside the workspace) and its deletion scores feed select_keep.
+ * keep_counts NULL: the actor's keep counts are used (gate and budget
+ * decide); otherwise these counts, with the actor's scores choosing which
+ * tokens go.  The arguments after workspace_bytes are dora_actor's
+ * (aw->dim == w->dim; gate, budget, k, actor_keep [batch], scores [t_cap]
+ * required; rho_next, interventions_next nullable); the actor's status word
+ * is the first word of actor_workspace.  cu_out, ids_in, ids_out required.
+ */
+int dora_pruned_block_actor(const dora_bf16* x_in, const int32_t* cu_in, const int32_t* ids_in,
+                            int32_t batch, int32_t max_seqlen, int32_t t_cap,
+                            const dora_block_weights* w, dora_bf16* x_out, int32_t* cu_out,
+                            int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
+                            float* x_out_moments, void* workspace, size_t workspace_bytes,
+                            const dora_actor_weights* aw, int32_t block, const float* rho,
+                            const int32_t* interventions, const int32_t* keep_counts,
+                            int32_t* gate, int32_t* budget, int32_t* k, int32_t* actor_keep,
+                            float* scores, float* rho_next, int32_t* interventions_next,
+                            void* actor_workspace, size_t actor_workspace_bytes,
+                            dora_stream_t stream);
+
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug
  * only: it blocks the host. */

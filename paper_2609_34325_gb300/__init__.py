@@ -23,7 +23,7 @@ __all__ = [
     "dora_fold_ln_linear", "dora_linear_ln", "dora_linear_residual_stats",
     "dora_folded_weights_size", "dora_fold_block_weights", "dora_compact_stats",
     "dora_merge_moments", "ActorWeights", "dora_actor", "dora_actor_workspace_size",
-    "alloc_actor_workspace",
+    "alloc_actor_workspace", "dora_pruned_block_actor",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -70,6 +70,10 @@ _SIGS = {
     "dora_actor_prepare": (ctypes.c_int, [_vp, _vp, _sz, _vp]),
     "dora_actor": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp,
                                   _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "dora_pruned_block_actor": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
+                                               _vp, _vp, _vp, _vp, _vp, _sz, _vp, _i32, _vp, _vp,
+                                               _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
+                                               _vp]),
 }
 EXPORTED_SYMBOLS = tuple(_SIGS)
 
@@ -555,3 +559,38 @@ def dora_actor(qkv, cu, weights: ActorWeights, block, max_seqlen, rho, intervent
         _ptr(rho), _ptr(interventions), _ptr(p_gate), _ptr(gate), _ptr(budget), _ptr(k),
         _ptr(keep_counts), _ptr(scores), _ptr(rho_next), _ptr(interventions_next), _ptr(z_out),
         _ptr(workspace), workspace.numel(), _stream(stream)), "dora_actor")
+
+
+def dora_pruned_block_actor(x_in, cu_in, weights: BlockWeights, max_seqlen, x_out, workspace,
+                            actor: ActorWeights, block, rho, interventions, gate, budget, k,
+                            actor_keep, scores, actor_workspace, ids_in, cu_out, ids_out,
+                            keep_counts=None, kept_idx=None, rho_next=None,
+                            interventions_next=None, x_in_moments=None, x_out_moments=None,
+                            stream=None):
+    """dora_pruned_block with the actor deciding the deletion at this block
+    (its scores; its keep counts unless ``keep_counts`` is given)."""
+    _req(x_in, torch.bfloat16, "x_in")
+    _req(x_out, torch.bfloat16, "x_out")
+    for n, t in (("cu_in", cu_in), ("ids_in", ids_in), ("cu_out", cu_out), ("ids_out", ids_out),
+                 ("interventions", interventions), ("gate", gate), ("budget", budget), ("k", k),
+                 ("actor_keep", actor_keep)):
+        _req(t, torch.int32, n)
+    for n, t in (("keep_counts", keep_counts), ("kept_idx", kept_idx),
+                 ("interventions_next", interventions_next)):
+        _req(t, torch.int32, n, optional=True)
+    _req(rho, torch.float32, "rho")
+    _req(scores, torch.float32, "scores")
+    for n, t in (("rho_next", rho_next), ("x_in_moments", x_in_moments),
+                 ("x_out_moments", x_out_moments)):
+        _req(t, torch.float32, n, optional=True)
+    _req(workspace, torch.uint8, "workspace")
+    _req(actor_workspace, torch.uint8, "actor_workspace")
+    t_cap = x_in.shape[0]
+    _check(load_library().dora_pruned_block_actor(
+        _ptr(x_in), _ptr(cu_in), _ptr(ids_in), cu_in.numel() - 1, int(max_seqlen), t_cap,
+        ctypes.byref(weights.c), _ptr(x_out), _ptr(cu_out), _ptr(ids_out), _ptr(kept_idx),
+        _ptr(x_in_moments), _ptr(x_out_moments), _ptr(workspace), workspace.numel(),
+        ctypes.byref(actor.c), int(block), _ptr(rho), _ptr(interventions), _ptr(keep_counts),
+        _ptr(gate), _ptr(budget), _ptr(k), _ptr(actor_keep), _ptr(scores), _ptr(rho_next),
+        _ptr(interventions_next), _ptr(actor_workspace), actor_workspace.numel(),
+        _stream(stream)), "dora_pruned_block_actor")

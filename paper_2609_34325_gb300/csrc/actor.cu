@@ -8,8 +8,10 @@
 //             tcgen05 GEMMs (LayerNorms folded in) and varlen attention;
 //   budget    the highest logit of MLP_B(LayerNorm(Z_CLS)) among the budgets
 //             k <= N_l - 4 (ties to the smaller), and
-//   selector  s_j = MLP_S(Z_j + W_k k / N_l), a 128 -> 64 -> 1 SiLU MLP:
-//             one CTA per image.
+//   selector  s_j = MLP_S(Z_j + W_k k / N_l), a 128 -> 64 -> 1 SiLU MLP,
+//             written W_1 Z_j + b_1 + (k / N_l) W_1 W_k: the first term is one
+//             tcgen05 GEMM over all tokens, W_1 W_k is made once per set of
+//             weights, and the rest runs per token.
 // The attention kernel works on heads of 64 lanes.  The encoder's heads of 32
 // are zero-padded to 64: the padded QKV rows and W_o columns are zero, so
 // every score, softmax weight and head output equals that of the 32-wide head
@@ -87,6 +89,15 @@ __global__ void pad_wo_kernel(const uint16_t* __restrict__ wo, uint16_t* __restr
   }
 }
 
+// The selector's W_1 W_k (fp32 [64]).
+__global__ void sel_wk_kernel(const uint16_t* __restrict__ w1, const uint16_t* __restrict__ w_k,
+                              float* __restrict__ out) {
+  const int h = threadIdx.x;
+  float a = 0.f;
+  for (int c = 0; c < W; ++c) a = fmaf(ld(w1, static_cast<size_t>(h) * W + c), ld(w_k, c), a);
+  out[h] = a;
+}
+
 // The input projection's bias at every block: bf16(b_in + e^C_l).
 __global__ void bias_in_kernel(const uint16_t* __restrict__ b_in, const uint16_t* __restrict__ emb,
                                uint16_t* __restrict__ out) {
@@ -132,11 +143,16 @@ __global__ void __launch_bounds__(128) gate_kernel(
   }
   __syncthreads();
   const int kin = dim + GE + 3;
-  if (t < GH) {
-    const uint16_t* wr = w1 + static_cast<size_t>(t) * kin;
-    float a = ld(b1, t);
-    for (int c = 0; c < kin; ++c) a = fmaf(ld(wr, c), z[c], a);
-    hid[t] = silu(a);
+  {
+    // hidden unit h is one warp's dot product, the lanes striding along it
+    const int warp = t >> 5, lane = t & 31;
+    for (int h = warp; h < GH; h += 4) {
+      const uint16_t* wr = w1 + static_cast<size_t>(h) * kin;
+      float a = 0.f;
+      for (int c = lane; c < kin; c += 32) a = fmaf(ld(wr, c), z[c], a);
+      a = warp_sum(a);
+      if (lane == 0) hid[h] = silu(a + ld(b1, h));
+    }
   }
   __syncthreads();
   if (t < 32) {
@@ -162,14 +178,14 @@ __global__ void __launch_bounds__(256) budget_select_kernel(
     const uint16_t* __restrict__ ln_w, const uint16_t* __restrict__ ln_b,
     const uint16_t* __restrict__ bw1, const uint16_t* __restrict__ bb1,
     const uint16_t* __restrict__ bw2, const uint16_t* __restrict__ bb2,
-    const uint16_t* __restrict__ w_k, const uint16_t* __restrict__ sw1,
-    const uint16_t* __restrict__ sb1, const uint16_t* __restrict__ sw2,
-    const uint16_t* __restrict__ sb2, const float* __restrict__ glogit,
+    const uint16_t* __restrict__ s1, const float* __restrict__ sel_wk,
+    const uint16_t* __restrict__ sw2, const uint16_t* __restrict__ sb2,
+    const float* __restrict__ glogit,
     const int32_t* __restrict__ interventions, int32_t* __restrict__ gate,
     int32_t* __restrict__ budget, int32_t* __restrict__ k_out, int32_t* __restrict__ keep,
     float* __restrict__ rho_next, int32_t* __restrict__ e_next, float* __restrict__ scores) {
   __shared__ float u[W], hb[W], logit[kMaxBudgets];
-  __shared__ float su[kSelWarps][W];
+  __shared__ float sck[SH], sw2s[SH];
   __shared__ int s_budget;
   const int i = blockIdx.x, t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int lo = cu[i], hi = cu[i + 1];
@@ -200,16 +216,23 @@ __global__ void __launch_bounds__(256) budget_select_kernel(
     }
   }
   __syncthreads();
-  if (t < W) {
-    float a = ld(bb1, t);
-    for (int c = 0; c < W; ++c) a = fmaf(ld(bw1, static_cast<size_t>(t) * W + c), u[c], a);
-    hb[t] = gelu(a);
+  // each output one warp's dot product over 128, the lanes striding along it
+  for (int h = warp; h < W; h += kSelWarps) {
+    float a = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) a = fmaf(ld(bw1, static_cast<size_t>(h) * W + lane + 32 * q),
+                                          u[lane + 32 * q], a);
+    a = warp_sum(a);
+    if (lane == 0) hb[h] = gelu(a + ld(bb1, h));
   }
   __syncthreads();
-  for (int m = t; m < m_out; m += blockDim.x) {
-    float a = ld(bb2, m);
-    for (int c = 0; c < W; ++c) a = fmaf(ld(bw2, static_cast<size_t>(m) * W + c), hb[c], a);
-    logit[m] = a;
+  for (int m = warp; m < m_out; m += kSelWarps) {
+    float a = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) a = fmaf(ld(bw2, static_cast<size_t>(m) * W + lane + 32 * q),
+                                          hb[lane + 32 * q], a);
+    a = warp_sum(a);
+    if (lane == 0) logit[m] = a + ld(bb2, m);
   }
   __syncthreads();
   if (t == 0) {
@@ -233,28 +256,30 @@ __global__ void __launch_bounds__(256) budget_select_kernel(
     scores[lo] = 0.f;
   }
   __syncthreads();
-  // selector: warp w scores visual tokens 1 + w, 1 + w + 8, ...; each lane
-  // owns two of the 64 hidden units
+  // selector tail: one thread per visual token, s = w_2 . silu(S1_j + (k / N_l)
+  // W_1 W_k) + b_2, with S1_j = W_1 Z_j + b_1 from the GEMM
   const float kr = n > 0 ? static_cast<float>(s_budget) / n : 0.f;
-  for (int j = 1 + warp; j <= n; j += kSelWarps) {
-    const size_t zr = static_cast<size_t>(lo + j) * W;
+  if (t < SH) {
+    sck[t] = kr * sel_wk[t];
+    sw2s[t] = ld(sw2, t);
+  }
+  __syncthreads();
+  const float b2 = ld(sb2, 0);
+  for (int j = 1 + t; j <= n; j += blockDim.x) {
+    const uint4* sr = reinterpret_cast<const uint4*>(s1 + static_cast<size_t>(lo + j) * SH);
+    float acc = 0.f;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int c = lane + 32 * q;
-      su[warp][c] = ld(z, zr + c) + ld(w_k, c) * kr;
-    }
-    __syncwarp();
-    float part = 0.f;
+    for (int q = 0; q < SH / 8; ++q) {
+      const uint4 v = sr[q];
+      const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int q = 0; q < SH / 32; ++q) {
-      const int hh = lane + 32 * q;
-      float a = ld(sb1, hh);
-      for (int c = 0; c < W; ++c) a = fmaf(ld(sw1, static_cast<size_t>(hh) * W + c), su[warp][c], a);
-      part += ld(sw2, hh) * silu(a);
+      for (int e = 0; e < 4; ++e) {
+        const int hh = 8 * q + 2 * e;
+        acc = fmaf(sw2s[hh], silu(__uint_as_float(wv[e] << 16) + sck[hh]), acc);
+        acc = fmaf(sw2s[hh + 1], silu(__uint_as_float(wv[e] & 0xFFFF0000u) + sck[hh + 1]), acc);
+      }
     }
-    part = warp_sum(part);
-    if (lane == 0) scores[lo + j] = part + ld(sb2, 0);
-    __syncwarp();
+    scores[lo + j] = acc + b2;
   }
 }
 
@@ -264,7 +289,8 @@ __global__ void __launch_bounds__(256) budget_select_kernel(
 size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
 
 struct Prep {
-  size_t bias_in, wqkv_f, cqkv_f, dqkv_f, wqkv_p, cqkv_p, dqkv_p, wo_p, wfc1, cfc1, dfc1, total;
+  size_t bias_in, wqkv_f, cqkv_f, dqkv_f, wqkv_p, cqkv_p, dqkv_p, wo_p, wfc1, cfc1, dfc1, sel_wk,
+      total;
 };
 
 Prep prep_layout(const dora_actor_weights* w) {
@@ -281,12 +307,13 @@ Prep prep_layout(const dora_actor_weights* w) {
   P.wfc1 = off;    off += up256(FF * W * 2);
   P.cfc1 = off;    off += up256(FF * 4);
   P.dfc1 = off;    off += up256(FF * 4);
+  P.sel_wk = off;  off += up256(SH * 4);
   P.total = off;
   return P;
 }
 
 struct Ws {
-  size_t status, x, mv, qkv, o, z1, sm, f, z, glogit, prep, total;
+  size_t status, x, mv, qkv, o, z1, sm, f, z, s1, glogit, prep, total;
 };
 
 Ws ws_layout(int32_t t_cap, int32_t batch, const dora_actor_weights* w) {
@@ -302,6 +329,7 @@ Ws ws_layout(int32_t t_cap, int32_t batch, const dora_actor_weights* w) {
   L.sm = off;     off += up256(t * 2 * 8);
   L.f = off;      off += up256(t * FF * 2);
   L.z = off;      off += up256(t * W * 2);
+  L.s1 = off;     off += up256(t * SH * 2);
   L.glogit = off; off += up256(b * 4);
   L.prep = off;   off += w->prepared != nullptr ? 0 : prep_layout(w).total;
   L.total = off;
@@ -340,6 +368,7 @@ cudaError_t prepare(const dora_actor_weights* w, uint8_t* prep, cudaStream_t str
   pad_wo_kernel<<<W, 256, 0, stream>>>(w->enc_w_o, reinterpret_cast<uint16_t*>(prep + P.wo_p));
   bias_in_kernel<<<w->depth, W, 0, stream>>>(w->enc_b_in, w->enc_emb,
                                              reinterpret_cast<uint16_t*>(prep + P.bias_in));
+  sel_wk_kernel<<<1, SH, 0, stream>>>(w->sel_w1, w->sel_w_k, reinterpret_cast<float*>(prep + P.sel_wk));
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   return launch_fold_ln(w->enc_w_fc1, FF, W, w->enc_ln2_w, w->enc_ln2_b, w->enc_b_fc1,
@@ -472,11 +501,17 @@ int dora_actor(const dora_bf16* qkv, const int32_t* cu, int32_t batch, int32_t m
       launch_linear(f, t_cap, rows, FF, w->enc_w_fc2, W, DORA_EPI_BIAS_RESIDUAL, e_f2, z, status,
                     stream) != cudaSuccess)
     return DORA_ERR_CUDA;
-  // budget and selector
+  // selector's first layer on every token, then budget head and selector tail
+  uint16_t* s1 = reinterpret_cast<uint16_t*>(ws + L.s1);
+  LinearEpi e_s;
+  e_s.bias = w->sel_b1;
+  if (launch_linear(z, t_cap, rows, W, w->sel_w1, SH, DORA_EPI_BIAS, e_s, s1, status, stream) !=
+      cudaSuccess)
+    return DORA_ERR_CUDA;
   budget_select_kernel<<<batch, 256, 0, stream>>>(
       z, cu, t_cap, w->n0, w->eps, w->bud_ln_w, w->bud_ln_b, w->bud_w1, w->bud_b1, w->bud_w2,
-      w->bud_b2, w->sel_w_k, w->sel_w1, w->sel_b1, w->sel_w2, w->sel_b2, glogit, interventions,
-      gate, budget, k, keep_counts, rho_next, interventions_next, scores);
+      w->bud_b2, s1, reinterpret_cast<const float*>(prep + P.sel_wk), w->sel_w2, w->sel_b2,
+      glogit, interventions, gate, budget, k, keep_counts, rho_next, interventions_next, scores);
   return cudaGetLastError() == cudaSuccess ? DORA_OK : DORA_ERR_CUDA;
 }
 

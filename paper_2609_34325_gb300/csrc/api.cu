@@ -418,13 +418,28 @@ size_t dora_workspace_size(int32_t t_cap, int32_t batch, const dora_block_weight
 
 int32_t* dora_workspace_status(void* workspace) { return static_cast<int32_t*>(workspace); }
 
-int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t* ids_in,
-                      int32_t batch, int32_t max_seqlen, int32_t t_cap,
-                      const dora_block_weights* w, const float* scores,
-                      const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
-                      int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
-                      float* x_out_moments, void* workspace, size_t workspace_bytes,
-                      dora_stream_t stream_) {
+// The actor run inside the block (dora_pruned_block_actor): its scores and,
+// unless the caller gives keep counts, its keep counts drive the deletion.
+struct ActorHook {
+  const dora_actor_weights* aw;
+  int32_t block;
+  const float* rho;
+  const int32_t* interventions;
+  int32_t *gate, *budget, *k, *keep;
+  float* scores;
+  float* rho_next;
+  int32_t* interventions_next;
+  void* ws;
+  size_t ws_bytes;
+};
+
+static int pruned_block_impl(const dora_bf16* x_in, const int32_t* cu_in, const int32_t* ids_in,
+                             int32_t batch, int32_t max_seqlen, int32_t t_cap,
+                             const dora_block_weights* w, const float* scores,
+                             const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
+                             int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
+                             float* x_out_moments, void* workspace, size_t workspace_bytes,
+                             dora_stream_t stream_, const ActorHook* hook) {
   DORA_CHECK_ARG(weights_ok(w));
   DORA_CHECK_ARG(batch >= 0 && batch <= 65535 && t_cap >= 0 && max_seqlen >= 0);
   DORA_CHECK_ARG(max_seqlen <= kMaxSeqlenSelect);
@@ -433,6 +448,7 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
   DORA_CHECK_ARG((reinterpret_cast<uintptr_t>(workspace) & 255u) == 0);
   DORA_CHECK_ARG(aligned8(x_in_moments) && aligned8(x_out_moments));
   if (scores) DORA_CHECK_ARG(keep_counts && cu_out && ids_in && ids_out);
+  if (hook) DORA_CHECK_ARG(!scores && cu_out && ids_in && ids_out && hook->scores && hook->keep);
   const WsLayout L = ws_layout(t_cap, w);
   DORA_CHECK_ARG(workspace_bytes >= L.total);
   DORA_CHECK_DEVICE();
@@ -461,7 +477,7 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
   const FoldLayout F = fold_layout(w);
   LinearEpi e_qkv, e_proj, e_fc1, e_fc2;
   e_qkv.stats_in = x_in_moments ? x_in_moments : mv;
-  e_fc1.stats_in = scores ? mv2 : mv;
+  e_fc1.stats_in = (scores || hook) ? mv2 : mv;      // the kept rows' moments after a deletion
   e_qkv.eps = e_fc1.eps = w->ln_eps;
   e_proj.slices = d / kSliceCols;
   e_qkv.colsum = reinterpret_cast<const float*>(fold + F.cqkv);
@@ -490,6 +506,18 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
     return DORA_ERR_CUDA;
   if (launch_merge_moments(sm, t_cap, rows_in, d / kSliceCols, mv, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
+  // the actor reads this block's keys (Sec. 3.2; deletion follows the
+  // attention residual, Eq. 1)
+  if (hook != nullptr) {
+    const int rc = dora_actor(qkv, cu_in, batch, max_seqlen, t_cap, hook->block, hook->aw,
+                              hook->rho, hook->interventions, nullptr, hook->gate, hook->budget,
+                              hook->k, hook->keep, hook->scores, hook->rho_next,
+                              hook->interventions_next, nullptr, hook->ws, hook->ws_bytes,
+                              stream_);
+    if (rc != DORA_OK) return rc;
+    scores = hook->scores;
+    if (keep_counts == nullptr) keep_counts = hook->keep;
+  }
   // H_keep: delete and compact, carrying the row moments of LayerNorm'
   const uint16_t* hk = hattn;
   const int32_t* rows_mid = rows_in;
@@ -516,6 +544,37 @@ int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t
           cudaSuccess)
     return DORA_ERR_CUDA;
   return DORA_OK;
+}
+
+int dora_pruned_block(const dora_bf16* x_in, const int32_t* cu_in, const int32_t* ids_in,
+                      int32_t batch, int32_t max_seqlen, int32_t t_cap,
+                      const dora_block_weights* w, const float* scores,
+                      const int32_t* keep_counts, dora_bf16* x_out, int32_t* cu_out,
+                      int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
+                      float* x_out_moments, void* workspace, size_t workspace_bytes,
+                      dora_stream_t stream) {
+  return pruned_block_impl(x_in, cu_in, ids_in, batch, max_seqlen, t_cap, w, scores, keep_counts,
+                           x_out, cu_out, ids_out, kept_idx, x_in_moments, x_out_moments,
+                           workspace, workspace_bytes, stream, nullptr);
+}
+
+int dora_pruned_block_actor(const dora_bf16* x_in, const int32_t* cu_in, const int32_t* ids_in,
+                            int32_t batch, int32_t max_seqlen, int32_t t_cap,
+                            const dora_block_weights* w, dora_bf16* x_out, int32_t* cu_out,
+                            int32_t* ids_out, int32_t* kept_idx, const float* x_in_moments,
+                            float* x_out_moments, void* workspace, size_t workspace_bytes,
+                            const dora_actor_weights* aw, int32_t block, const float* rho,
+                            const int32_t* interventions, const int32_t* keep_counts,
+                            int32_t* gate, int32_t* budget, int32_t* k, int32_t* actor_keep,
+                            float* scores, float* rho_next, int32_t* interventions_next,
+                            void* actor_workspace, size_t actor_workspace_bytes,
+                            dora_stream_t stream) {
+  DORA_CHECK_ARG(aw != nullptr && aw->dim == (w ? w->dim : -1));
+  const ActorHook hook{aw, block, rho, interventions, gate, budget, k, actor_keep, scores,
+                       rho_next, interventions_next, actor_workspace, actor_workspace_bytes};
+  return pruned_block_impl(x_in, cu_in, ids_in, batch, max_seqlen, t_cap, w, nullptr,
+                           keep_counts, x_out, cu_out, ids_out, kept_idx, x_in_moments,
+                           x_out_moments, workspace, workspace_bytes, stream, &hook);
 }
 
 int dora_read_status(const int32_t* status_dev, int32_t* code) {

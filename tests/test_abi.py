@@ -106,9 +106,10 @@ def test_actor_struct_sizes_and_host_checks(lib):
     prep = lib.dora_actor_prepared_size(ctypes.byref(w))
     assert prep > 0
     # per row: X, Z1, Z (128 bf16 each), padded qkv (768), attention out (256),
-    # feed-forward (256), row moments and two slice moments; per image the gate logit
+    # feed-forward (256), selector hidden (64), row moments and two slice
+    # moments; per image the gate logit
     t, b = 50000, 256
-    per_rows = t * (3 * 256 + 1536 + 512 + 512 + 8 + 16) + 4 * b
+    per_rows = t * (3 * 256 + 1536 + 512 + 512 + 128 + 8 + 16) + 4 * b
     n = lib.dora_actor_workspace_size(t, b, ctypes.byref(w))
     assert per_rows + prep <= n < per_rows + prep + 16 * 256
     w.prepared = 256

@@ -951,3 +951,67 @@ def test_actor_edges_short_images_and_gate_bias():
         assert np.array_equal(got["keep"], lens - got["k"])
         assert np.all(got["k"][~feasible] == 0)
         _check_actor(cfg, cu, qkv, rho, e_prev, wa, got, 0, [0, 1, 2, 3, 4, 6, 7])
+
+
+@pytest.mark.parametrize("given_counts", [True, False])
+def test_block_with_actor_equals_actor_then_block(given_counts):
+    """dora_pruned_block_actor gives the same bits as running dora_actor on the
+    block's QKV output (computed through the public entries) and then
+    dora_pruned_block with the actor's scores and the given (or the actor's)
+    keep counts."""
+    cfg = S.get_config("cfg2")
+    cu, ids = S.initial_layout(cfg)
+    t = int(cu[-1])
+    x = S.activations_bf16(cfg, 27)
+    wb = S.block_weights(cfg, 0, 27, random_affine=True)
+    wf = _device_weights(cfg, wb).fold()
+    wa = S.actor_weights(cfg.dim, cfg.depth, cfg.n_vis0, 27, gate_bias=1.0)
+    aw = P.ActorWeights({k_: bf(v) for k_, v in wa.items()}, cfg.dim, cfg.depth, cfg.n_vis0).prepare()
+    keeps, _ = S.keep_schedule(cfg, 27)
+    b = cfg.batch
+    i32z = lambda n: torch.zeros(n, dtype=torch.int32, device=dev())
+    rho = torch.zeros(b, dtype=torch.float32, device=dev())
+    e0 = i32z(b)
+    ws = P.alloc_workspace(t, b, wf)
+    aws = P.alloc_actor_workspace(t, b, aw)
+    # the block with the actor inside
+    out = {n: i32z(b) for n in ("gate", "budget", "k", "keep")}
+    scores = torch.zeros(t, dtype=torch.float32, device=dev())
+    x_out = torch.zeros(t, cfg.dim, dtype=torch.bfloat16, device=dev())
+    cu_out, ids_out = i32z(b + 1), i32z(t)
+    P.dora_pruned_block_actor(bf(x), i32(cu), wf, cfg.n_tokens, x_out, ws, aw, 0, rho, e0,
+                              out["gate"], out["budget"], out["k"], out["keep"], scores, aws,
+                              i32(ids), cu_out, ids_out,
+                              keep_counts=i32(keeps[0]) if given_counts else None)
+    torch.cuda.synchronize()
+    assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+    assert P.dora_read_status(P.dora_workspace_status(aws)) == 0
+    # the same through the public entries
+    W = {k_: bf(v) for k_, v in wb.items()}
+    mv = torch.zeros(t, 2, dtype=torch.float32, device=dev())
+    P.dora_row_stats(bf(x), mv)
+    wq = torch.zeros(3 * cfg.dim, cfg.dim, dtype=torch.bfloat16, device=dev())
+    cq = torch.zeros(3 * cfg.dim, dtype=torch.float32, device=dev())
+    dq = torch.zeros(3 * cfg.dim, dtype=torch.float32, device=dev())
+    P.dora_fold_ln_linear(W["w_qkv"], W["ln1_w"], W["ln1_b"], wq, cq, dq, bias=W["b_qkv"])
+    qkv = torch.zeros(t, 3 * cfg.dim, dtype=torch.bfloat16, device=dev())
+    P.dora_linear_ln(bf(x), mv, cfg.ln_eps, wq, cq, dq, qkv)
+    ref = {n: i32z(b) for n in ("gate", "budget", "k", "keep")}
+    scores2 = torch.zeros(t, dtype=torch.float32, device=dev())
+    P.dora_actor(qkv, i32(cu), aw, 0, cfg.n_tokens, rho, e0, ref["gate"], ref["budget"], ref["k"],
+                 ref["keep"], scores2, P.alloc_actor_workspace(t, b, aw))
+    for n in ref:
+        assert torch.equal(out[n], ref[n]), n
+    assert torch.equal(scores, scores2)
+    x_out2 = torch.zeros(t, cfg.dim, dtype=torch.bfloat16, device=dev())
+    cu2, ids2 = i32z(b + 1), i32z(t)
+    P.dora_pruned_block(bf(x), i32(cu), wf, cfg.n_tokens, x_out2, P.alloc_workspace(t, b, wf),
+                        ids_in=i32(ids), scores=scores2,
+                        keep_counts=i32(keeps[0]) if given_counts else ref["keep"],
+                        cu_out=cu2, ids_out=ids2)
+    torch.cuda.synchronize()
+    assert torch.equal(cu_out, cu2) and torch.equal(ids_out, ids2)
+    t_out = int(cu2[-1].item())
+    assert torch.equal(x_out[:t_out], x_out2[:t_out])
+    if not given_counts:
+        assert torch.equal(torch.diff(cu_out), out["keep"])
