@@ -41,6 +41,7 @@ __all__ = [
     "uniform_f32", "normal_f64", "f32_to_bf16_bits", "bf16_bits_to_f32",
     "activations_bf16", "block_weights", "score_table", "keep_schedule",
     "initial_layout", "compression_from_counts", "actor_weights", "ACTOR_SHAPES",
+    "images_bf16", "embed_head_weights",
 ]
 
 _M64 = np.uint64(0xFFFFFFFFFFFFFFFF)
@@ -56,6 +57,8 @@ TAG_KEEP = 4       # per-image budget law draws
 TAG_BUMP = 5       # cfg5 bump centre / width
 TAG_LNAFF = 6      # optional random LayerNorm affine (tests)
 TAG_ACTOR = 7      # + (which << 8): actor weights
+TAG_IMG = 8        # input images
+TAG_EMBHEAD = 9    # + (which << 8): patch embedding and classifier weights
 
 
 def splitmix64(x: np.ndarray) -> np.ndarray:
@@ -366,4 +369,41 @@ def actor_weights(dim: int, depth: int, n0: int, seed: int = 0, gate_bias: float
             out[name] = f32_to_bf16_bits(v).reshape(shape)
         else:
             out[name] = _normal_bf16(seed, tag, count, 1.0 / np.sqrt(shape[1])).reshape(shape)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# input images and the forward's two ends (patch embedding, classifier)
+# ---------------------------------------------------------------------------
+
+def images_bf16(cfg: Config, seed: int = 0, patch: int = 16, channels: int = 3) -> np.ndarray:
+    """bf16 bit patterns of N(0, 1) images [B, C, H, W] with H = W = patch *
+    sqrt(n_vis0) (224 for 196 visual tokens): normalised pixels, as a
+    preprocessing pipeline hands them to the model."""
+    g = int(round(np.sqrt(cfg.n_vis0)))
+    assert g * g == cfg.n_vis0
+    side = g * patch
+    count = cfg.batch * channels * side * side
+    return _normal_bf16(seed, TAG_IMG, count, 1.0).reshape(cfg.batch, channels, side, side)
+
+
+def embed_head_weights(cfg: Config, seed: int = 0, patch: int = 16, channels: int = 3,
+                       classes: int = 1000) -> dict:
+    """bf16 bit patterns of the patch embedding (w_pe [d, C patch^2], b_pe, cls,
+    pos [N, d]) and the classifier (norm_w, norm_b, w_head [classes, d],
+    b_head), randomly initialised."""
+    d, k = cfg.dim, channels * patch * patch
+    shapes = {"w_pe": (d, k), "b_pe": (d,), "cls": (d,), "pos": (cfg.n_tokens, d),
+              "norm_w": (d,), "norm_b": (d,), "w_head": (classes, d), "b_head": (classes,)}
+    out = {}
+    for which, (name, shape) in enumerate(shapes.items()):
+        count = int(np.prod(shape))
+        tag = TAG_EMBHEAD + (which << 8)
+        if name in ("w_pe", "w_head"):
+            out[name] = _normal_bf16(seed, tag, count, 1.0 / np.sqrt(shape[1])).reshape(shape)
+        else:
+            v = normal_f64(seed, tag, np.arange(count, dtype=np.uint64)) * (0.1 if name.startswith("norm") else 0.02)
+            if name == "norm_w":
+                v = v + 1.0
+            out[name] = f32_to_bf16_bits(v).reshape(shape)
     return out

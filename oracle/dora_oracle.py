@@ -26,6 +26,10 @@ block of Eq. 1 (Sec. 3.1), in float64, from bf16/fp32 inputs decoded exactly:
   ``actor_block``   the deterministic actor that produces each block's gate,
                     removal count and deletion scores (Sec. 3.2 "The actor";
                     Appendix A.1-A.3).
+* ``patch_embed``, ``classifier_head``  the forward's two ends, which the
+                    paper's GFLOPs and throughput include (App. E.4): the
+                    strided patch convolution with CLS and position
+                    embeddings, and LayerNorm + linear on each CLS row.
 
 Readings where the paper is silent (all listed in the design doc):
 
@@ -457,3 +461,35 @@ def actor_block(keys: np.ndarray, cu: np.ndarray, block: int, n0: int, depth: in
                 scores=scores, z=z, logits=logits,
                 rho_next=np.where(gate == 1, k / np.maximum(n_vis, 1), 0.0),
                 interventions_next=np.asarray(interventions) + gate)
+
+
+# ----------------------------------------------------------------------------
+# O7: the two ends of the forward (backbones of Sec. 4.1; App. E.4 counts them)
+# ----------------------------------------------------------------------------
+
+def patch_embed(images: np.ndarray, w_pe: np.ndarray, b_pe: np.ndarray, cls: np.ndarray,
+                pos: np.ndarray, patch: int) -> np.ndarray:
+    """ViT input tokens: a patch x patch convolution with stride patch (weights
+    [d, C, patch, patch] stored as [d, C * patch * patch]), then each image's
+    CLS token prepended and the position embeddings added.  ``images``
+    [B, C, H, W] (bf16 bits or float); returns [B * (g_h g_w + 1), d] packed
+    image after image, row 0 of each image its CLS token."""
+    im = bf16_to_f64(images) if np.asarray(images).dtype == np.uint16 else np.asarray(images,
+                                                                                     np.float64)
+    b, c, h, w = im.shape
+    gh, gw = h // patch, w // patch
+    p = im.reshape(b, c, gh, patch, gw, patch).transpose(0, 2, 4, 1, 3, 5)
+    p = p.reshape(b * gh * gw, c * patch * patch)
+    d = w_pe.shape[0]
+    emb = linear(p, w_pe, b_pe).reshape(b, gh * gw, d) + pos[1:]
+    out = np.concatenate([np.broadcast_to(cls + pos[0], (b, 1, d)), emb], axis=1)
+    return out.reshape(b * (gh * gw + 1), d)
+
+
+def classifier_head(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.ndarray,
+                    eps: float, w_head: np.ndarray, b_head: np.ndarray) -> np.ndarray:
+    """The classifier of a CLS-readout ViT: the final LayerNorm on each image's
+    CLS row (row cu[i]) and a linear layer to the class logits [B, classes]."""
+    x = np.asarray(x, dtype=np.float64)
+    rows = np.asarray(cu[:-1], dtype=np.int64)
+    return linear(layernorm(x[rows], ln_w, ln_b, eps), w_head, b_head)

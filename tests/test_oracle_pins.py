@@ -568,3 +568,57 @@ def test_actor_block_decisions_and_history():
         assert np.allclose(r["rho_next"], r["k"] / n_vis)
         assert np.array_equal(r["interventions_next"], e_prev + r["gate"])
         assert np.all(r["scores"][cu[:-1]] == 0.0)
+
+
+# ---------------------------------------------------------------------------
+# patch embedding and classifier (the ends of the forward that App. E.4 counts)
+# ---------------------------------------------------------------------------
+
+def test_patch_embed_is_a_strided_convolution():
+    """Every token against a direct convolution written as loops, plus the CLS
+    row and the position embeddings."""
+    rng = np.random.default_rng(11)
+    b, c, h, w, p, d = 2, 2, 8, 12, 4, 3
+    im = rng.standard_normal((b, c, h, w))
+    wc = rng.standard_normal((d, c, p, p))
+    bias = rng.standard_normal(d)
+    cls = rng.standard_normal(d)
+    gh, gw = h // p, w // p
+    pos = rng.standard_normal((gh * gw + 1, d))
+    out = O.patch_embed(im, wc.reshape(d, -1), bias, cls, pos, p)
+    assert out.shape == (b * (gh * gw + 1), d)
+    for i in range(b):
+        base = i * (gh * gw + 1)
+        assert np.allclose(out[base], cls + pos[0], rtol=0, atol=1e-14)
+        for py in range(gh):
+            for px in range(gw):
+                for o in range(d):
+                    acc = bias[o]
+                    for ch in range(c):
+                        for ky in range(p):
+                            for kx in range(p):
+                                acc += wc[o, ch, ky, kx] * im[i, ch, py * p + ky, px * p + kx]
+                    tok = 1 + py * gw + px
+                    assert abs(out[base + tok, o] - (acc + pos[tok, o])) < 1e-12
+
+
+def test_classifier_reads_only_cls_rows():
+    """Logits depend on each image's CLS row alone (LayerNorm then linear):
+    changing every other row leaves them unchanged; with a unit LayerNorm and
+    an identity head the logits are the normalised CLS row."""
+    rng = np.random.default_rng(12)
+    d = 8
+    cu = np.array([0, 5, 6, 10])
+    x = rng.standard_normal((10, d))
+    g, be = 1 + 0.1 * rng.standard_normal(d), 0.1 * rng.standard_normal(d)
+    wh, bh = rng.standard_normal((4, d)), rng.standard_normal(4)
+    a = O.classifier_head(x, cu, g, be, 1e-6, wh, bh)
+    x2 = x.copy()
+    mask = np.ones(10, bool)
+    mask[cu[:-1]] = False
+    x2[mask] = rng.standard_normal((mask.sum(), d))
+    assert np.array_equal(a, O.classifier_head(x2, cu, g, be, 1e-6, wh, bh))
+    ident = O.classifier_head(x, cu, np.ones(d), np.zeros(d), 0.0, np.eye(d), np.zeros(d))
+    r = x[cu[:-1]]
+    ref = (r - r.mean(1, keepdims=True)) / r.std(1, keepdims=True)
+    assert np.allclose(ident, ref, rtol=0, atol=1e-12)
