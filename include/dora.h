@@ -502,6 +502,47 @@ int dora_pruned_block_actor(const dora_bf16* x_in, const int32_t* cu_in, const i
                             void* actor_workspace, size_t actor_workspace_bytes,
                             dora_stream_t stream);
 
+/*
+ * The two ends of the forward, which the paper's GFLOPs and throughput count
+ * (App. E.4): patch embedding and the classifier head.
+ *
+ * dora_patch_embed -- images bf16 [batch, channels, height, width] (NCHW) to
+ * the packed tokens x0 bf16 [batch * (g + 1), dim], g = (height / patch) *
+ * (width / patch): row 0 of each image is cls + pos[0], row 1 + p the patch
+ * p (row-major over the patch grid) embedded by the patch x patch, stride
+ * patch convolution (w_pe bf16 [dim, channels * patch * patch], the
+ * [dim, C, p, p] kernel flattened; b_pe bf16 [dim], nullable) plus pos[1 + p]
+ * (pos bf16 [g + 1, dim]; cls bf16 [dim]).  patch % 8 == 0, height and
+ * width multiples of patch, channels * patch^2 % 64 == 0, dim % 64 == 0.
+ * The convolution is a relayout (patchify) and one tcgen05 GEMM with fp32
+ * accumulation (its output rounded to bf16), then the position add.
+ * workspace: dora_embed_workspace_size bytes, 256-byte aligned; its first
+ * word is a status word.
+ */
+size_t dora_embed_workspace_size(int32_t batch, int32_t channels, int32_t height, int32_t width,
+                                 int32_t patch, int32_t dim);
+int dora_patch_embed(const dora_bf16* images, int32_t batch, int32_t channels, int32_t height,
+                     int32_t width, int32_t patch, int32_t dim, const dora_bf16* w_pe,
+                     const dora_bf16* b_pe, const dora_bf16* cls, const dora_bf16* pos,
+                     dora_bf16* x0, void* workspace, size_t workspace_bytes, dora_stream_t stream);
+
+/*
+ * dora_classifier_head -- logits bf16 [batch, classes] = LayerNorm(x[cu[i]])
+ * W_head^T + b_head for each image i: the final LayerNorm (norm_w, norm_b
+ * bf16 [dim], epsilon eps, biased variance, fp32) on the CLS row, then a
+ * tcgen05 GEMM (w_head bf16 [classes, dim]; b_head bf16 [classes], nullable).
+ * classes % 32 == 0 (pad the head with zero rows), dim % 64 == 0; x bf16
+ * [t_cap, dim] packed, cu int32 [batch + 1].  An empty image gives the
+ * logits of a zero row.  workspace: dora_head_workspace_size bytes,
+ * 256-byte aligned, status word first.
+ */
+size_t dora_head_workspace_size(int32_t batch, int32_t dim);
+int dora_classifier_head(const dora_bf16* x, const int32_t* cu, int32_t batch, int32_t t_cap,
+                         int32_t dim, const dora_bf16* norm_w, const dora_bf16* norm_b,
+                         float eps, const dora_bf16* w_head, const dora_bf16* b_head,
+                         int32_t classes, dora_bf16* logits, void* workspace,
+                         size_t workspace_bytes, dora_stream_t stream);
+
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug
  * only: it blocks the host. */

@@ -23,7 +23,8 @@ __all__ = [
     "dora_fold_ln_linear", "dora_linear_ln", "dora_linear_residual_stats",
     "dora_folded_weights_size", "dora_fold_block_weights", "dora_compact_stats",
     "dora_merge_moments", "ActorWeights", "dora_actor", "dora_actor_workspace_size",
-    "alloc_actor_workspace", "dora_pruned_block_actor",
+    "alloc_actor_workspace", "dora_pruned_block_actor", "dora_patch_embed",
+    "dora_classifier_head",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -70,6 +71,12 @@ _SIGS = {
     "dora_actor_prepare": (ctypes.c_int, [_vp, _vp, _sz, _vp]),
     "dora_actor": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp,
                                   _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "dora_embed_workspace_size": (_sz, [_i32, _i32, _i32, _i32, _i32, _i32]),
+    "dora_patch_embed": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp,
+                                        _vp, _vp, _vp, _sz, _vp]),
+    "dora_head_workspace_size": (_sz, [_i32, _i32]),
+    "dora_classifier_head": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _f32, _vp, _vp,
+                                            _i32, _vp, _vp, _sz, _vp]),
     "dora_pruned_block_actor": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
                                                _vp, _vp, _vp, _vp, _vp, _sz, _vp, _i32, _vp, _vp,
                                                _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
@@ -594,3 +601,55 @@ def dora_pruned_block_actor(x_in, cu_in, weights: BlockWeights, max_seqlen, x_ou
         _ptr(gate), _ptr(budget), _ptr(k), _ptr(actor_keep), _ptr(scores), _ptr(rho_next),
         _ptr(interventions_next), _ptr(actor_workspace), actor_workspace.numel(),
         _stream(stream)), "dora_pruned_block_actor")
+
+
+# ---------------------------------------------------------------------------
+# the forward's two ends
+# ---------------------------------------------------------------------------
+
+def dora_patch_embed(images, w_pe, b_pe, cls, pos, patch, x0, workspace=None, stream=None):
+    """Packed tokens x0 [B * (g + 1), d] from images [B, C, H, W]: strided patch
+    convolution (w_pe [d, C * patch^2]), CLS first, position embeddings added."""
+    for n, t in (("images", images), ("w_pe", w_pe), ("cls", cls), ("pos", pos), ("x0", x0)):
+        _req(t, torch.bfloat16, n)
+    _req(b_pe, torch.bfloat16, "b_pe", optional=True)
+    b, c, h, w = images.shape
+    d = w_pe.shape[0]
+    n = int(load_library().dora_embed_workspace_size(b, c, h, w, int(patch), d))
+    if workspace is None:
+        workspace = torch.zeros(n, dtype=torch.uint8, device=images.device)
+    _req(workspace, torch.uint8, "workspace")
+    g = (h // patch) * (w // patch)
+    if tuple(x0.shape) != (b * (g + 1), d) or tuple(pos.shape) != (g + 1, d):
+        raise ValueError("x0 must be [B * (g + 1), d] and pos [g + 1, d]")
+    _check(load_library().dora_patch_embed(_ptr(images), b, c, h, w, int(patch), d, _ptr(w_pe),
+                                           _ptr(b_pe), _ptr(cls), _ptr(pos), _ptr(x0),
+                                           _ptr(workspace), workspace.numel(), _stream(stream)),
+           "dora_patch_embed")
+    return workspace
+
+
+def dora_classifier_head(x, cu, norm_w, norm_b, eps, w_head, b_head, logits, workspace=None,
+                         stream=None):
+    """logits [B, classes] = LayerNorm(x[cu[i]]) W_head^T + b_head per image
+    (classes a multiple of 32: pad the head with zero rows)."""
+    for n, t in (("x", x), ("norm_w", norm_w), ("norm_b", norm_b), ("w_head", w_head),
+                 ("logits", logits)):
+        _req(t, torch.bfloat16, n)
+    _req(b_head, torch.bfloat16, "b_head", optional=True)
+    _req(cu, torch.int32, "cu")
+    t_cap, d = x.shape
+    b = cu.numel() - 1
+    classes = w_head.shape[0]
+    n = int(load_library().dora_head_workspace_size(b, d))
+    if workspace is None:
+        workspace = torch.zeros(n, dtype=torch.uint8, device=x.device)
+    _req(workspace, torch.uint8, "workspace")
+    if tuple(logits.shape) != (b, classes):
+        raise ValueError("logits must be [B, classes]")
+    _check(load_library().dora_classifier_head(_ptr(x), _ptr(cu), b, t_cap, d, _ptr(norm_w),
+                                               _ptr(norm_b), float(eps), _ptr(w_head),
+                                               _ptr(b_head), classes, _ptr(logits),
+                                               _ptr(workspace), workspace.numel(),
+                                               _stream(stream)), "dora_classifier_head")
+    return workspace

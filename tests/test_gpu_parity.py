@@ -1015,3 +1015,54 @@ def test_block_with_actor_equals_actor_then_block(given_counts):
     assert torch.equal(x_out[:t_out], x_out2[:t_out])
     if not given_counts:
         assert torch.equal(torch.diff(cu_out), out["keep"])
+
+
+# ---------------------------------------------------------------------------
+# patch embedding and classifier head (the ends of the forward, App. E.4)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("b,c,h,w,patch,d", [(8, 3, 224, 224, 16, 192), (3, 3, 64, 96, 16, 768),
+                                             (2, 4, 32, 32, 8, 128)])
+def test_patch_embed_matches_oracle(b, c, h, w, patch, d):
+    rng = np.random.default_rng(b * 100 + d)
+    g = (h // patch) * (w // patch)
+    k = c * patch * patch
+    im = S.f32_to_bf16_bits(rng.standard_normal((b, c, h, w)))
+    wpe = S.f32_to_bf16_bits(rng.standard_normal((d, k)) / np.sqrt(k))
+    bpe = S.f32_to_bf16_bits(0.02 * rng.standard_normal(d))
+    cls = S.f32_to_bf16_bits(0.02 * rng.standard_normal(d))
+    pos = S.f32_to_bf16_bits(0.02 * rng.standard_normal((g + 1, d)))
+    x0 = torch.full((b * (g + 1), d), 9.0, dtype=torch.bfloat16, device=dev())
+    ws = P.dora_patch_embed(bf(im), bf(wpe), bf(bpe), bf(cls), bf(pos), patch, x0)
+    torch.cuda.synchronize()
+    assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+    ref = O.patch_embed(im, O.bf16_to_f64(wpe), O.bf16_to_f64(bpe), O.bf16_to_f64(cls),
+                        O.bf16_to_f64(pos), patch)
+    assert_close(f64(x0), ref, f"patch embed {b}x{c}x{h}x{w}/{patch} d={d}")
+
+
+@pytest.mark.parametrize("name", ["cfg1", "cfg3"])
+def test_classifier_head_matches_oracle(name):
+    cfg = S.get_config(name)
+    keeps, _ = S.keep_schedule(cfg, 13)
+    lens = keeps[-1]
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    rng = np.random.default_rng(13)
+    x = S.f32_to_bf16_bits(rng.uniform(-3, 3, (t, 1)) + rng.standard_normal((t, cfg.dim)))
+    wh = S.embed_head_weights(cfg, 13)
+    classes = 1024                                   # 1000 padded with zero rows
+    w_head = np.zeros((classes, cfg.dim), np.uint16)
+    w_head[:1000] = wh["w_head"]
+    b_head = np.zeros(classes, np.uint16)
+    b_head[:1000] = wh["b_head"]
+    logits = torch.full((cfg.batch, classes), 9.0, dtype=torch.bfloat16, device=dev())
+    ws = P.dora_classifier_head(bf(x), i32(cu), bf(wh["norm_w"]), bf(wh["norm_b"]), 1e-6,
+                                bf(w_head), bf(b_head), logits)
+    torch.cuda.synchronize()
+    assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+    ref = O.classifier_head(O.bf16_to_f64(x), cu, O.bf16_to_f64(wh["norm_w"]),
+                            O.bf16_to_f64(wh["norm_b"]), 1e-6, O.bf16_to_f64(w_head),
+                            O.bf16_to_f64(b_head))
+    assert_close(f64(logits), ref, f"classifier {name}")
+    assert torch.all(logits[:, 1000:] == 0)
