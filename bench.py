@@ -440,6 +440,53 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
     except Exception as e:                       # context figure only
         result["graph"] = {"unavailable": f"{type(e).__name__}: {e}"[:200]}
 
+    # the complete online forward (App. E.4): patch embedding from the images,
+    # the blocks (the actor choosing the deleted tokens at the pruning
+    # blocks), and the classifier head; and the same unpruned, for DORA/Native
+    if split == 1:
+        eh = S.embed_head_weights(cfg, args.seed)
+        E = {k: bf(v) for k, v in eh.items()}
+        w_head = torch.zeros(1024, cfg.dim, dtype=torch.bfloat16, device=dev)
+        w_head[:1000] = E["w_head"]
+        b_head = torch.zeros(1024, dtype=torch.bfloat16, device=dev)
+        b_head[:1000] = E["b_head"]
+        imgs = [bf(S.images_bf16(cfg, args.seed + 7 + r)) for r in range(nsets)]
+        x0 = torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev)
+        logits = torch.zeros(cfg.batch, 1024, dtype=torch.bfloat16, device=dev)
+        ews = P.dora_patch_embed(imgs[0], E["w_pe"], E["b_pe"], E["cls"], E["pos"], 16, x0,
+                                 stream=stream)
+        hws = None
+
+        def full_step(i, pruned):
+            nonlocal hws
+            r = i % nsets
+            P.dora_patch_embed(imgs[r], E["w_pe"], E["b_pe"], E["cls"], E["pos"], 16, x0, ews,
+                               stream=stream)
+            (xf, cuf), = forward(dict(sets[r], x=x0), pruned, with_actor=pruned)
+            hws = P.dora_classifier_head(xf, cuf, E["norm_w"], E["norm_b"], 1e-6, w_head, b_head,
+                                         logits, hws, stream=stream)
+
+        fsecs, _ = timed(lambda i: full_step(i, True), args.steps, max(args.warmup, 3))
+        fdsecs, _ = timed(lambda i: full_step(i, False), args.steps, max(args.warmup, 3))
+        lens = hw.lengths_per_block(0)
+        sched = dict(zip(cfg.prune_blocks, hw.sets[0]["keeps"]))
+        fl = A.trajectory_flops(cfg.depth, cfg.dim, cfg.mlp_dim, cfg.n_tokens, sched,
+                                include_embed_head=True)
+        for l in cfg.prune_blocks:
+            fl = fl + A.actor_flops(lens[l][0], cfg.dim, cfg.n_vis0, True)
+        fld = A.trajectory_flops(cfg.depth, cfg.dim, cfg.mlp_dim, cfg.n_tokens, {},
+                                 include_embed_head=True)
+        result["full_forward"] = {
+            "value": round(cfg.batch * args.steps * world / fsecs, 1), "unit": UNIT,
+            "ms_per_step": round(1000 * fsecs / args.steps, 4),
+            "dense_value": round(cfg.batch * args.steps * world / fdsecs, 1),
+            "speedup_vs_dense": round(fdsecs / fsecs, 4),
+            "gflops_per_image": round(float(fl.mean()) / 1e9, 3),
+            "gflops_per_image_dense": round(float(fld.mean()) / 1e9, 3),
+            "what": "images (device-resident, 3x224x224 bf16) -> patch embedding -> 12 blocks "
+                    "(actor at the pruning blocks, configured keep counts) -> LayerNorm + "
+                    "classifier; dense = the same without deletion or actor"}
+
     # context: torch eager dense forward of the same shapes and weights
     # (cuBLAS linears, scaled_dot_product_attention), not this library
     try:

@@ -96,3 +96,20 @@ def select_compact_bytes(t_in: int, t_out: int, batch: int, dim: int, fused_ln: 
 
 def gemm_flops(m: int, n: int, k: int) -> float:
     return 2.0 * m * n * k
+
+
+def actor_flops(n_tokens: int | np.ndarray, dim: int, n0: int,
+                controller: bool | np.ndarray = True) -> np.ndarray:
+    """FLOPs of the actor at one block for one image (App. A.1; App. E.4
+    counts them): the gate always, and when it opens the controller -- the
+    width-128 encoder over the N_l + 1 tokens (input projection, QKV, four
+    heads of 32, output projection, 128 -> 256 -> 128 feed-forward), the
+    budget head on CLS and the 128 -> 64 -> 1 selector on the visual tokens."""
+    n = np.asarray(n_tokens, dtype=np.float64)
+    gate = 2.0 * (dim + 19) * 64 + 2.0 * 64
+    w = 128.0
+    enc = (2.0 * n * dim * w + 2.0 * 3 * w + 2.0 * n * w * 3 * w + 4.0 * n * n * w
+           + 2.0 * n * w * w + 2.0 * n * w * 256 * 2)
+    budget = 2.0 * w * w + 2.0 * w * ((n0 - 4) // 2)
+    selector = 2.0 * (n - 1) * (w * 64 + 64)
+    return gate + np.where(np.asarray(controller), enc + budget + selector, 0.0)
