@@ -39,7 +39,7 @@ constexpr int SH = 64;          // selector hidden units
 constexpr int kMaxDim = 2048;
 constexpr int kMaxN0 = 1028;    // budget-head outputs (n0 - 4) / 2 <= 512
 constexpr int kMaxBudgets = (kMaxN0 - 4) / 2;
-constexpr int kSelWarps = 8;
+constexpr int kGateStagedInputs = 1536;   // gate weights staged in shared memory up to d + 19 = 1536
 
 __device__ __forceinline__ float ld(const uint16_t* __restrict__ p, size_t i) {
   return __uint_as_float(static_cast<uint32_t>(p[i]) << 16);
@@ -107,22 +107,67 @@ __global__ void bias_in_kernel(const uint16_t* __restrict__ b_in, const uint16_t
 }
 
 // ---------------------------------------------------------------------------
-// gate (Appendix A.1): one CTA of 128 threads per image
+// gate (Appendix A.1) and budget head (Sec. 3.2; Appendix A.1-A.3): one CTA per
+// image.  Their weights are transposed once ([inputs, outputs]), so the
+// threads computing neighbouring outputs read each input's weights together,
+// and every thread keeps several independent loads in flight.
 // ---------------------------------------------------------------------------
+__global__ void transpose_kernel(const uint16_t* __restrict__ w, int rows, int cols,
+                                 uint16_t* __restrict__ wt) {
+  for (int idx = blockIdx.x * blockDim.x + threadIdx.x; idx < rows * cols;
+       idx += gridDim.x * blockDim.x) {
+    const int c = idx / rows, r = idx % rows;    // wt [cols, rows]
+    wt[idx] = w[static_cast<size_t>(r) * cols + c];
+  }
+}
+
+// Copy n16 16-byte words from global to shared memory, 8 loads in flight.
+__device__ __forceinline__ void stage(uint4* __restrict__ dst, const uint4* __restrict__ src,
+                                      int n16) {
+  int i = threadIdx.x;
+  for (; i + 7 * static_cast<int>(blockDim.x) < n16; i += 8 * blockDim.x) {
+    uint4 v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = src[i + e * blockDim.x];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) dst[i + e * blockDim.x] = v[e];
+  }
+  for (; i < n16; i += blockDim.x) dst[i] = src[i];
+}
+
+// sum_c wt[c * stride + o] * v[c] over c in [c0, c1), 8 loads in flight
+__device__ __forceinline__ float dot_t(const uint16_t* __restrict__ wt, int stride, int o,
+                                       const float* __restrict__ v, int c0, int c1) {
+  float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  int c = c0;
+  for (; c + 7 < c1; c += 8) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) a[e] = fmaf(ld(wt, static_cast<size_t>(c + e) * stride + o), v[c + e], a[e]);
+  }
+  for (; c < c1; ++c) a[0] = fmaf(ld(wt, static_cast<size_t>(c) * stride + o), v[c], a[0]);
+  return ((a[0] + a[1]) + (a[2] + a[3])) + ((a[4] + a[5]) + (a[6] + a[7]));
+}
+
 // h_l = [N_l / N0, rho_l, E_<l / (L - 1)]; the gate logit and p^G; and W_h h_l
-// added to the image's CLS row of the encoder input x [rows, 128].
-__global__ void __launch_bounds__(128) gate_kernel(
-    const uint16_t* __restrict__ qkv, int dim, const int32_t* __restrict__ cu, int t_cap, int block,
-    int depth, int n0, const float* __restrict__ rho, const int32_t* __restrict__ interventions,
-    const uint16_t* __restrict__ w1, const uint16_t* __restrict__ b1,
-    const uint16_t* __restrict__ w2, const uint16_t* __restrict__ b2,
-    const uint16_t* __restrict__ emb, const uint16_t* __restrict__ w_h,
-    uint16_t* __restrict__ x, float* __restrict__ glogit, float* __restrict__ p_gate) {
+// added to the image's CLS row of the encoder input x [rows, 128].  256
+// threads: hidden unit t % 64 over a quarter t / 64 of the d + 19 inputs.
+__global__ void __launch_bounds__(256) gate_kernel(
+    const uint16_t* __restrict__ qkv, int dim, const int32_t* __restrict__ cu, int t_cap,
+    int block, int depth, int n0, const float* __restrict__ rho,
+    const int32_t* __restrict__ interventions, const uint16_t* __restrict__ w1t,
+    const uint16_t* __restrict__ b1, const uint16_t* __restrict__ w2,
+    const uint16_t* __restrict__ b2, const uint16_t* __restrict__ emb,
+    const uint16_t* __restrict__ w_h, uint16_t* __restrict__ x, float* __restrict__ glogit,
+    float* __restrict__ p_gate) {
   __shared__ float z[kMaxDim + GE + 3];
-  __shared__ float hid[GH];
+  __shared__ float part[4][GH];
+  extern __shared__ __align__(16) uint4 wsm[];          // W_1^T when it fits (else empty)
   const int i = blockIdx.x, t = threadIdx.x;
   const int lo = cu[i], hi = cu[i + 1];
   const int n = (lo < 0 || hi > t_cap) ? -1 : hi - lo - 1;   // visual tokens
+  const int kin_ = dim + GE + 3;
+  const bool staged = kin_ <= kGateStagedInputs;
+  if (staged && n >= 0) stage(wsm, reinterpret_cast<const uint4*>(w1t), kin_ * GH * 2 / 16);
   if (n < 0) {                                       // empty (or outside the buffer): closed
     if (t == 0) {
       glogit[i] = -INFINITY;
@@ -133,6 +178,7 @@ __global__ void __launch_bounds__(128) gate_kernel(
   const float h0 = static_cast<float>(n) / static_cast<float>(n0);
   const float h1 = rho[i];
   const float h2 = static_cast<float>(interventions[i]) / static_cast<float>(max(depth - 1, 1));
+  const int kin = dim + GE + 3;
   const size_t krow = static_cast<size_t>(lo) * 3 * dim + dim;   // the CLS key
   for (int c = t; c < dim; c += blockDim.x) z[c] = ld(qkv, krow + c);
   if (t < GE) z[dim + t] = ld(emb, static_cast<size_t>(block) * GE + t);
@@ -142,21 +188,20 @@ __global__ void __launch_bounds__(128) gate_kernel(
     z[dim + GE + 2] = h2;
   }
   __syncthreads();
-  const int kin = dim + GE + 3;
   {
-    // hidden unit h is one warp's dot product, the lanes striding along it
-    const int warp = t >> 5, lane = t & 31;
-    for (int h = warp; h < GH; h += 4) {
-      const uint16_t* wr = w1 + static_cast<size_t>(h) * kin;
-      float a = 0.f;
-      for (int c = lane; c < kin; c += 32) a = fmaf(ld(wr, c), z[c], a);
-      a = warp_sum(a);
-      if (lane == 0) hid[h] = silu(a + ld(b1, h));
-    }
+    const int h = t % GH, q = t / GH;
+    const int c0 = (kin * q) / 4, c1 = (kin * (q + 1)) / 4;
+    part[q][h] = dot_t(staged ? reinterpret_cast<const uint16_t*>(wsm) : w1t, GH, h, z, c0, c1);
   }
   __syncthreads();
   if (t < 32) {
-    const float s = warp_sum(ld(w2, t) * hid[t] + ld(w2, t + 32) * hid[t + 32]);
+    float s = 0.f;
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int h = t + 32 * e;
+      s += ld(w2, h) * silu(((part[0][h] + part[1][h]) + (part[2][h] + part[3][h])) + ld(b1, h));
+    }
+    s = warp_sum(s);
     if (t == 0) {
       const float lg = s + ld(b2, 0);
       glogit[i] = lg;
@@ -164,33 +209,36 @@ __global__ void __launch_bounds__(128) gate_kernel(
     }
   }
   // the history enters the encoder on the CLS token only
-  uint16_t* xr = x + static_cast<size_t>(lo) * W;
-  const float v = ld(w_h, t * 3) * h0 + ld(w_h, t * 3 + 1) * h1 + ld(w_h, t * 3 + 2) * h2;
-  xr[t] = to_bf16(ld(xr, t) + v);
+  if (t < W) {
+    uint16_t* xr = x + static_cast<size_t>(lo) * W;
+    const float v = ld(w_h, t * 3) * h0 + ld(w_h, t * 3 + 1) * h1 + ld(w_h, t * 3 + 2) * h2;
+    xr[t] = to_bf16(ld(xr, t) + v);
+  }
 }
 
-// ---------------------------------------------------------------------------
-// budget head and selector (Sec. 3.2, Eq. 2; Appendix A.1-A.3): one CTA of
-// 256 threads per image
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) budget_select_kernel(
+// LayerNorm(Z_CLS) -> 128 -> 128 GELU -> M logits; the highest feasible logit
+// (k <= N_l - 4, ties to the smaller k) is the budget.  128 threads.
+__global__ void __launch_bounds__(128) budget_kernel(
     const uint16_t* __restrict__ z, const int32_t* __restrict__ cu, int t_cap, int n0, float eps,
     const uint16_t* __restrict__ ln_w, const uint16_t* __restrict__ ln_b,
-    const uint16_t* __restrict__ bw1, const uint16_t* __restrict__ bb1,
-    const uint16_t* __restrict__ bw2, const uint16_t* __restrict__ bb2,
-    const uint16_t* __restrict__ s1, const float* __restrict__ sel_wk,
-    const uint16_t* __restrict__ sw2, const uint16_t* __restrict__ sb2,
-    const float* __restrict__ glogit,
-    const int32_t* __restrict__ interventions, int32_t* __restrict__ gate,
-    int32_t* __restrict__ budget, int32_t* __restrict__ k_out, int32_t* __restrict__ keep,
-    float* __restrict__ rho_next, int32_t* __restrict__ e_next, float* __restrict__ scores) {
+    const uint16_t* __restrict__ bw1t, const uint16_t* __restrict__ bb1,
+    const uint16_t* __restrict__ bw2t, const uint16_t* __restrict__ bb2,
+    const float* __restrict__ glogit, const int32_t* __restrict__ interventions,
+    int32_t* __restrict__ gate, int32_t* __restrict__ budget, int32_t* __restrict__ k_out,
+    int32_t* __restrict__ keep, float* __restrict__ rho_next, int32_t* __restrict__ e_next,
+    float* __restrict__ scores) {
   __shared__ float u[W], hb[W], logit[kMaxBudgets];
-  __shared__ float sck[SH], sw2s[SH];
-  __shared__ int s_budget;
+  extern __shared__ __align__(16) uint4 bsm[];          // W_1^T [128, 128], W_2^T [128, M]
   const int i = blockIdx.x, t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int lo = cu[i], hi = cu[i + 1];
   const int n = (lo < 0 || hi > t_cap) ? -1 : hi - lo - 1;
   const int m_out = (n0 - 4) / 2;
+  uint16_t* const w1s = reinterpret_cast<uint16_t*>(bsm);
+  uint16_t* const w2s = w1s + W * W;
+  if (n >= 0) {
+    stage(bsm, reinterpret_cast<const uint4*>(bw1t), W * W * 2 / 16);
+    stage(reinterpret_cast<uint4*>(w2s), reinterpret_cast<const uint4*>(bw2t), W * m_out * 2 / 16);
+  }
   if (n < 0) {
     if (t == 0) {
       gate[i] = budget[i] = k_out[i] = keep[i] = 0;
@@ -216,24 +264,9 @@ __global__ void __launch_bounds__(256) budget_select_kernel(
     }
   }
   __syncthreads();
-  // each output one warp's dot product over 128, the lanes striding along it
-  for (int h = warp; h < W; h += kSelWarps) {
-    float a = 0.f;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) a = fmaf(ld(bw1, static_cast<size_t>(h) * W + lane + 32 * q),
-                                          u[lane + 32 * q], a);
-    a = warp_sum(a);
-    if (lane == 0) hb[h] = gelu(a + ld(bb1, h));
-  }
+  hb[t] = gelu(dot_t(w1s, W, t, u, 0, W) + ld(bb1, t));
   __syncthreads();
-  for (int m = warp; m < m_out; m += kSelWarps) {
-    float a = 0.f;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) a = fmaf(ld(bw2, static_cast<size_t>(m) * W + lane + 32 * q),
-                                          hb[lane + 32 * q], a);
-    a = warp_sum(a);
-    if (lane == 0) logit[m] = a + ld(bb2, m);
-  }
+  for (int m = t; m < m_out; m += blockDim.x) logit[m] = dot_t(w2s, m_out, m, hb, 0, W) + ld(bb2, m);
   __syncthreads();
   if (t == 0) {
     int best = -1;
@@ -252,13 +285,26 @@ __global__ void __launch_bounds__(256) budget_select_kernel(
     keep[i] = n + 1 - kk;
     if (rho_next != nullptr) rho_next[i] = n > 0 ? static_cast<float>(kk) / n : 0.f;
     if (e_next != nullptr) e_next[i] = interventions[i] + g;
-    s_budget = bud;
     scores[lo] = 0.f;
   }
-  __syncthreads();
-  // selector tail: one thread per visual token, s = w_2 . silu(S1_j + (k / N_l)
-  // W_1 W_k) + b_2, with S1_j = W_1 Z_j + b_1 from the GEMM
-  const float kr = n > 0 ? static_cast<float>(s_budget) / n : 0.f;
+}
+
+// ---------------------------------------------------------------------------
+// selector tail (Eq. 2): one thread per visual token, s = w_2 . silu(S1_j +
+// (k / N_l) W_1 W_k) + b_2, with S1_j = W_1 Z_j + b_1 from the GEMM and k the
+// image's budget
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) selector_kernel(
+    const uint16_t* __restrict__ s1, const int32_t* __restrict__ cu, int t_cap,
+    const int32_t* __restrict__ budget, const float* __restrict__ sel_wk,
+    const uint16_t* __restrict__ sw2, const uint16_t* __restrict__ sb2,
+    float* __restrict__ scores) {
+  __shared__ float sck[SH], sw2s[SH];
+  const int i = blockIdx.x, t = threadIdx.x;
+  const int lo = cu[i], hi = cu[i + 1];
+  const int n = (lo < 0 || hi > t_cap) ? -1 : hi - lo - 1;
+  if (n <= 0) return;
+  const float kr = static_cast<float>(budget[i]) / n;
   if (t < SH) {
     sck[t] = kr * sel_wk[t];
     sw2s[t] = ld(sw2, t);
@@ -268,7 +314,7 @@ __global__ void __launch_bounds__(256) budget_select_kernel(
   for (int j = 1 + t; j <= n; j += blockDim.x) {
     const uint4* sr = reinterpret_cast<const uint4*>(s1 + static_cast<size_t>(lo + j) * SH);
     float acc = 0.f;
-#pragma unroll
+#pragma unroll 2
     for (int q = 0; q < SH / 8; ++q) {
       const uint4 v = sr[q];
       const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
@@ -290,7 +336,7 @@ size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
 
 struct Prep {
   size_t bias_in, wqkv_f, cqkv_f, dqkv_f, wqkv_p, cqkv_p, dqkv_p, wo_p, wfc1, cfc1, dfc1, sel_wk,
-      total;
+      gate_w1t, bud_w1t, bud_w2t, total;
 };
 
 Prep prep_layout(const dora_actor_weights* w) {
@@ -308,6 +354,9 @@ Prep prep_layout(const dora_actor_weights* w) {
   P.cfc1 = off;    off += up256(FF * 4);
   P.dfc1 = off;    off += up256(FF * 4);
   P.sel_wk = off;  off += up256(SH * 4);
+  P.gate_w1t = off; off += up256(static_cast<size_t>(w->dim + GE + 3) * GH * 2);
+  P.bud_w1t = off; off += up256(W * W * 2);
+  P.bud_w2t = off; off += up256(static_cast<size_t>(W) * ((w->n0 - 4) / 2) * 2);
   P.total = off;
   return P;
 }
@@ -369,6 +418,12 @@ cudaError_t prepare(const dora_actor_weights* w, uint8_t* prep, cudaStream_t str
   bias_in_kernel<<<w->depth, W, 0, stream>>>(w->enc_b_in, w->enc_emb,
                                              reinterpret_cast<uint16_t*>(prep + P.bias_in));
   sel_wk_kernel<<<1, SH, 0, stream>>>(w->sel_w1, w->sel_w_k, reinterpret_cast<float*>(prep + P.sel_wk));
+  transpose_kernel<<<64, 256, 0, stream>>>(w->gate_w1, GH, w->dim + GE + 3,
+                                           reinterpret_cast<uint16_t*>(prep + P.gate_w1t));
+  transpose_kernel<<<64, 256, 0, stream>>>(w->bud_w1, W, W,
+                                           reinterpret_cast<uint16_t*>(prep + P.bud_w1t));
+  transpose_kernel<<<64, 256, 0, stream>>>(w->bud_w2, (w->n0 - 4) / 2, W,
+                                           reinterpret_cast<uint16_t*>(prep + P.bud_w2t));
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   return launch_fold_ln(w->enc_w_fc1, FF, W, w->enc_ln2_w, w->enc_ln2_b, w->enc_b_fc1,
@@ -463,9 +518,18 @@ int dora_actor(const dora_bf16* qkv, const int32_t* cu, int32_t batch, int32_t m
                     stream, 3 * d) != cudaSuccess)
     return DORA_ERR_CUDA;
   // gate, and the history term on every CLS row
-  gate_kernel<<<batch, 128, 0, stream>>>(qkv, d, cu, t_cap, block, w->depth, w->n0, rho, interventions,
-                                         w->gate_w1, w->gate_b1, w->gate_w2, w->gate_b2,
-                                         w->gate_emb, w->enc_w_h, x, glogit, p_gate);
+  const int kin = d + GE + 3;
+  const size_t gate_smem = kin <= kGateStagedInputs ? static_cast<size_t>(kin) * GH * 2 : 0;
+  const size_t bud_smem = static_cast<size_t>(W) * (W + (w->n0 - 4) / 2) * 2;
+  if (cudaFuncSetAttribute(gate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(gate_smem)) != cudaSuccess ||
+      cudaFuncSetAttribute(budget_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(bud_smem)) != cudaSuccess)
+    return DORA_ERR_CUDA;
+  gate_kernel<<<batch, 256, gate_smem, stream>>>(
+      qkv, d, cu, t_cap, block, w->depth, w->n0, rho, interventions,
+      reinterpret_cast<const uint16_t*>(prep + P.gate_w1t), w->gate_b1, w->gate_w2, w->gate_b2,
+      w->gate_emb, w->enc_w_h, x, glogit, p_gate);
   if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
   // Z1 = X + W_o Attention(LayerNorm1(X)) + b_o
   LinearEpi e_q;
@@ -508,10 +572,15 @@ int dora_actor(const dora_bf16* qkv, const int32_t* cu, int32_t batch, int32_t m
   if (launch_linear(z, t_cap, rows, W, w->sel_w1, SH, DORA_EPI_BIAS, e_s, s1, status, stream) !=
       cudaSuccess)
     return DORA_ERR_CUDA;
-  budget_select_kernel<<<batch, 256, 0, stream>>>(
-      z, cu, t_cap, w->n0, w->eps, w->bud_ln_w, w->bud_ln_b, w->bud_w1, w->bud_b1, w->bud_w2,
-      w->bud_b2, s1, reinterpret_cast<const float*>(prep + P.sel_wk), w->sel_w2, w->sel_b2,
-      glogit, interventions, gate, budget, k, keep_counts, rho_next, interventions_next, scores);
+  budget_kernel<<<batch, 128, bud_smem, stream>>>(
+      z, cu, t_cap, w->n0, w->eps, w->bud_ln_w, w->bud_ln_b,
+      reinterpret_cast<const uint16_t*>(prep + P.bud_w1t), w->bud_b1,
+      reinterpret_cast<const uint16_t*>(prep + P.bud_w2t), w->bud_b2, glogit, interventions, gate,
+      budget, k, keep_counts, rho_next,
+      interventions_next, scores);
+  selector_kernel<<<batch, 256, 0, stream>>>(s1, cu, t_cap, budget,
+                                             reinterpret_cast<const float*>(prep + P.sel_wk),
+                                             w->sel_w2, w->sel_b2, scores);
   return cudaGetLastError() == cudaSuccess ? DORA_OK : DORA_ERR_CUDA;
 }
 
