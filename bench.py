@@ -40,6 +40,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # dram__bytes_write.sum), keyed by the sha256 of the kernel source it was
 # taken on; reported as null once the source changes.
 NCU_TRAFFIC = {
+    # profiles/gemm_tcgen05_deit_base_b256.md: mean over the 48 GEMM launches
+    # of one forward step
     "b34dcbc477c16fbd82653b7888b9deb4fa8716d95e482f5d9899e205d6137ff3": 188246208,
 }
 
