@@ -162,6 +162,9 @@ class Config:
     ln_eps: float = 1e-6
     head_dim: int = 64
     grid: int = 14          # patch grid side (N0 = grid^2)
+    patch: int = 16         # patch side in pixels
+    layerscale: bool = False  # per-channel scales on both residual branches (DINOv2)
+    readout: str = "cls"    # "cls", or "lc1": LN(CLS) ++ mean of LN(surviving visual tokens)
     note: str = field(default="", compare=False)
 
     @property
@@ -179,6 +182,9 @@ CONFIGS = {
                    "heavy_tail"),
     "cfg5": Config("vit_base384_12blk_b64", 64, 577, 768, 12, 3072, 12, (2, 4, 6, 8, 10),
                    "geometric", score_law="bump", rho_lo=0.15, rho_hi=1.0, grid=24),
+    # DINOv2-B/14 (Table 3: N0 = 256): LayerScale, LC1 readout, 14-pixel patches
+    "cfg6": Config("dinov2_base14_12blk_b256", 256, 257, 768, 12, 3072, 12, (3, 6, 9), "fraction",
+                   f_lo=0.20, f_hi=0.45, grid=16, patch=14, layerscale=True, readout="lc1"),
 }
 
 
@@ -230,6 +236,11 @@ def block_weights(cfg: Config, block: int, seed: int = 0, random_affine: bool = 
         out[nm] = _normal_bf16(seed, tag, r * c, 0.02).reshape(r, c)
     vec = {"b_qkv": 3 * d, "b_proj": d, "b_fc1": m, "b_fc2": d,
            "ln1_w": d, "ln1_b": d, "ln2_w": d, "ln2_b": d}
+    if cfg.layerscale:
+        for which, nm in enumerate(("ls1", "ls2")):
+            u = uniform_f64(seed, TAG_LNAFF + (block << 8) + ((10 + which) << 4),
+                            np.arange(d, dtype=np.uint64))
+            out[nm] = f32_to_bf16_bits(0.05 + 0.45 * u)          # learned scales ~ 0.05-0.5
     for which, (nm, size) in enumerate(vec.items()):
         if random_affine:
             tag = TAG_LNAFF + (block << 8) + (which << 4)
@@ -376,10 +387,12 @@ def actor_weights(dim: int, depth: int, n0: int, seed: int = 0, gate_bias: float
 # input images and the forward's two ends (patch embedding, classifier)
 # ---------------------------------------------------------------------------
 
-def images_bf16(cfg: Config, seed: int = 0, patch: int = 16, channels: int = 3) -> np.ndarray:
+def images_bf16(cfg: Config, seed: int = 0, patch: int | None = None,
+                channels: int = 3) -> np.ndarray:
     """bf16 bit patterns of N(0, 1) images [B, C, H, W] with H = W = patch *
     sqrt(n_vis0) (224 for 196 visual tokens): normalised pixels, as a
     preprocessing pipeline hands them to the model."""
+    patch = cfg.patch if patch is None else patch
     g = int(round(np.sqrt(cfg.n_vis0)))
     assert g * g == cfg.n_vis0
     side = g * patch
@@ -387,14 +400,16 @@ def images_bf16(cfg: Config, seed: int = 0, patch: int = 16, channels: int = 3) 
     return _normal_bf16(seed, TAG_IMG, count, 1.0).reshape(cfg.batch, channels, side, side)
 
 
-def embed_head_weights(cfg: Config, seed: int = 0, patch: int = 16, channels: int = 3,
+def embed_head_weights(cfg: Config, seed: int = 0, patch: int | None = None, channels: int = 3,
                        classes: int = 1000) -> dict:
     """bf16 bit patterns of the patch embedding (w_pe [d, C patch^2], b_pe, cls,
-    pos [N, d]) and the classifier (norm_w, norm_b, w_head [classes, d],
-    b_head), randomly initialised."""
+    pos [N, d]) and the classifier (norm_w, norm_b, w_head [classes, d] -- or
+    [classes, 2 d] for the LC1 readout -- and b_head), randomly initialised."""
+    patch = cfg.patch if patch is None else patch
     d, k = cfg.dim, channels * patch * patch
+    hin = 2 * d if cfg.readout == "lc1" else d
     shapes = {"w_pe": (d, k), "b_pe": (d,), "cls": (d,), "pos": (cfg.n_tokens, d),
-              "norm_w": (d,), "norm_b": (d,), "w_head": (classes, d), "b_head": (classes,)}
+              "norm_w": (d,), "norm_b": (d,), "w_head": (classes, hin), "b_head": (classes,)}
     out = {}
     for which, (name, shape) in enumerate(shapes.items()):
         count = int(np.prod(shape))

@@ -263,13 +263,18 @@ def block_attention_half(x: np.ndarray, cu: np.ndarray, wf: dict, heads: int, ep
     xn = layernorm(x, wf["ln1_w"], wf["ln1_b"], eps)
     qkv = linear(xn, wf["w_qkv"], wf["b_qkv"])
     o = varlen_attention(qkv, cu, heads, head_dim)
-    return x + linear(o, wf["w_proj"], wf["b_proj"])
+    a = linear(o, wf["w_proj"], wf["b_proj"])
+    if "ls1" in wf:                                   # LayerScale (DINOv2 backbones)
+        a = a * wf["ls1"]
+    return x + a
 
 
 def block_mlp_half(h_keep: np.ndarray, wf: dict, eps: float) -> np.ndarray:
     """Second line of Eq. 1: H_{l+1} = H_keep + MLP(LayerNorm'(H_keep))."""
     y = linear(layernorm(h_keep, wf["ln2_w"], wf["ln2_b"], eps), wf["w_fc1"], wf["b_fc1"])
     y = linear(gelu(y), wf["w_fc2"], wf["b_fc2"])
+    if "ls2" in wf:                                   # LayerScale (DINOv2 backbones)
+        y = y * wf["ls2"]
     return h_keep + y
 
 
@@ -493,3 +498,24 @@ def classifier_head(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.nd
     x = np.asarray(x, dtype=np.float64)
     rows = np.asarray(cu[:-1], dtype=np.int64)
     return linear(layernorm(x[rows], ln_w, ln_b, eps), w_head, b_head)
+
+
+def lc1_readout(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.ndarray,
+                eps: float) -> np.ndarray:
+    """DINOv2's LC1 readout (App. E.2, baseline implementations): the final
+    LayerNorm applied to every token, then each image's normalised CLS row
+    concatenated with the mean of its normalised surviving visual rows
+    ([B, 2 d]; an image without visual tokens contributes a zero mean)."""
+    x = np.asarray(x, dtype=np.float64)
+    cu = np.asarray(cu, dtype=np.int64)
+    d = x.shape[1]
+    out = np.zeros((len(cu) - 1, 2 * d))
+    for i in range(len(cu) - 1):
+        lo, hi = int(cu[i]), int(cu[i + 1])
+        if hi <= lo:
+            continue
+        xn = layernorm(x[lo:hi], ln_w, ln_b, eps)
+        out[i, :d] = xn[0]
+        if hi - lo > 1:
+            out[i, d:] = xn[1:].mean(axis=0)
+    return out

@@ -622,3 +622,51 @@ def test_classifier_reads_only_cls_rows():
     r = x[cu[:-1]]
     ref = (r - r.mean(1, keepdims=True)) / r.std(1, keepdims=True)
     assert np.allclose(ident, ref, rtol=0, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# DINOv2 pieces: LayerScale and the LC1 readout (App. E.2; Table 3)
+# ---------------------------------------------------------------------------
+
+def test_layerscale_zero_leaves_the_residual_stream():
+    """With both LayerScales zero the block passes its (compacted) input
+    through: x_out = x[kept]; with both equal to one it is the plain block."""
+    cfg = S.get_config("cfg1", batch=3)
+    cu, ids = S.initial_layout(cfg)
+    x = O.bf16_to_f64(S.activations_bf16(cfg, 5))
+    wf = O.decode_weights(S.block_weights(cfg, 0, 5, random_affine=True))
+    keeps, _ = S.keep_schedule(cfg, 5)
+    sc = O.gather_scores(S.score_table(cfg, 0, 5), cu, ids)
+    z = dict(wf, ls1=np.zeros(cfg.dim), ls2=np.zeros(cfg.dim))
+    r = O.pruned_block(x, cu, ids, z, cfg.heads, cfg.ln_eps, sc, keeps[0])
+    assert np.array_equal(r["x_out"], x[r["kept_idx"]])
+    one = dict(wf, ls1=np.ones(cfg.dim), ls2=np.ones(cfg.dim))
+    a = O.pruned_block(x, cu, ids, one, cfg.heads, cfg.ln_eps, sc, keeps[0])
+    b = O.pruned_block(x, cu, ids, wf, cfg.heads, cfg.ln_eps, sc, keeps[0])
+    assert np.array_equal(a["x_out"], b["x_out"])
+
+
+def test_lc1_readout_loops_and_invariants():
+    """Element by element against loops; a single visual token's mean is that
+    token; the mean does not depend on the order of the visual tokens."""
+    rng = np.random.default_rng(21)
+    d = 6
+    cu = np.array([0, 4, 6, 7, 11])
+    x = rng.standard_normal((11, d)) * 2 + 1
+    g, be = 1 + 0.1 * rng.standard_normal(d), 0.1 * rng.standard_normal(d)
+    r = O.lc1_readout(x, cu, g, be, 1e-6)
+    for i in range(4):
+        lo, hi = cu[i], cu[i + 1]
+        rows = []
+        for j in range(lo, hi):
+            mu = sum(x[j]) / d
+            var = sum((v - mu) ** 2 for v in x[j]) / d
+            rows.append([(x[j][c] - mu) / math.sqrt(var + 1e-6) * g[c] + be[c] for c in range(d)])
+        assert np.allclose(r[i, :d], rows[0], rtol=0, atol=1e-12)
+        mean = [sum(rw[c] for rw in rows[1:]) / max(len(rows) - 1, 1) for c in range(d)]
+        assert np.allclose(r[i, d:], mean if len(rows) > 1 else np.zeros(d), rtol=0, atol=1e-12)
+    # image 1 has one visual token: its mean is that token's normalised row
+    assert np.allclose(r[1, d:], O.layernorm(x[5:6], g, be, 1e-6)[0], rtol=0, atol=1e-12)
+    xp = x.copy()
+    xp[8:11] = x[[10, 8, 9]]
+    assert np.allclose(O.lc1_readout(xp, cu, g, be, 1e-6), r, rtol=0, atol=1e-12)
