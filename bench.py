@@ -9,6 +9,10 @@ token id.  One step = one forward of the whole batch: at each pruning block
 the score gather (actor stand-in) and dora_pruned_block, elsewhere
 dora_pruned_block without deletion.
 
+``--config cfg6`` runs the DINOv2-B/14 shape instead (257 tokens, LayerScale
+folded into the attention-output and fc2 weights at load, 14-pixel patches
+and the LC1 head in the complete-forward leg).
+
 Prints one JSON line.  ``--impl reference`` times the fp64 CPU oracle on the
 same workload instead (bounded samples, host cores only).
 """
@@ -384,7 +388,7 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
         "data": "synthetic (seeded bf16 N(0,1) activations, N(0,0.02) weights, U(0,1) score "
                 "tables); no trained weights or images",
         "config": {
-            "workload": f"{cfg.name}: DeiT-B shape, batch {cfg.batch}/GPU, N={cfg.n_tokens}, "
+            "workload": f"{cfg.name}: batch {cfg.batch}/GPU, N={cfg.n_tokens}, "
                         f"D={cfg.dim}, H={cfg.heads}, MLP {cfg.mlp_dim}, {cfg.depth} blocks, "
                         f"prune at {'/'.join(map(str, cfg.prune_blocks))}",
             "global_batch": cfg.batch * world, "seq_len": cfg.n_tokens,
@@ -445,36 +449,40 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
     if split == 1:
         eh = S.embed_head_weights(cfg, args.seed)
         E = {k: bf(v) for k, v in eh.items()}
-        w_head = torch.zeros(1024, cfg.dim, dtype=torch.bfloat16, device=dev)
+        lc1 = cfg.readout == "lc1"                 # DINOv2: [LN CLS, mean LN visual] features
+        head = P.dora_classifier_head_lc1 if lc1 else P.dora_classifier_head
+        w_head = torch.zeros(1024, E["w_head"].shape[1], dtype=torch.bfloat16, device=dev)
         w_head[:1000] = E["w_head"]
         b_head = torch.zeros(1024, dtype=torch.bfloat16, device=dev)
         b_head[:1000] = E["b_head"]
         imgs = [bf(S.images_bf16(cfg, args.seed + 7 + r)) for r in range(nsets)]
+        side = int(imgs[0].shape[-1])
         x0 = torch.zeros(t_cap, cfg.dim, dtype=torch.bfloat16, device=dev)
         logits = torch.zeros(cfg.batch, 1024, dtype=torch.bfloat16, device=dev)
-        ews = P.dora_patch_embed(imgs[0], E["w_pe"], E["b_pe"], E["cls"], E["pos"], 16, x0,
-                                 stream=stream)
+        ews = P.dora_patch_embed(imgs[0], E["w_pe"], E["b_pe"], E["cls"], E["pos"], cfg.patch,
+                                 x0, stream=stream)
         hws = None
 
         def full_step(i, pruned):
             nonlocal hws
             r = i % nsets
-            P.dora_patch_embed(imgs[r], E["w_pe"], E["b_pe"], E["cls"], E["pos"], 16, x0, ews,
-                               stream=stream)
+            P.dora_patch_embed(imgs[r], E["w_pe"], E["b_pe"], E["cls"], E["pos"], cfg.patch, x0,
+                               ews, stream=stream)
             (xf, cuf), = forward(dict(sets[r], x=x0), pruned, with_actor=pruned)
-            hws = P.dora_classifier_head(xf, cuf, E["norm_w"], E["norm_b"], 1e-6, w_head, b_head,
-                                         logits, hws, stream=stream)
+            hws = head(xf, cuf, E["norm_w"], E["norm_b"], 1e-6, w_head, b_head, logits, hws,
+                       stream=stream)
 
         fsecs, _ = timed(lambda i: full_step(i, True), args.steps, max(args.warmup, 3))
         fdsecs, _ = timed(lambda i: full_step(i, False), args.steps, max(args.warmup, 3))
         lens = hw.lengths_per_block(0)
         sched = dict(zip(cfg.prune_blocks, hw.sets[0]["keeps"]))
+        rm = 2 if lc1 else 1
         fl = A.trajectory_flops(cfg.depth, cfg.dim, cfg.mlp_dim, cfg.n_tokens, sched,
-                                include_embed_head=True)
+                                include_embed_head=True, patch=cfg.patch, readout_mult=rm)
         for l in cfg.prune_blocks:
             fl = fl + A.actor_flops(lens[l][0], cfg.dim, cfg.n_vis0, True)
         fld = A.trajectory_flops(cfg.depth, cfg.dim, cfg.mlp_dim, cfg.n_tokens, {},
-                                 include_embed_head=True)
+                                 include_embed_head=True, patch=cfg.patch, readout_mult=rm)
         result["full_forward"] = {
             "value": round(cfg.batch * args.steps * world / fsecs, 1), "unit": UNIT,
             "ms_per_step": round(1000 * fsecs / args.steps, 4),
@@ -482,7 +490,8 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
             "speedup_vs_dense": round(fdsecs / fsecs, 4),
             "gflops_per_image": round(float(fl.mean()) / 1e9, 3),
             "gflops_per_image_dense": round(float(fld.mean()) / 1e9, 3),
-            "what": "images (device-resident, 3x224x224 bf16) -> patch embedding -> 12 blocks "
+            "what": f"images (device-resident, 3x{side}x{side} bf16) -> patch embedding "
+                    f"({cfg.patch}-pixel patches) -> {cfg.depth} blocks "
                     "(actor at the pruning blocks, configured keep counts) -> LayerNorm + "
                     "classifier; dense = the same without deletion or actor"}
 

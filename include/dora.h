@@ -512,12 +512,15 @@ int dora_pruned_block_actor(const dora_bf16* x_in, const int32_t* cu_in, const i
  * p (row-major over the patch grid) embedded by the patch x patch, stride
  * patch convolution (w_pe bf16 [dim, channels * patch * patch], the
  * [dim, C, p, p] kernel flattened; b_pe bf16 [dim], nullable) plus pos[1 + p]
- * (pos bf16 [g + 1, dim]; cls bf16 [dim]).  patch % 8 == 0, height and
- * width multiples of patch, channels * patch^2 % 64 == 0, dim % 64 == 0.
- * The convolution is a relayout (patchify) and one tcgen05 GEMM with fp32
- * accumulation (its output rounded to bf16), then the position add.
- * workspace: dora_embed_workspace_size bytes, 256-byte aligned; its first
- * word is a status word.
+ * (pos bf16 [g + 1, dim]; cls bf16 [dim]).  1 <= patch <= 64, 1 <= channels
+ * <= 64, height and width multiples of patch, dim % 64 == 0.  The
+ * convolution is a relayout (patchify) and one tcgen05 GEMM with fp32
+ * accumulation (its output rounded to bf16), then the position add.  When
+ * K = channels * patch^2 is not a multiple of 64 (DINOv2's 14-pixel patches:
+ * K = 588) the patch matrix is K-padded with zero columns to the next
+ * multiple of 64 and a zero-padded copy of w_pe is written to the workspace
+ * on each call.  workspace: dora_embed_workspace_size bytes, 256-byte
+ * aligned; its first word is a status word.
  */
 size_t dora_embed_workspace_size(int32_t batch, int32_t channels, int32_t height, int32_t width,
                                  int32_t patch, int32_t dim);
@@ -542,6 +545,43 @@ int dora_classifier_head(const dora_bf16* x, const int32_t* cu, int32_t batch, i
                          float eps, const dora_bf16* w_head, const dora_bf16* b_head,
                          int32_t classes, dora_bf16* logits, void* workspace,
                          size_t workspace_bytes, dora_stream_t stream);
+
+/*
+ * DINOv2 backbones (App. E.2: register-free DINOv2-B/14 with its LC1 readout
+ * and LayerScale kept).
+ *
+ * dora_classifier_head_lc1 -- logits bf16 [batch, classes] = u_i W_head^T +
+ * b_head with u_i = [LN(x[cu[i]]), mean over j in (cu[i], cu[i+1]) of
+ * LN(x[j])] (2 * dim features): the final LayerNorm (norm_w, norm_b bf16
+ * [dim], epsilon eps, biased variance, fp32) applied to every surviving row,
+ * CLS first, then the mean of the normalised visual rows (zero for an image
+ * with only its CLS row; an empty image gives u = 0).  w_head bf16
+ * [classes, 2 * dim], b_head bf16 [classes] (nullable), classes % 32 == 0,
+ * dim % 64 == 0 and dim <= 2048; x bf16 [t_cap, dim] packed, cu int32
+ * [batch + 1].  u is rounded to bf16 before the tcgen05 GEMM.  workspace:
+ * dora_head_lc1_workspace_size bytes, 256-byte aligned, status word first
+ * (DORA_ERR_DEVICE_SEQLEN for cu outside [0, t_cap]).
+ */
+size_t dora_head_lc1_workspace_size(int32_t batch, int32_t dim);
+int dora_classifier_head_lc1(const dora_bf16* x, const int32_t* cu, int32_t batch, int32_t t_cap,
+                             int32_t dim, const dora_bf16* norm_w, const dora_bf16* norm_b,
+                             float eps, const dora_bf16* w_head, const dora_bf16* b_head,
+                             int32_t classes, dora_bf16* logits, void* workspace,
+                             size_t workspace_bytes, dora_stream_t stream);
+
+/*
+ * dora_fold_layerscale -- LayerScale (per-channel scale gamma on a residual
+ * branch, x + gamma * (W h + b)) folded into the branch's last linear:
+ * w_out[i, :] = bf16(gamma_i * w[i, :]), b_out[i] = bf16(gamma_i * b_i).
+ * w, w_out bf16 [n, k] (nn.Linear layout, k % 8 == 0, 16-byte aligned;
+ * w_out == w is allowed), gamma bf16 [n]; b and b_out bf16 [n], both null or
+ * both set (b_out == b allowed).  Each output is the round-to-nearest-even of
+ * the exact product.  Called once per block for the attention output and
+ * fc2 linears; the folded weights then run through dora_pruned_block.
+ */
+int dora_fold_layerscale(const dora_bf16* w, const dora_bf16* b, const dora_bf16* gamma,
+                         int32_t n, int32_t k, dora_bf16* w_out, dora_bf16* b_out,
+                         dora_stream_t stream);
 
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug

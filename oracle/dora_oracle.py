@@ -519,3 +519,10 @@ def lc1_readout(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.ndarra
         if hi - lo > 1:
             out[i, d:] = xn[1:].mean(axis=0)
     return out
+
+
+def classifier_head_lc1(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.ndarray,
+                        eps: float, w_head: np.ndarray, b_head: np.ndarray) -> np.ndarray:
+    """Class logits from the LC1 features (App. E.2): the linear layer
+    w_head [classes, 2 d] applied to lc1_readout's [B, 2 d] rows."""
+    return linear(lc1_readout(x, cu, ln_w, ln_b, eps), w_head, b_head)

@@ -24,7 +24,7 @@ __all__ = [
     "dora_folded_weights_size", "dora_fold_block_weights", "dora_compact_stats",
     "dora_merge_moments", "ActorWeights", "dora_actor", "dora_actor_workspace_size",
     "alloc_actor_workspace", "dora_pruned_block_actor", "dora_patch_embed",
-    "dora_classifier_head",
+    "dora_classifier_head", "dora_classifier_head_lc1", "dora_fold_layerscale",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -75,6 +75,10 @@ _SIGS = {
     "dora_patch_embed": (ctypes.c_int, [_vp, _i32, _i32, _i32, _i32, _i32, _i32, _vp, _vp, _vp,
                                         _vp, _vp, _vp, _sz, _vp]),
     "dora_head_workspace_size": (_sz, [_i32, _i32]),
+    "dora_head_lc1_workspace_size": (_sz, [_i32, _i32]),
+    "dora_classifier_head_lc1": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _f32, _vp,
+                                                _vp, _i32, _vp, _vp, _sz, _vp]),
+    "dora_fold_layerscale": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp]),
     "dora_classifier_head": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _f32, _vp, _vp,
                                             _i32, _vp, _vp, _sz, _vp]),
     "dora_pruned_block_actor": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
@@ -375,12 +379,25 @@ class BlockWeights:
     NAMES = ("ln1_w", "ln1_b", "w_qkv", "b_qkv", "w_proj", "b_proj", "ln2_w", "ln2_b", "w_fc1",
              "b_fc1", "w_fc2", "b_fc2")
 
-    def __init__(self, tensors: dict, dim: int, heads: int, mlp_dim: int, ln_eps: float = 1e-6):
+    def __init__(self, tensors: dict, dim: int, heads: int, mlp_dim: int, ln_eps: float = 1e-6,
+                 stream=None):
+        """Optional ``ls1``/``ls2`` (bf16 [dim], DINOv2 LayerScale) are folded
+        here, on ``stream``, into scaled copies of w_proj/b_proj and
+        w_fc2/b_fc2 (dora_fold_layerscale); the given tensors are not changed."""
         self.tensors = {}
         for n in self.NAMES:
             t = tensors.get(n)
             _req(t, torch.bfloat16, n, optional=n.startswith("b_"))
             self.tensors[n] = t
+        for ls, wn, bn in (("ls1", "w_proj", "b_proj"), ("ls2", "w_fc2", "b_fc2")):
+            g = tensors.get(ls)
+            if g is None:
+                continue
+            _req(g, torch.bfloat16, ls)
+            w, b = self.tensors[wn], self.tensors[bn]
+            if g.numel() != w.shape[0]:
+                raise ValueError(f"{ls} must have {w.shape[0]} entries")
+            self.tensors[wn], self.tensors[bn] = dora_fold_layerscale(w, b, g, stream=stream)
         self.dim, self.heads, self.mlp_dim, self.ln_eps = dim, heads, mlp_dim, ln_eps
         self.folded = None
         self.c = _BlockWeightsC(*[_ptr(self.tensors[n]) for n in self.NAMES], dim, heads, mlp_dim,
@@ -626,6 +643,48 @@ def dora_patch_embed(images, w_pe, b_pe, cls, pos, patch, x0, workspace=None, st
                                            _ptr(b_pe), _ptr(cls), _ptr(pos), _ptr(x0),
                                            _ptr(workspace), workspace.numel(), _stream(stream)),
            "dora_patch_embed")
+    return workspace
+
+
+def dora_fold_layerscale(w, b, gamma, w_out=None, b_out=None, stream=None):
+    """(bf16(gamma_i w[i, :]), bf16(gamma_i b_i)): LayerScale folded into a
+    linear's rows.  Outputs are allocated when not given; b may be None."""
+    _req(w, torch.bfloat16, "w")
+    _req(gamma, torch.bfloat16, "gamma")
+    _req(b, torch.bfloat16, "b", optional=True)
+    n, k = w.shape
+    w_out = torch.empty_like(w) if w_out is None else w_out
+    if b is not None and b_out is None:
+        b_out = torch.empty_like(b)
+    _check(load_library().dora_fold_layerscale(_ptr(w), _ptr(b), _ptr(gamma), n, k, _ptr(w_out),
+                                               _ptr(b_out) if b is not None else None,
+                                               _stream(stream)), "dora_fold_layerscale")
+    return w_out, b_out
+
+
+def dora_classifier_head_lc1(x, cu, norm_w, norm_b, eps, w_head, b_head, logits, workspace=None,
+                             stream=None):
+    """logits [B, classes] from DINOv2's LC1 features [LN(CLS), mean LN(visual
+    rows)] of each image (w_head [classes, 2 d], classes a multiple of 32)."""
+    for n, t in (("x", x), ("norm_w", norm_w), ("norm_b", norm_b), ("w_head", w_head),
+                 ("logits", logits)):
+        _req(t, torch.bfloat16, n)
+    _req(b_head, torch.bfloat16, "b_head", optional=True)
+    _req(cu, torch.int32, "cu")
+    t_cap, d = x.shape
+    b = cu.numel() - 1
+    classes = w_head.shape[0]
+    if tuple(w_head.shape) != (classes, 2 * d) or tuple(logits.shape) != (b, classes):
+        raise ValueError("w_head must be [classes, 2 d] and logits [B, classes]")
+    n = int(load_library().dora_head_lc1_workspace_size(b, d))
+    if workspace is None:
+        workspace = torch.zeros(n, dtype=torch.uint8, device=x.device)
+    _req(workspace, torch.uint8, "workspace")
+    _check(load_library().dora_classifier_head_lc1(_ptr(x), _ptr(cu), b, t_cap, d, _ptr(norm_w),
+                                                   _ptr(norm_b), float(eps), _ptr(w_head),
+                                                   _ptr(b_head), classes, _ptr(logits),
+                                                   _ptr(workspace), workspace.numel(),
+                                                   _stream(stream)), "dora_classifier_head_lc1")
     return workspace
 
 

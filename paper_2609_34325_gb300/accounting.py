@@ -47,7 +47,8 @@ def native_gflops(n_tokens: int, dim: int, mlp_dim: int, depth: int, patch: int,
 
 
 def trajectory_flops(depth: int, dim: int, mlp_dim: int, n0: int, schedule: dict,
-                     include_embed_head: bool = False, patch: int = 16) -> np.ndarray:
+                     include_embed_head: bool = False, patch: int = 16,
+                     readout_mult: int = 1) -> np.ndarray:
     """Per-image FLOPs of the blocks along realised trajectories.
 
     ``schedule`` maps a pruning block index to the int array of tokens each
@@ -64,7 +65,7 @@ def trajectory_flops(depth: int, dim: int, mlp_dim: int, n0: int, schedule: dict
         else:
             total += block_flops(n, n, dim, mlp_dim)
     if include_embed_head:
-        total += embed_flops(n0 - 1, patch, dim) + head_flops(dim)
+        total += embed_flops(n0 - 1, patch, dim) + head_flops(dim, readout_mult=readout_mult)
     return total
 
 

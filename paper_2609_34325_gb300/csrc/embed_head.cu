@@ -5,7 +5,13 @@
 //                     image's CLS token prepended and the position embeddings
 //                     added, into the packed token layout of the blocks;
 //   classifier head   the final LayerNorm on each image's CLS row and the
-//                     linear layer to the class logits (tcgen05 GEMM).
+//                     linear layer to the class logits (tcgen05 GEMM);
+//   LC1 head          DINOv2's readout (App. E.2): the final LayerNorm on every
+//                     surviving token, normalised CLS ++ the mean of the
+//                     normalised visual rows of each image, then the linear
+//                     layer on the 2 d features;
+//   LayerScale fold   DINOv2's per-channel branch scales folded once into the
+//                     rows of the attention output and fc2 linears.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -50,6 +56,52 @@ __global__ void patchify_kernel(const uint4* __restrict__ img, int batch, int ch
     const long long row = (static_cast<long long>(b) * gh + y / p) * gw + x / p;
     const int col8 = (c * p * p + (y % p) * p + x % p) / 8;
     out[row * kcols8 + col8] = img[s];
+  }
+}
+
+// Any patch side: one thread writes 8 consecutive columns of one row of the
+// K-padded patch matrix [B gh gw, kpad] (2-byte gathers; columns >= C p^2 are
+// zero).  Column order as above: c * p * p + dy * p + dx.
+__global__ void patchify_any_kernel(const uint16_t* __restrict__ img, int batch, int ch, int h,
+                                    int w, int p, int kpad, uint4* __restrict__ out) {
+  const int gw = w / p, gh = h / p, pp = p * p, k = ch * pp, kp8 = kpad / 8;
+  const long long total = static_cast<long long>(batch) * gh * gw * kp8;
+  for (long long s = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; s < total;
+       s += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int c8 = static_cast<int>(s % kp8);
+    long long r = s / kp8;
+    const int gx = static_cast<int>(r % gw);
+    r /= gw;
+    const int gy = static_cast<int>(r % gh);
+    const long long b = r / gh;
+    uint32_t v[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      uint32_t pair = 0;
+#pragma unroll
+      for (int hlf = 0; hlf < 2; ++hlf) {
+        const int col = c8 * 8 + 2 * e + hlf;
+        if (col < k) {
+          const int c = col / pp, rem = col - c * pp, dy = rem / p, dx = rem - dy * p;
+          const long long pix =
+              ((b * ch + c) * h + gy * p + dy) * static_cast<long long>(w) + gx * p + dx;
+          pair |= static_cast<uint32_t>(img[pix]) << (16 * hlf);
+        }
+      }
+      v[e] = pair;
+    }
+    out[s] = make_uint4(v[0], v[1], v[2], v[3]);
+  }
+}
+
+// w [d, k] -> [d, kpad] with zero columns k..kpad-1 (the GEMM's B for K-padded patches).
+__global__ void pad_cols_kernel(const uint16_t* __restrict__ w, int d, int k, int kpad,
+                                uint16_t* __restrict__ out) {
+  const long long total = static_cast<long long>(d) * kpad;
+  for (long long s = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; s < total;
+       s += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(s % kpad);
+    out[s] = j < k ? w[(s / kpad) * k + j] : static_cast<uint16_t>(0);
   }
 }
 
@@ -107,6 +159,116 @@ __global__ void cls_ln_kernel(const uint16_t* __restrict__ x, const int32_t* __r
   }
 }
 
+// LC1 readout of one image per CTA (16 warps): rows lo..hi-1 of x are layer-
+// normalised (fp32, biased variance, row held in registers: dim <= 2048); the
+// CLS row goes to u[i, 0:d], the others are summed per warp in shared memory
+// and their mean goes to u[i, d:2d] (zero for an image without visual rows).
+constexpr int kLc1Warps = 16;
+constexpr int kLc1MaxDim = 2048;
+
+__global__ void __launch_bounds__(kLc1Warps * 32)
+    lc1_pool_kernel(const uint16_t* __restrict__ x, const int32_t* __restrict__ cu, int t_cap,
+                    int dim, const uint16_t* __restrict__ gam, const uint16_t* __restrict__ bet,
+                    float eps, uint16_t* __restrict__ u, int32_t* status) {
+  extern __shared__ float acc[];                 // [kLc1Warps][dim]
+  const int img = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int d8 = dim / 8;
+  const int lo = cu[img], hi = cu[img + 1];
+  uint16_t* ur = u + static_cast<size_t>(img) * 2 * dim;
+  const bool bad = lo < 0 || hi < lo || hi > t_cap;
+  if (bad || hi == lo) {
+    if (bad && threadIdx.x == 0) record_status(status, DORA_ERR_DEVICE_SEQLEN);
+    for (int c = threadIdx.x; c < 2 * dim; c += blockDim.x) ur[c] = 0;
+    return;
+  }
+  for (int c = lane; c < dim; c += 32) acc[warp * dim + c] = 0.f;
+  __syncwarp();
+  constexpr int kChunks = kLc1MaxDim / 8 / 32;
+  for (int j = lo + warp; j < hi; j += kLc1Warps) {
+    const uint4* xr = reinterpret_cast<const uint4*>(x + static_cast<size_t>(j) * dim);
+    uint4 q[kChunks];
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < kChunks; ++i) {
+      const int c8 = lane + 32 * i;
+      q[i] = c8 < d8 ? xr[c8] : make_uint4(0, 0, 0, 0);
+      s += lo_f(q[i].x) + hi_f(q[i].x) + lo_f(q[i].y) + hi_f(q[i].y) + lo_f(q[i].z) +
+           hi_f(q[i].z) + lo_f(q[i].w) + hi_f(q[i].w);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    const float mean = s / dim;
+    float v2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < kChunks; ++i) {
+      if (lane + 32 * i >= d8) continue;
+      const uint32_t wv[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float a = lo_f(wv[e]) - mean, b = hi_f(wv[e]) - mean;
+        v2 += a * a + b * b;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v2 += __shfl_xor_sync(0xffffffffu, v2, o);
+    const float rstd = rsqrtf(v2 / dim + eps);
+#pragma unroll
+    for (int i = 0; i < kChunks; ++i) {
+      const int c8 = lane + 32 * i;
+      if (c8 >= d8) continue;
+      const uint32_t wv[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
+      const uint4 g4 = reinterpret_cast<const uint4*>(gam)[c8];
+      const uint4 b4 = reinterpret_cast<const uint4*>(bet)[c8];
+      const uint32_t gv[4] = {g4.x, g4.y, g4.z, g4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
+      float n[8];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        n[2 * e] = (lo_f(wv[e]) - mean) * rstd * lo_f(gv[e]) + lo_f(bv[e]);
+        n[2 * e + 1] = (hi_f(wv[e]) - mean) * rstd * hi_f(gv[e]) + hi_f(bv[e]);
+      }
+      if (j == lo) {
+        reinterpret_cast<uint4*>(ur)[c8] = make_uint4(pack2(n[0], n[1]), pack2(n[2], n[3]),
+                                                      pack2(n[4], n[5]), pack2(n[6], n[7]));
+      } else {
+        float* a = acc + warp * dim + c8 * 8;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) a[e] += n[e];
+      }
+    }
+  }
+  __syncthreads();
+  const float inv = hi - lo > 1 ? 1.f / static_cast<float>(hi - lo - 1) : 0.f;
+  for (int c = threadIdx.x; c < dim; c += blockDim.x) {
+    float t = 0.f;
+#pragma unroll
+    for (int wp = 0; wp < kLc1Warps; ++wp) t += acc[wp * dim + c];
+    const __nv_bfloat16 hv = __float2bfloat16_rn(t * inv);
+    ur[dim + c] = *reinterpret_cast<const uint16_t*>(&hv);
+  }
+}
+
+// LayerScale fold: out[i, :] = bf16(gamma_i * w[i, :]) and bout[i] =
+// bf16(gamma_i * b_i).  A product of two bf16 values is exact in fp32, so each
+// output is the round-to-nearest-even of the exact product.
+__global__ void layerscale_fold_kernel(const uint4* __restrict__ w, const uint16_t* __restrict__ b,
+                                       const uint16_t* __restrict__ gam, int n, int k8,
+                                       uint4* __restrict__ out, uint16_t* __restrict__ bout) {
+  const long long total = static_cast<long long>(n) * k8;
+  for (long long s = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; s < total;
+       s += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const int row = static_cast<int>(s / k8);
+    const float g = __uint_as_float(static_cast<uint32_t>(gam[row]) << 16);
+    const uint4 v = w[s];
+    out[s] = make_uint4(pack2(g * lo_f(v.x), g * hi_f(v.x)), pack2(g * lo_f(v.y), g * hi_f(v.y)),
+                        pack2(g * lo_f(v.z), g * hi_f(v.z)), pack2(g * lo_f(v.w), g * hi_f(v.w)));
+    if (b != nullptr && s % k8 == 0) {
+      const __nv_bfloat16 hv = __float2bfloat16_rn(g * __uint_as_float(
+                                                           static_cast<uint32_t>(b[row]) << 16));
+      bout[row] = *reinterpret_cast<const uint16_t*>(&hv);
+    }
+  }
+}
+
 size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
 
 int grid_for(long long work) {
@@ -125,7 +287,9 @@ size_t dora_embed_workspace_size(int32_t batch, int32_t channels, int32_t height
                                  int32_t patch, int32_t dim) {
   if (batch < 0 || channels <= 0 || patch <= 0 || height <= 0 || width <= 0 || dim <= 0) return 0;
   const size_t tok = static_cast<size_t>(batch) * (height / patch) * (width / patch);
-  return 256 + embed::up256(tok * channels * patch * patch * 2) + embed::up256(tok * dim * 2);
+  const size_t k = static_cast<size_t>(channels) * patch * patch, kpad = (k + 63) / 64 * 64;
+  return 256 + embed::up256(tok * kpad * 2) + embed::up256(tok * dim * 2) +
+         (kpad != k ? embed::up256(static_cast<size_t>(dim) * kpad * 2) : 0);
 }
 
 int dora_patch_embed(const dora_bf16* images, int32_t batch, int32_t channels, int32_t height,
@@ -133,9 +297,9 @@ int dora_patch_embed(const dora_bf16* images, int32_t batch, int32_t channels, i
                      const dora_bf16* b_pe, const dora_bf16* cls, const dora_bf16* pos,
                      dora_bf16* x0, void* workspace, size_t workspace_bytes,
                      dora_stream_t stream_) {
-  if (batch < 0 || batch > 65535 || channels <= 0 || patch <= 0 || patch % 8 != 0 ||
-      height <= 0 || width <= 0 || height % patch != 0 || width % patch != 0 || dim <= 0 ||
-      dim % 64 != 0 || dim > (1 << 16) || (channels * patch * patch) % 64 != 0)
+  if (batch < 0 || batch > 65535 || channels <= 0 || channels > 64 || patch <= 0 ||
+      patch > 64 || height <= 0 || width <= 0 || height % patch != 0 || width % patch != 0 ||
+      dim <= 0 || dim % 64 != 0 || dim > (1 << 16))
     return DORA_ERR_INVALID_ARG;
   const void* req[] = {images, w_pe, cls, pos, x0, workspace};
   for (const void* p : req)
@@ -154,18 +318,35 @@ int dora_patch_embed(const dora_bf16* images, int32_t batch, int32_t channels, i
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   int32_t* status = reinterpret_cast<int32_t*>(ws);
-  const int k = channels * patch * patch;
+  const int k = channels * patch * patch, kpad = (k + 63) / 64 * 64;
   uint16_t* patches = reinterpret_cast<uint16_t*>(ws + 256);
-  uint16_t* emb = reinterpret_cast<uint16_t*>(ws + 256 + embed::up256(tok * k * 2));
-  const long long segs = static_cast<long long>(batch) * channels * height * (width / 8);
-  embed::patchify_kernel<<<embed::grid_for(segs), 256, 0, stream>>>(
-      reinterpret_cast<const uint4*>(images), batch, channels, height, width, patch,
-      reinterpret_cast<uint4*>(patches));
+  uint16_t* emb = reinterpret_cast<uint16_t*>(ws + 256 + embed::up256(tok * kpad * 2));
+  const uint16_t* w_gemm = w_pe;
+  if (patch % 8 == 0 && kpad == k) {
+    const long long segs = static_cast<long long>(batch) * channels * height * (width / 8);
+    embed::patchify_kernel<<<embed::grid_for(segs), 256, 0, stream>>>(
+        reinterpret_cast<const uint4*>(images), batch, channels, height, width, patch,
+        reinterpret_cast<uint4*>(patches));
+  } else {
+    // K padded to a multiple of the GEMM's 64-wide K step: zero patch columns
+    // and a zero-padded copy of the weights in the workspace
+    uint16_t* wp = reinterpret_cast<uint16_t*>(ws + 256 + embed::up256(tok * kpad * 2) +
+                                               embed::up256(tok * dim * 2));
+    const long long segs = tok * (kpad / 8);
+    embed::patchify_any_kernel<<<embed::grid_for(segs), 256, 0, stream>>>(
+        images, batch, channels, height, width, patch, kpad, reinterpret_cast<uint4*>(patches));
+    if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
+    if (kpad != k) {
+      embed::pad_cols_kernel<<<embed::grid_for(static_cast<long long>(dim) * kpad), 256, 0,
+                               stream>>>(w_pe, dim, k, kpad, wp);
+      w_gemm = wp;
+    }
+  }
   if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
   LinearEpi ep;
   ep.bias = b_pe;
-  if (launch_linear(patches, static_cast<int32_t>(tok), nullptr, k, w_pe, dim, DORA_EPI_BIAS, ep,
-                    emb, status, stream) != cudaSuccess)
+  if (launch_linear(patches, static_cast<int32_t>(tok), nullptr, kpad, w_gemm, dim, DORA_EPI_BIAS,
+                    ep, emb, status, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
   const long long total = static_cast<long long>(batch) * (g + 1) * (dim / 8);
   embed::assemble_kernel<<<embed::grid_for(total), 256, 0, stream>>>(
@@ -215,6 +396,75 @@ int dora_classifier_head(const dora_bf16* x, const int32_t* cu, int32_t batch, i
                        stream) == cudaSuccess
              ? DORA_OK
              : DORA_ERR_CUDA;
+}
+
+size_t dora_head_lc1_workspace_size(int32_t batch, int32_t dim) {
+  if (batch < 0 || dim <= 0) return 0;
+  return 256 + embed::up256(static_cast<size_t>(batch) * 2 * dim * 2);
+}
+
+int dora_classifier_head_lc1(const dora_bf16* x, const int32_t* cu, int32_t batch, int32_t t_cap,
+                             int32_t dim, const dora_bf16* norm_w, const dora_bf16* norm_b,
+                             float eps, const dora_bf16* w_head, const dora_bf16* b_head,
+                             int32_t classes, dora_bf16* logits, void* workspace,
+                             size_t workspace_bytes, dora_stream_t stream_) {
+  if (batch < 0 || batch > 65535 || t_cap < 0 || dim <= 0 || dim % 64 != 0 ||
+      dim > embed::kLc1MaxDim || classes <= 0 || classes % 32 != 0 || classes > (1 << 16) ||
+      !(eps >= 0.f))
+    return DORA_ERR_INVALID_ARG;
+  const void* req[] = {x, cu, norm_w, norm_b, w_head, logits, workspace};
+  for (const void* p : req)
+    if (p == nullptr) return DORA_ERR_INVALID_ARG;
+  const void* al[] = {x, norm_w, norm_b, w_head, b_head, logits};
+  for (const void* p : al)
+    if ((reinterpret_cast<uintptr_t>(p) & 15u) != 0) return DORA_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0 ||
+      workspace_bytes < dora_head_lc1_workspace_size(batch, dim))
+    return DORA_ERR_INVALID_ARG;
+  const int dev = checked_device();
+  if (dev == -1) return DORA_ERR_CUDA;
+  if (dev < 0) return DORA_ERR_UNSUPPORTED;
+  if (batch == 0) return DORA_OK;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  int32_t* status = reinterpret_cast<int32_t*>(ws);
+  uint16_t* u = reinterpret_cast<uint16_t*>(ws + 256);
+  const int smem = embed::kLc1Warps * dim * 4;
+  static bool attr_set[64] = {false};
+  if (dev < 64 && !attr_set[dev]) {
+    if (cudaFuncSetAttribute(embed::lc1_pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             embed::kLc1Warps * embed::kLc1MaxDim * 4) != cudaSuccess)
+      return DORA_ERR_CUDA;
+    attr_set[dev] = true;
+  }
+  embed::lc1_pool_kernel<<<batch, embed::kLc1Warps * 32, smem, stream>>>(
+      x, cu, t_cap, dim, norm_w, norm_b, eps, u, status);
+  if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
+  LinearEpi ep;
+  ep.bias = b_head;
+  return launch_linear(u, batch, nullptr, 2 * dim, w_head, classes, DORA_EPI_BIAS, ep, logits,
+                       status, stream) == cudaSuccess
+             ? DORA_OK
+             : DORA_ERR_CUDA;
+}
+
+int dora_fold_layerscale(const dora_bf16* w, const dora_bf16* b, const dora_bf16* gamma,
+                         int32_t n, int32_t k, dora_bf16* w_out, dora_bf16* b_out,
+                         dora_stream_t stream_) {
+  if (n <= 0 || k <= 0 || k % 8 != 0 || static_cast<long long>(n) * k > (1LL << 34))
+    return DORA_ERR_INVALID_ARG;
+  const void* al[] = {w, gamma, w_out};
+  for (const void* p : al)
+    if (p == nullptr || (reinterpret_cast<uintptr_t>(p) & 15u) != 0) return DORA_ERR_INVALID_ARG;
+  if ((b == nullptr) != (b_out == nullptr)) return DORA_ERR_INVALID_ARG;
+  const int dev = checked_device();
+  if (dev == -1) return DORA_ERR_CUDA;
+  if (dev < 0) return DORA_ERR_UNSUPPORTED;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  embed::layerscale_fold_kernel<<<embed::grid_for(static_cast<long long>(n) * (k / 8)), 256, 0,
+                                  stream>>>(reinterpret_cast<const uint4*>(w), b, gamma, n, k / 8,
+                                            reinterpret_cast<uint4*>(w_out), b_out);
+  return cudaGetLastError() == cudaSuccess ? DORA_OK : DORA_ERR_CUDA;
 }
 
 }  // extern "C"

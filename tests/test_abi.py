@@ -21,7 +21,7 @@ def lib():
 def _declared_functions():
     src = open(os.path.join(ROOT, "include", "dora.h")).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(dora_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(dora_[a-z0-9_]+)\s*\(", src)))
 
 
 def test_header_declares_the_entry_points():
@@ -132,3 +132,24 @@ def test_actor_struct_sizes_and_host_checks(lib):
         a = list(args); a[6] = ctypes.byref(w2)
         assert lib.dora_actor(*a) == 1
         assert lib.dora_actor_prepare(ctypes.byref(w2), 256, 1 << 20, None) == 1
+
+
+def test_dinov2_entry_points_host_checks(lib):
+    # LC1 head: dim above the kernel's register-held row (2048)
+    assert lib.dora_classifier_head_lc1(16, 16, 4, 100, 4096, 16, 16, ctypes.c_float(1e-6), 16,
+                                        16, 1024, 16, 256, 1 << 20, None) == 1
+    # LC1 head: classes not a multiple of 32
+    assert lib.dora_classifier_head_lc1(16, 16, 4, 100, 768, 16, 16, ctypes.c_float(1e-6), 16,
+                                        16, 1000, 16, 256, 1 << 20, None) == 1
+    assert lib.dora_head_lc1_workspace_size(4, 768) >= 256 + 4 * 2 * 768 * 2
+    # LayerScale fold: k % 8, bias without its output
+    assert lib.dora_fold_layerscale(16, None, 16, 8, 12, 16, None, None) == 1
+    assert lib.dora_fold_layerscale(16, 16, 16, 8, 16, 16, None, None) == 1
+    # patch embedding: patch 0, image side not a multiple of the patch
+    assert lib.dora_patch_embed(16, 1, 3, 224, 224, 0, 768, 16, 16, 16, 16, 16, 256, 1 << 30,
+                                None) == 1
+    assert lib.dora_patch_embed(16, 1, 3, 225, 224, 14, 768, 16, 16, 16, 16, 16, 256, 1 << 30,
+                                None) == 1
+    # the 14-pixel patch workspace holds the K-padded (588 -> 640) patches and weight copy
+    n = lib.dora_embed_workspace_size(2, 3, 224, 224, 14, 768)
+    assert n >= 256 + 2 * 256 * 640 * 2 + 2 * 256 * 768 * 2 + 768 * 640 * 2

@@ -1022,7 +1022,10 @@ def test_block_with_actor_equals_actor_then_block(given_counts):
 # ---------------------------------------------------------------------------
 
 @pytest.mark.parametrize("b,c,h,w,patch,d", [(8, 3, 224, 224, 16, 192), (3, 3, 64, 96, 16, 768),
-                                             (2, 4, 32, 32, 8, 128)])
+                                             (2, 4, 32, 32, 8, 128),
+                                             (2, 3, 224, 224, 14, 768),    # DINOv2: K 588 -> 640
+                                             (3, 1, 42, 28, 7, 128),       # K 49 -> 64
+                                             (1, 4, 24, 40, 4, 64)])       # generic path, K 64
 def test_patch_embed_matches_oracle(b, c, h, w, patch, d):
     rng = np.random.default_rng(b * 100 + d)
     g = (h // patch) * (w // patch)
@@ -1066,3 +1069,82 @@ def test_classifier_head_matches_oracle(name):
                             O.bf16_to_f64(b_head))
     assert_close(f64(logits), ref, f"classifier {name}")
     assert torch.all(logits[:, 1000:] == 0)
+
+
+# ---------------------------------------------------------------------------
+# DINOv2 backbone: LayerScale fold, LayerScale blocks, LC1 readout
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,k,bias,inplace", [(768, 768, True, False), (768, 3072, True, True),
+                                              (96, 40, False, False)])
+def test_fold_layerscale_bit_exact(n, k, bias, inplace):
+    """A bf16 x bf16 product is exact in fp32, so the fold is the
+    round-to-nearest-even of gamma_i * w_ij: checked bit for bit."""
+    rng = np.random.default_rng(n + k)
+    w = S.f32_to_bf16_bits(rng.standard_normal((n, k)) * 0.05)
+    b = S.f32_to_bf16_bits(rng.standard_normal(n) * 0.02)
+    g = S.f32_to_bf16_bits(rng.uniform(0.05, 0.5, n) * np.where(rng.random(n) < 0.1, -1, 1))
+    wt, bt, gt = bf(w), bf(b) if bias else None, bf(g)
+    wo, bo = P.dora_fold_layerscale(wt, bt, gt, w_out=wt if inplace else None,
+                                    b_out=bt if inplace and bias else None)
+    torch.cuda.synchronize()
+    gf = O.bf16_to_f64(g).astype(np.float32)
+    want_w = S.f32_to_bf16_bits(gf[:, None] * O.bf16_to_f64(w).astype(np.float32))
+    got_w = wo.cpu().view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(got_w, want_w)
+    if bias:
+        want_b = S.f32_to_bf16_bits(gf * O.bf16_to_f64(b).astype(np.float32))
+        assert np.array_equal(bo.cpu().view(torch.int16).numpy().view(np.uint16), want_b)
+
+
+def test_dinov2_block_with_layerscale():
+    """A DINOv2-B/14 block (257 tokens, LayerScale on both branches) pruned
+    by scores: the block on folded weights against the oracle's block with
+    the scales applied to the branch outputs."""
+    cfg = S.get_config("cfg6", batch=6)
+    cu, ids = S.initial_layout(cfg)
+    x = S.activations_bf16(cfg, 41)
+    wb = S.block_weights(cfg, 3, 41, random_affine=True)
+    assert "ls1" in wb and "ls2" in wb
+    keeps, _ = S.keep_schedule(cfg, 41)
+    scores = O.gather_scores(S.score_table(cfg, 3, 41), cu, ids)
+    w = _device_weights(cfg, wb)
+    r = _run_block(cfg, x, cu, ids, w, scores, keeps[0])
+    assert r["status"] == 0
+    ref = O.pruned_block(O.bf16_to_f64(x), cu, ids, O.decode_weights(wb), cfg.heads, cfg.ln_eps,
+                         scores, keeps[0])
+    t_out = int(ref["cu_out"][-1])
+    assert np.array_equal(r["cu_out"], ref["cu_out"])
+    assert np.array_equal(r["kept"][:t_out], ref["kept_idx"])
+    assert_close(f64(r["x_out"][:t_out]), ref["x_out"], "dinov2 block")
+
+
+@pytest.mark.parametrize("name,dim", [("cfg6", 768), ("cfg1", 192), ("cfg4", 1024)])
+def test_classifier_head_lc1_matches_oracle(name, dim):
+    cfg = S.get_config(name, batch=24)
+    keeps, _ = S.keep_schedule(cfg, 17)
+    lens = np.array(keeps[-1])
+    lens[3] = 1                                      # CLS only: zero visual mean
+    lens[5] = 2                                      # one visual token
+    lens[7] = 0                                      # empty image
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    rng = np.random.default_rng(17)
+    x = S.f32_to_bf16_bits(rng.uniform(-3, 3, (t, 1)) + rng.standard_normal((t, dim)))
+    nw = S.f32_to_bf16_bits(1 + 0.1 * rng.standard_normal(dim))
+    nb = S.f32_to_bf16_bits(0.1 * rng.standard_normal(dim))
+    classes = 1024
+    w_head = np.zeros((classes, 2 * dim), np.uint16)
+    w_head[:1000] = S.f32_to_bf16_bits(rng.standard_normal((1000, 2 * dim)) / np.sqrt(2 * dim))
+    b_head = np.zeros(classes, np.uint16)
+    b_head[:1000] = S.f32_to_bf16_bits(0.02 * rng.standard_normal(1000))
+    logits = torch.full((cfg.batch, classes), 9.0, dtype=torch.bfloat16, device=dev())
+    ws = P.dora_classifier_head_lc1(bf(x), i32(cu), bf(nw), bf(nb), 1e-6, bf(w_head), bf(b_head),
+                                    logits)
+    torch.cuda.synchronize()
+    assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
+    ref = O.classifier_head_lc1(O.bf16_to_f64(x), cu, O.bf16_to_f64(nw), O.bf16_to_f64(nb), 1e-6,
+                                O.bf16_to_f64(w_head), O.bf16_to_f64(b_head))
+    assert_close(f64(logits), ref, f"lc1 head {name}")
+    assert torch.all(logits[:, 1000:] == 0)
+
