@@ -41,12 +41,13 @@ UNIT = "images/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM traffic per GEMM launch from an ncu capture (dram__bytes_read.sum +
-# dram__bytes_write.sum), keyed by the sha256 of the kernel source it was
-# taken on; reported as null once the source changes.
+# dram__bytes_write.sum), keyed by the workload and the sha256 of the kernel
+# source it was taken on; reported as null once the source changes and for a
+# workload without a capture.
 NCU_TRAFFIC = {
     # profiles/gemm_tcgen05_deit_base_b256.md: mean over the 48 GEMM launches
     # of one forward step
-    "b34dcbc477c16fbd82653b7888b9deb4fa8716d95e482f5d9899e205d6137ff3": 188246208,
+    ("cfg3", "b34dcbc477c16fbd82653b7888b9deb4fa8716d95e482f5d9899e205d6137ff3"): 188246208,
 }
 
 
@@ -587,7 +588,7 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
     # per-kernel pass: the same step driven kernel by kernel with events
     kern = profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap,
                            steps=max(3, min(args.steps, 20)))
-    result.update(roofline_report(kern, peaks, peak_src))
+    result.update(roofline_report(kern, peaks, peak_src, args.config))
     return result, hw
 
 
@@ -758,12 +759,12 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
     return agg
 
 
-def roofline_report(kern, peaks, peak_src):
+def roofline_report(kern, peaks, peak_src, workload):
     tag = f"of {peak_src}"
     g = kern["gemm"]
     gemm_tf = g["flops"] / (g["ms"] * 1e-3) / 1e12
     src = os.path.join(ROOT, "paper_2609_34325_gb300", "csrc", "gemm_tcgen05.cu")
-    tr = NCU_TRAFFIC.get(sha256_of(src))
+    tr = NCU_TRAFFIC.get((workload, sha256_of(src)))
     out = {"roofline": {"kernel": "gemm_tcgen05 (QKV/proj/fc1/fc2)", "bound": "tensor",
                         "achieved": round(gemm_tf, 1), "peak": peaks["bf16_tflops_sustained"],
                         "unit": "TFLOP/s", "frac": round(gemm_tf / peaks["bf16_tflops_sustained"], 4),

@@ -30,8 +30,11 @@ block of Eq. 1 (Sec. 3.1), in float64, from bf16/fp32 inputs decoded exactly:
                     paper's GFLOPs and throughput include (App. E.4): the
                     strided patch convolution with CLS and position
                     embeddings, and LayerNorm + linear on each CLS row.
+* ``lc1_readout``, ``classifier_head_lc1``, LayerScale in the block halves
+                    the DINOv2-B/14 backbone (App. E.2): LayerScale on both
+                    residual branches and the LC1 readout.
 
-Readings where the paper is silent (all listed in the design doc):
+Readings where the paper is silent:
 
 * Ties: among equal scores the lower index is kept (equivalently the higher
   index is removed first).  Scores are ordered by a total order on fp32:
@@ -44,6 +47,9 @@ Readings where the paper is silent (all listed in the design doc):
   the smaller removal count; the encoder's attention scale is 1/sqrt(32);
   every image gets a budget and selector scores (the gate only decides
   whether they are used); E_<l / (L - 1) divides by 1 when L = 1.
+* DINOv2: LayerScale multiplies each branch's output (after its last linear,
+  before the residual add) per channel; the LC1 mean runs over the visual
+  rows that survive the last deletion, zero when none does.
 
 Parity pins: every function here is checked in ``tests/test_oracle_pins.py``
 against brute force, closed forms, invariants the paper fixes, or an

@@ -763,7 +763,7 @@ def test_block_chained_row_moments():
     assert_close(f64(outs[1][:t_out]), f64(outs[0][:t_out]), "chained vs unchained")
 
 
-@pytest.mark.parametrize("name", ["cfg3", "cfg4", "cfg5"])
+@pytest.mark.parametrize("name", ["cfg3", "cfg4", "cfg5", "cfg6"])
 def test_block_full_size_sampled_images(name):
     cfg = S.get_config(name)
     cu, ids = S.initial_layout(cfg)
