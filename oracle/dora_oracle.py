@@ -30,6 +30,10 @@ block of Eq. 1 (Sec. 3.1), in float64, from bf16/fp32 inputs decoded exactly:
                     paper's GFLOPs and throughput include (App. E.4): the
                     strided patch convolution with CLS and position
                     embeddings, and LayerNorm + linear on each CLS row.
+* ``pl_sample_gumbel``, ``pl_logprob``, ``pl_logprob_grad``, ``kd_cost``
+                    the training side: Plackett-Luce ordered sampling and
+                    log-probability (App. A.3) and the shadows' fidelity cost
+                    (App. B.2).
 * ``lc1_readout``, ``classifier_head_lc1``, LayerScale in the block halves
                     the DINOv2-B/14 backbone (App. E.2): LayerScale on both
                     residual branches and the LC1 readout.
@@ -50,6 +54,9 @@ Readings where the paper is silent:
 * DINOv2: LayerScale multiplies each branch's output (after its last linear,
   before the residual add) per channel; the LC1 mean runs over the visual
   rows that survive the last deletion, zero when none does.
+* Training: the ordered sample is the Gumbel-top-k of the scores (keys
+  formed in fp32, noise an input); the fidelity cost runs over the true
+  classes only.
 
 Parity pins: every function here is checked in ``tests/test_oracle_pins.py``
 against brute force, closed forms, invariants the paper fixes, or an
@@ -532,3 +539,83 @@ def classifier_head_lc1(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: n
     """Class logits from the LC1 features (App. E.2): the linear layer
     w_head [classes, 2 d] applied to lc1_readout's [B, 2 d] rows."""
     return linear(lc1_readout(x, cu, ln_w, ln_b, eps), w_head, b_head)
+
+
+# ----------------------------------------------------------------------------
+# O8: training side (App. A.3 "Training-time sampling"; App. B.2-B.3 shadow
+# evaluation and its fidelity cost)
+# ----------------------------------------------------------------------------
+
+def pl_sample_gumbel(scores: np.ndarray, gumbel: np.ndarray, k: int) -> np.ndarray:
+    """Ordered removal sequence (i_1, ..., i_k) drawn without replacement from
+    the Plackett-Luce distribution of the selector scores (App. A.3), as the
+    Gumbel-top-k of the scores: the k largest keys s_j + g_j in decreasing
+    order, g_j standard Gumbel noise supplied by the caller.  The keys are
+    formed in fp32 (the precision the decision is taken in on both sides);
+    ties go to the lower index, -0 equals +0 and NaN ranks above +inf."""
+    s = np.asarray(scores, dtype=np.float32)
+    g = np.asarray(gumbel, dtype=np.float32)
+    keys = score_order_key((s + g).astype(np.float32))
+    order = sorted(range(len(s)), key=lambda j: (-int(keys[j]), j))
+    return np.array(order[:k], dtype=np.int64)
+
+
+def _logsumexp(v: np.ndarray) -> float:
+    v = np.asarray(v, dtype=np.float64)
+    m = float(np.max(v))
+    return m + math.log(float(np.sum(np.exp(v - m))))
+
+
+def pl_logprob(scores: np.ndarray, order: np.ndarray) -> float:
+    """Plackett-Luce log-probability of the ordered sequence (App. A.3):
+    sum over t of s_{i_t} - log sum_{j in R_t} exp(s_j), with R_t the indices
+    not yet removed before step t."""
+    s = np.asarray(scores, dtype=np.float64)
+    remaining = list(range(len(s)))
+    total = 0.0
+    for i in order:
+        total += s[int(i)] - _logsumexp(s[remaining])
+        remaining.remove(int(i))
+    return total
+
+
+def pl_logprob_grad(scores: np.ndarray, order: np.ndarray) -> np.ndarray:
+    """Gradient of pl_logprob with respect to every score: each step t adds 1
+    at i_t and subtracts the softmax of the scores over R_t."""
+    s = np.asarray(scores, dtype=np.float64)
+    grad = np.zeros(len(s))
+    remaining = list(range(len(s)))
+    for i in order:
+        r = np.array(remaining)
+        p = np.exp(s[r] - _logsumexp(s[r]))
+        grad[r] -= p
+        grad[int(i)] += 1.0
+        remaining.remove(int(i))
+    return grad
+
+
+def log_softmax(z: np.ndarray) -> np.ndarray:
+    z = np.asarray(z, dtype=np.float64)
+    return z - _logsumexp(z)
+
+
+def kd_cost(z_native: np.ndarray, z: np.ndarray, tau: float = 3.0) -> float:
+    """Per-image fidelity cost of a shadow (App. B.2): tau^2 times the KL
+    divergence from softmax(z_native / tau) to softmax(z / tau), tau = 3."""
+    lp_n = log_softmax(np.asarray(z_native, dtype=np.float64) / tau)
+    lp = log_softmax(np.asarray(z, dtype=np.float64) / tau)
+    return tau * tau * float(np.sum(np.exp(lp_n) * (lp_n - lp)))
+
+
+def shadow_forwards(x: np.ndarray, cu: np.ndarray, ids: np.ndarray, blocks: list, heads: int,
+                    eps: float, prune: dict, head_dim: int = 64) -> dict:
+    """Complete-prefix shadows (App. B.2): for each pruning block l of the
+    rollout, the forward that replays the rollout's deletions at blocks
+    0..l and runs every later block without deletion; key -1 is the empty
+    prefix (the Native forward).  Each value is forward()'s result."""
+    out = {-1: forward(x, cu, ids, blocks, heads, eps, {}, head_dim)}
+    for l in sorted(prune):
+        out[l] = forward(x, cu, ids, blocks, heads, eps,
+                         {b: v for b, v in prune.items() if b <= l}, head_dim)
+    return out
+

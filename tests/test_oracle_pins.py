@@ -6,6 +6,8 @@ import math
 import os
 
 import numpy as np
+import scipy.special
+import scipy.stats
 import pytest
 import torch
 
@@ -410,6 +412,12 @@ def test_compression_identity_and_calibration():
         c = S.compression_from_counts(cfg, *S.keep_schedule(cfg, seed))
         assert abs(c.mean() - 0.38) <= 0.01
         assert c.min() < 0.30 and c.max() > 0.45          # per-image spread
+    # DINOv2-B: the paper reports 22.9-40.1% compression, mean 34.8% (Sec. 4.3)
+    cfg = S.get_config("cfg6")
+    for seed in range(3):
+        c = S.compression_from_counts(cfg, *S.keep_schedule(cfg, seed))
+        assert abs(c.mean() - 0.348) <= 0.01
+        assert c.min() < 0.26 and c.max() > 0.40
 
 
 # ---------------------------------------------------------------------------
@@ -670,3 +678,120 @@ def test_lc1_readout_loops_and_invariants():
     xp = x.copy()
     xp[8:11] = x[[10, 8, 9]]
     assert np.allclose(O.lc1_readout(xp, cu, g, be, 1e-6), r, rtol=0, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# training side: Plackett-Luce sampling / log-probability (App. A.3), the
+# shadows' fidelity cost (App. B.2)
+# ---------------------------------------------------------------------------
+
+def test_pl_logprob_is_a_distribution_over_ordered_sequences():
+    """exp(log pi) summed over every ordered k-sequence of n items is 1, and a
+    sequential draw's probabilities multiply out to it."""
+    rng = np.random.default_rng(3)
+    for n, k in ((4, 1), (5, 2), (5, 3), (4, 4)):
+        s = rng.standard_normal(n) * 2
+        tot = sum(math.exp(O.pl_logprob(s, np.array(p)))
+                  for p in itertools.permutations(range(n), k))
+        assert abs(tot - 1) < 1e-12
+        # hand product for one sequence
+        seq = list(itertools.permutations(range(n), k))[-1]
+        prob, rem = 1.0, list(range(n))
+        for i in seq:
+            prob *= math.exp(s[i]) / sum(math.exp(s[j]) for j in rem)
+            rem.remove(i)
+        assert abs(math.log(prob) - O.pl_logprob(s, np.array(seq))) < 1e-12
+
+
+def test_pl_logprob_closed_forms():
+    rng = np.random.default_rng(4)
+    s = rng.standard_normal(9)
+    # k = 1: the log-softmax entry; equal scores: -sum_t log(n - t + 1)
+    for i in range(9):
+        assert abs(O.pl_logprob(s, np.array([i])) - scipy.special.log_softmax(s)[i]) < 1e-12
+    order = np.array([4, 0, 7, 2])
+    assert abs(O.pl_logprob(np.full(9, 0.3), order) + sum(math.log(9 - t) for t in range(4))) \
+        < 1e-12
+    # shift invariance; a full permutation's last step contributes 0
+    assert abs(O.pl_logprob(s + 5.0, order) - O.pl_logprob(s, order)) < 1e-12
+    full = np.array([3, 1, 8, 0, 2, 5, 4, 7, 6])
+    assert abs(O.pl_logprob(s, full) - O.pl_logprob(s, full[:-1])) < 1e-12
+
+
+def test_pl_logprob_grad_matches_finite_differences():
+    rng = np.random.default_rng(5)
+    s = rng.standard_normal(7)
+    order = np.array([2, 6, 0])
+    g = O.pl_logprob_grad(s, order)
+    h = 1e-6
+    for j in range(7):
+        e = np.zeros(7)
+        e[j] = h
+        fd = (O.pl_logprob(s + e, order) - O.pl_logprob(s - e, order)) / (2 * h)
+        assert abs(fd - g[j]) < 1e-8
+    assert abs(g.sum()) < 1e-12                       # shift invariance
+
+
+def test_gumbel_top_k_is_a_plackett_luce_sample():
+    """The Gumbel-top-k order has the Plackett-Luce law: empirical frequencies
+    of every ordered pair of 4 items against exp(log pi), within 5 sigma."""
+    rng = np.random.default_rng(6)
+    s = np.array([0.8, -0.4, 0.1, 1.5], dtype=np.float32)
+    draws = 40000
+    counts = {}
+    u = rng.random((draws, 4))
+    gum = -np.log(-np.log(u))
+    for r in range(draws):
+        key = tuple(O.pl_sample_gumbel(s, gum[r], 2))
+        counts[key] = counts.get(key, 0) + 1
+    for seq in itertools.permutations(range(4), 2):
+        p = math.exp(O.pl_logprob(s.astype(np.float64), np.array(seq)))
+        f = counts.get(seq, 0) / draws
+        assert abs(f - p) <= 5 * math.sqrt(p * (1 - p) / draws), (seq, f, p)
+
+
+def test_gumbel_top_k_order_rules():
+    s = np.array([0.5, 2.0, -1.0, 2.0, 0.0, -0.0, np.nan], dtype=np.float32)
+    z = np.zeros(7, dtype=np.float32)
+    # NaN first, equal keys by lower index, -0 == +0
+    assert O.pl_sample_gumbel(s, z, 7).tolist() == [6, 1, 3, 0, 4, 5, 2]
+    assert O.pl_sample_gumbel(s[:6], z[:6], 2).tolist() == [1, 3]
+    # keys are fp32 sums: 1 + 2^-24 rounds to 1, so index order decides
+    a = np.array([1.0, 1.0], dtype=np.float32)
+    g = np.array([2.0 ** -24, 0.0], dtype=np.float32)
+    assert O.pl_sample_gumbel(a, g[::-1].copy(), 2).tolist() == [0, 1]
+
+
+def test_kd_cost_pins():
+    rng = np.random.default_rng(7)
+    zn, z = rng.standard_normal(10) * 4, rng.standard_normal(10) * 4
+    assert O.kd_cost(zn, zn) == 0.0
+    assert O.kd_cost(zn, z) > 0                        # Gibbs
+    pn = scipy.special.softmax(zn / 3)
+    q = scipy.special.softmax(z / 3)
+    assert abs(O.kd_cost(zn, z) - 9 * scipy.stats.entropy(pn, q)) < 1e-12
+    # two classes: tau^2 [p log(p/q) + (1-p) log((1-p)/(1-q))] with logistic p, q
+    a, b = 1.7, -0.6
+    p, qq = 1 / (1 + math.exp(-a / 3)), 1 / (1 + math.exp(-b / 3))
+    closed = 9 * (p * math.log(p / qq) + (1 - p) * math.log((1 - p) / (1 - qq)))
+    assert abs(O.kd_cost(np.array([a, 0.0]), np.array([b, 0.0])) - closed) < 1e-12
+    # invariant to a constant added to either logit vector
+    assert abs(O.kd_cost(zn + 3, z - 2) - O.kd_cost(zn, z)) < 1e-12
+
+
+def test_shadow_prefixes_end_at_native_and_rollout():
+    """The empty prefix is the dense forward, the full prefix the rollout; a
+    prefix ending at block l equals the rollout through block l."""
+    cfg = S.get_config("cfg1", batch=2, depth=3, prune_blocks=(0, 2))
+    cu, ids = S.initial_layout(cfg)
+    x = O.bf16_to_f64(S.activations_bf16(cfg, 8))
+    blocks = [O.decode_weights(S.block_weights(cfg, l, 8)) for l in range(3)]
+    keeps, _ = S.keep_schedule(cfg, 8)
+    prune = {l: (S.score_table(cfg, l, 8), keeps[j]) for j, l in enumerate(cfg.prune_blocks)}
+    sh = O.shadow_forwards(x, cu, ids, blocks, cfg.heads, cfg.ln_eps, prune)
+    dense = O.forward(x, cu, ids, blocks, cfg.heads, cfg.ln_eps)
+    roll = O.forward(x, cu, ids, blocks, cfg.heads, cfg.ln_eps, prune)
+    assert np.array_equal(sh[-1]["x"], dense["x"])
+    assert np.array_equal(sh[2]["x"], roll["x"])
+    assert np.array_equal(sh[0]["kept"][0], roll["kept"][0])
+    assert np.array_equal(sh[0]["cu"], O.cu_from_counts(keeps[0]))
