@@ -583,6 +583,68 @@ int dora_fold_layerscale(const dora_bf16* w, const dora_bf16* b, const dora_bf16
                          int32_t n, int32_t k, dora_bf16* w_out, dora_bf16* b_out,
                          dora_stream_t stream);
 
+/*
+ * Training side (App. A.3 "Training-time sampling and deterministic
+ * inference"; App. B.2 "Shadow evaluation procedure").  Scores are fp32,
+ * row-aligned with the packed tokens (cu int32 [batch + 1]); each image's CLS
+ * row cu[i] takes no part, visual token j of image i is row cu[i] + 1 + j, and
+ * an image holds at most 2048 visual tokens (longer: DORA_ERR_DEVICE_SEQLEN,
+ * treated as empty).  Device errors go to *status (nullable device int32).
+ *
+ * dora_pl_sample -- the ordered removal sequence (i_1..i_k) of each image,
+ * drawn without replacement from the Plackett-Luce distribution of its scores
+ * as the Gumbel-top-k: the k_i largest keys s_j + g_j (fp32 sum; -0 == +0,
+ * NaN above +inf, equal keys by lower j) in decreasing order.  gumbel fp32
+ * [t_cap] row-aligned standard Gumbel noise, drawn by the caller; k int32
+ * [batch] (device); order int32 [batch, k_cap] out: order[i, t] = j of the
+ * (t+1)-th removal, -1 for t >= k_i.  k_i outside [0, min(n_i, k_cap)] is
+ * clamped and raises DORA_ERR_DEVICE_BAD_COUNT.
+ */
+int dora_pl_sample(const float* scores, const float* gumbel, const int32_t* cu, int32_t batch,
+                   int32_t t_cap, const int32_t* k, int32_t k_cap, int32_t* order,
+                   int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_pl_logprob -- logp fp32 [batch]: log pi_S(i | k) = sum_t [s_{i_t} -
+ * log sum_{j in R_t} exp(s_j)], R_t the visual tokens not removed before step
+ * t (App. A.3), for the sequences in order int32 [batch, k_cap] (the first k_i
+ * entries used).  grad fp32 [t_cap] (nullable): dlogp_i * d log pi / d s_j for
+ * every visual row (CLS rows 0), dlogp fp32 [batch] (nullable: 1).  fp32,
+ * log-sum-exp scans without cancellation.  A sequence entry outside
+ * [0, n_i) or repeated gives logp NaN, NaN gradients and
+ * DORA_ERR_DEVICE_BAD_COUNT.
+ */
+int dora_pl_logprob(const float* scores, const int32_t* cu, int32_t batch, int32_t t_cap,
+                    const int32_t* k, const int32_t* order, int32_t k_cap, float* logp,
+                    float* grad, const float* dlogp, int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_branch -- complete-prefix shadows as extra sequences of the packed
+ * batch (App. B.2): the rows of sequences src int32 [n_branch] (device, each
+ * in [0, batch)) are copied, in order, after row cu[batch] of x bf16
+ * [t_cap, dim] (in place), with their ids int32 [t_cap] and row moments
+ * x_moments fp32 [t_cap, 2] (both nullable).  cu_out int32 [batch + 1 +
+ * n_branch]: cu followed by the appended sequences' ends (cu_out == cu is
+ * allowed when it has the room); len_out int32 [n_branch] (nullable): their
+ * lengths, which are also their keep counts at every later block.  Rows past
+ * t_cap are not written (DORA_ERR_DEVICE_SEQLEN, the sequence gets length 0).
+ */
+int dora_branch(dora_bf16* x, int32_t* ids, float* x_moments, const int32_t* cu, int32_t batch,
+                int32_t t_cap, int32_t dim, const int32_t* src, int32_t n_branch,
+                int32_t* cu_out, int32_t* len_out, int32_t* status, dora_stream_t stream);
+
+/*
+ * dora_kd_cost -- cost fp32 [shadows]: D = tau^2 sum_c p^N_c log(p^N_c /
+ * p_c), p^N = softmax(z_native[img] / tau), p = softmax(z[s] / tau) over the
+ * first `classes` columns (App. B.2; tau = 3 there).  z_native bf16
+ * [batch, ld], z bf16 [shadows, ld] (row pitch ld >= classes: padded heads);
+ * shadow_image int32 [shadows] (device, nullable: shadow s compares with
+ * image s); fp32 arithmetic.
+ */
+int dora_kd_cost(const dora_bf16* z_native, const dora_bf16* z, const int32_t* shadow_image,
+                 int32_t shadows, int32_t batch, int32_t classes, int32_t ld, float tau,
+                 float* cost, int32_t* status, dora_stream_t stream);
+
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug
  * only: it blocks the host. */

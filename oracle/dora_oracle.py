@@ -70,6 +70,7 @@ import numpy as np
 
 DORA_OK = 0
 DORA_ERR_DEVICE_BAD_COUNT = 5
+DORA_ERR_DEVICE_SEQLEN = 6
 
 
 # ----------------------------------------------------------------------------

@@ -25,6 +25,7 @@ __all__ = [
     "dora_merge_moments", "ActorWeights", "dora_actor", "dora_actor_workspace_size",
     "alloc_actor_workspace", "dora_pruned_block_actor", "dora_patch_embed",
     "dora_classifier_head", "dora_classifier_head_lc1", "dora_fold_layerscale",
+    "dora_pl_sample", "dora_pl_logprob", "dora_branch", "dora_kd_cost",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -79,6 +80,12 @@ _SIGS = {
     "dora_classifier_head_lc1": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _f32, _vp,
                                                 _vp, _i32, _vp, _vp, _sz, _vp]),
     "dora_fold_layerscale": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp]),
+    "dora_pl_sample": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _i32, _vp, _vp, _vp]),
+    "dora_pl_logprob": (ctypes.c_int, [_vp, _vp, _i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp,
+                                       _vp]),
+    "dora_branch": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _vp, _i32, _vp, _vp, _vp,
+                                   _vp]),
+    "dora_kd_cost": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _i32, _f32, _vp, _vp, _vp]),
     "dora_classifier_head": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _f32, _vp, _vp,
                                             _i32, _vp, _vp, _sz, _vp]),
     "dora_pruned_block_actor": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
@@ -712,3 +719,84 @@ def dora_classifier_head(x, cu, norm_w, norm_b, eps, w_head, b_head, logits, wor
                                                _ptr(workspace), workspace.numel(),
                                                _stream(stream)), "dora_classifier_head")
     return workspace
+
+
+# ---------------------------------------------------------------------------
+# training side: Plackett-Luce sampling and log-probability, shadow branching,
+# fidelity cost
+# ---------------------------------------------------------------------------
+
+def dora_pl_sample(scores, gumbel, cu, k, order, status=None, stream=None):
+    """Gumbel-top-k removal sequences: order int32 [B, k_cap] (-1 past k_i)."""
+    _req(scores, torch.float32, "scores")
+    _req(gumbel, torch.float32, "gumbel")
+    _req(cu, torch.int32, "cu")
+    _req(k, torch.int32, "k")
+    _req(order, torch.int32, "order")
+    b = cu.numel() - 1
+    if order.dim() != 2 or order.shape[0] != b or k.numel() != b:
+        raise ValueError("order must be [B, k_cap] and k [B]")
+    _check(load_library().dora_pl_sample(_ptr(scores), _ptr(gumbel), _ptr(cu), b, scores.numel(),
+                                         _ptr(k), order.shape[1], _ptr(order), _ptr(status),
+                                         _stream(stream)), "dora_pl_sample")
+    return order
+
+
+def dora_pl_logprob(scores, cu, k, order, logp, grad=None, dlogp=None, status=None, stream=None):
+    """Plackett-Luce log-probabilities logp [B] and, optionally, their gradient
+    with respect to the row-aligned scores (times dlogp)."""
+    _req(scores, torch.float32, "scores")
+    _req(cu, torch.int32, "cu")
+    _req(k, torch.int32, "k")
+    _req(order, torch.int32, "order")
+    _req(logp, torch.float32, "logp")
+    _req(grad, torch.float32, "grad", optional=True)
+    _req(dlogp, torch.float32, "dlogp", optional=True)
+    b = cu.numel() - 1
+    if order.dim() != 2 or order.shape[0] != b or logp.numel() != b:
+        raise ValueError("order must be [B, k_cap] and logp [B]")
+    if grad is not None and grad.numel() != scores.numel():
+        raise ValueError("grad must match scores")
+    _check(load_library().dora_pl_logprob(_ptr(scores), _ptr(cu), b, scores.numel(), _ptr(k),
+                                          _ptr(order), order.shape[1], _ptr(logp), _ptr(grad),
+                                          _ptr(dlogp), _ptr(status), _stream(stream)),
+           "dora_pl_logprob")
+    return logp
+
+
+def dora_branch(x, cu, src, cu_out, ids=None, x_moments=None, len_out=None, status=None,
+                stream=None):
+    """Append copies of sequences src (device int32) after row cu[-1] of x,
+    in place; cu_out [B + 1 + len(src)]."""
+    _req(x, torch.bfloat16, "x")
+    _req(cu, torch.int32, "cu")
+    _req(src, torch.int32, "src")
+    _req(cu_out, torch.int32, "cu_out")
+    _req(ids, torch.int32, "ids", optional=True)
+    _req(x_moments, torch.float32, "x_moments", optional=True)
+    _req(len_out, torch.int32, "len_out", optional=True)
+    b, nb = cu.numel() - 1, src.numel()
+    if cu_out.numel() < b + 1 + nb:
+        raise ValueError("cu_out needs B + 1 + len(src) entries")
+    t_cap, d = x.shape
+    _check(load_library().dora_branch(_ptr(x), _ptr(ids), _ptr(x_moments), _ptr(cu), b, t_cap, d,
+                                      _ptr(src), nb, _ptr(cu_out), _ptr(len_out), _ptr(status),
+                                      _stream(stream)), "dora_branch")
+    return cu_out
+
+
+def dora_kd_cost(z_native, z, cost, classes, shadow_image=None, tau=3.0, status=None,
+                 stream=None):
+    """Fidelity costs [S]: tau^2 KL(softmax(z_native[img] / tau) || softmax(z[s] / tau))
+    over the first `classes` logits of each row."""
+    _req(z_native, torch.bfloat16, "z_native")
+    _req(z, torch.bfloat16, "z")
+    _req(cost, torch.float32, "cost")
+    _req(shadow_image, torch.int32, "shadow_image", optional=True)
+    if z.shape[1] != z_native.shape[1] or cost.numel() != z.shape[0]:
+        raise ValueError("z and z_native need the same row pitch; cost one entry per row of z")
+    _check(load_library().dora_kd_cost(_ptr(z_native), _ptr(z), _ptr(shadow_image), z.shape[0],
+                                       z_native.shape[0], int(classes), z.shape[1], float(tau),
+                                       _ptr(cost), _ptr(status), _stream(stream)), "dora_kd_cost")
+    return cost
+

@@ -18,7 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libdora.so")
 SOURCES = ["token_ops.cu", "gemm_tcgen05.cu", "attn_tcgen05.cu", "api.cu", "noalloc.cu",
-           "actor.cu", "embed_head.cu"]
+           "actor.cu", "embed_head.cu", "training.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -1,0 +1,346 @@
+"""GPU parity of the training side (App. A.3 sampling and log-probability;
+App. B.2 complete-prefix shadows and their fidelity cost) through the C ABI,
+against the fp64 oracle on the same seeded inputs.  Sampled orders, sequence
+boundaries, ids and branched rows must match bit for bit; log-probabilities,
+gradients and costs within the fp32 bounds stated in each test."""
+import numpy as np
+import pytest
+import scipy.special
+import torch
+
+import __graft_entry__ as G
+import dora_synth as S
+import oracle as O
+import paper_2609_34325_gb300 as P
+from helpers import assert_close, bf, bits, dev, f32, f64, i32
+from paper_2609_34325_gb300.shadow import ShadowRollout
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA device")
+    G.build()
+    P.load_library()
+    torch.cuda.set_device(0)
+
+
+def _status():
+    return torch.zeros(1, dtype=torch.int32, device=dev())
+
+
+def _gumbel(rng, t):
+    u = rng.random(t)
+    return (-np.log(-np.log(u))).astype(np.float32)
+
+
+def _pruned_layout(name, seed, block=-1):
+    cfg = S.get_config(name)
+    keeps, _ = S.keep_schedule(cfg, seed)
+    lens = np.asarray(keeps[block]) if block is not None else np.full(cfg.batch, cfg.n_tokens)
+    return O.cu_from_counts(lens)
+
+
+def _run_sample(scores, gumbel, cu, k, k_cap):
+    b = len(cu) - 1
+    order = torch.full((b, k_cap), 77, dtype=torch.int32, device=dev())
+    st = _status()
+    P.dora_pl_sample(f32(scores), f32(gumbel), i32(cu), i32(k), order, status=st)
+    torch.cuda.synchronize()
+    return order.cpu().numpy(), int(st.item())
+
+
+def _oracle_orders(scores, gumbel, cu, k, k_cap):
+    out = np.full((len(cu) - 1, k_cap), -1, dtype=np.int64)
+    for i in range(len(cu) - 1):
+        lo, hi = int(cu[i]), int(cu[i + 1])
+        n = max(hi - lo - 1, 0)
+        if n == 0 or k[i] == 0:
+            continue
+        out[i, :k[i]] = O.pl_sample_gumbel(scores[lo + 1:hi], gumbel[lo + 1:hi], int(k[i]))
+    return out
+
+
+@pytest.mark.parametrize("name,block", [("cfg1", None), ("cfg3", 0), ("cfg3", -1),
+                                        ("cfg5", None)])
+def test_pl_sample_bit_exact(name, block):
+    cu = _pruned_layout(name, 3, block)
+    t = int(cu[-1])
+    rng = np.random.default_rng(t)
+    scores = rng.standard_normal(t).astype(np.float32) * 2
+    gumbel = _gumbel(rng, t)
+    n = np.diff(cu) - 1
+    k = np.array([rng.integers(0, m + 1) for m in n])
+    k[0] = n[0]                                         # a full permutation
+    k_cap = int(n.max())
+    got, st = _run_sample(scores, gumbel, cu, k, k_cap)
+    assert st == 0
+    assert np.array_equal(got, _oracle_orders(scores, gumbel, cu, k, k_cap))
+
+
+def test_pl_sample_ties_nan_signed_zero_and_counts():
+    lens = [9, 1, 0, 12, 6, 40]
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    rng = np.random.default_rng(9)
+    scores = rng.integers(-2, 3, t).astype(np.float32)   # many exact ties
+    gumbel = np.zeros(t, dtype=np.float32)
+    scores[cu[0] + 3] = np.nan
+    scores[cu[3] + 2], scores[cu[3] + 5] = -0.0, 0.0
+    gumbel[cu[5] + 1:cu[5] + 20] = rng.integers(-1, 2, 19).astype(np.float32) * 0.5
+    k = np.array([8, 0, 0, 11, 3, 39])
+    got, st = _run_sample(scores, gumbel, cu, k, 40)
+    assert st == 0
+    assert np.array_equal(got, _oracle_orders(scores, gumbel, cu, k, 40))
+    # k above the visual count, and above k_cap: clamped and flagged
+    got, st = _run_sample(scores, gumbel, cu, np.array([9, 1, 0, 11, 3, 39]), 39)
+    assert st == O.DORA_ERR_DEVICE_BAD_COUNT
+    assert np.array_equal(got[0, :8], _oracle_orders(scores, gumbel, cu, [8] + [0] * 5, 39)[0, :8])
+
+
+def _check_logprob(scores, cu, orders, k, dlogp, grad_rtol=2e-4):
+    b = len(cu) - 1
+    k_cap = orders.shape[1]
+    logp = torch.full((b,), 5.0, dtype=torch.float32, device=dev())
+    grad = torch.full((int(cu[-1]),), 5.0, dtype=torch.float32, device=dev())
+    st = _status()
+    P.dora_pl_logprob(f32(scores), i32(cu), i32(k), i32(orders), logp, grad=grad,
+                      dlogp=f32(dlogp), status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    lp, g = logp.cpu().numpy().astype(np.float64), grad.cpu().numpy().astype(np.float64)
+    for i in range(b):
+        lo, hi = int(cu[i]), int(cu[i + 1])
+        if hi - lo < 1:
+            continue
+        s = scores[lo + 1:hi].astype(np.float64)
+        seq = orders[i, :k[i]]
+        ref = O.pl_logprob(s, seq)
+        # fp32 bound: every term s_{i_t} - L_t carries ~1e-6 of its magnitude
+        scale = sum(abs(s[j]) + abs(scipy.special.logsumexp(np.delete(s, seq[:t])))
+                    for t, j in enumerate(seq)) if len(seq) else 0.0
+        assert abs(lp[i] - ref) <= 1e-5 * scale + 1e-6, (i, lp[i], ref)
+        gref = dlogp[i] * O.pl_logprob_grad(s, seq)
+        assert g[lo] == 0.0
+        err = np.abs(g[lo + 1:hi] - gref)
+        assert np.all(err <= grad_rtol * (1 + np.abs(gref))), (i, err.max())
+
+
+@pytest.mark.parametrize("scale", [1.0, 30.0])
+def test_pl_logprob_and_gradient_match_oracle(scale):
+    cu = _pruned_layout("cfg3", 4, 0)[:65]               # 64 images after the first deletion
+    t = int(cu[-1])
+    rng = np.random.default_rng(int(scale))
+    scores = (rng.standard_normal(t) * scale).astype(np.float32)
+    n = np.diff(cu) - 1
+    k = np.array([rng.integers(0, m + 1) for m in n])
+    k[1], k[2] = 0, n[2]
+    k_cap = int(n.max())
+    orders, st = _run_sample(scores, _gumbel(rng, t), cu, k, k_cap)
+    assert st == 0
+    _check_logprob(scores, cu, orders, k, rng.uniform(-2, 2, len(k)))
+
+
+def test_pl_logprob_bad_sequences_give_nan_and_status():
+    cu = O.cu_from_counts([6, 6])
+    scores = np.arange(12, dtype=np.float32)
+    orders = np.array([[0, 0, -1], [1, 7, -1]], dtype=np.int32)   # repeat; out of range
+    logp = torch.zeros(2, dtype=torch.float32, device=dev())
+    st = _status()
+    P.dora_pl_logprob(f32(scores), i32(cu), i32([2, 2]), i32(orders), logp, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == O.DORA_ERR_DEVICE_BAD_COUNT
+    assert torch.isnan(logp).all()
+
+
+def test_kd_cost_matches_oracle():
+    rng = np.random.default_rng(11)
+    b, shadows, classes, ld = 16, 40, 1000, 1024
+    zn = np.zeros((b, ld), np.float32)
+    zn[:, :classes] = rng.standard_normal((b, classes)) * 3
+    z = np.zeros((shadows, ld), np.float32)
+    img = rng.integers(0, b, shadows)
+    z[:, :classes] = zn[img, :classes] + rng.standard_normal((shadows, classes)) * \
+        rng.uniform(0, 2, (shadows, 1))
+    z[:, classes:] = 50.0                                # padding must be ignored
+    zn_b, z_b = S.f32_to_bf16_bits(zn), S.f32_to_bf16_bits(z)
+    cost = torch.zeros(shadows, dtype=torch.float32, device=dev())
+    st = _status()
+    P.dora_kd_cost(bf(zn_b), bf(z_b), cost, classes, shadow_image=i32(img), tau=3.0, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    got = cost.cpu().numpy().astype(np.float64)
+    zn64, z64 = O.bf16_to_f64(zn_b), O.bf16_to_f64(z_b)
+    for s in range(shadows):
+        ref = O.kd_cost(zn64[img[s], :classes], z64[s, :classes], 3.0)
+        assert abs(got[s] - ref) <= 1e-4 * (1 + ref), (s, got[s], ref)
+
+
+def test_branch_copies_rows_ids_and_moments_bit_exact():
+    rng = np.random.default_rng(12)
+    lens = [5, 0, 9, 3]
+    cu = O.cu_from_counts(lens)
+    t, d, t_cap = int(cu[-1]), 192, 64
+    x = S.f32_to_bf16_bits(rng.standard_normal((t_cap, d)))
+    ids = rng.integers(0, 1000, t_cap).astype(np.int32)
+    mv = rng.standard_normal((t_cap, 2)).astype(np.float32)
+    src = np.array([2, 1, 0, 2], dtype=np.int32)
+    xt, it, mt = bf(x), i32(ids), f32(mv)
+    cu_out = torch.full((len(lens) + 1 + len(src),), -5, dtype=torch.int32, device=dev())
+    lens_out = torch.zeros(len(src), dtype=torch.int32, device=dev())
+    st = _status()
+    P.dora_branch(xt, i32(cu), i32(src), cu_out, ids=it, x_moments=mt, len_out=lens_out, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    want_lens = [lens[s] for s in src]
+    want_cu = np.concatenate([cu, cu[-1] + np.cumsum(want_lens)])
+    assert np.array_equal(cu_out.cpu().numpy(), want_cu)
+    assert lens_out.cpu().numpy().tolist() == want_lens
+    rows = np.concatenate([np.arange(cu[s], cu[s + 1]) for s in src]).astype(np.int64)
+    end = t + len(rows)
+    xb = bits(xt)
+    assert np.array_equal(xb[:t], x[:t]) and np.array_equal(xb[end:], x[end:])
+    assert np.array_equal(xb[t:end], x[rows])
+    assert np.array_equal(it.cpu().numpy()[t:end], ids[rows])
+    assert np.array_equal(mt.cpu().numpy()[t:end], mv[rows])
+    # no room: the overflowing sequence gets length 0 and the status says so
+    cu_small = torch.zeros(len(lens) + 2, dtype=torch.int32, device=dev())
+    st = _status()
+    P.dora_branch(bf(x[:t + 4]), i32(cu), i32([2]), cu_small, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == O.DORA_ERR_DEVICE_SEQLEN
+    assert cu_small.cpu().numpy()[-1] == t
+
+
+def _shadow_case(batch=4, depth=4, prune=(0, 2, 3), seed=13):
+    cfg = S.get_config("cfg1", batch=batch, depth=depth, prune_blocks=prune)
+    cu, ids = S.initial_layout(cfg)
+    x = S.activations_bf16(cfg, seed)
+    wbs = [S.block_weights(cfg, l, seed, random_affine=True) for l in range(depth)]
+    keeps, _ = S.keep_schedule(cfg, seed)
+    tables = [S.score_table(cfg, l, seed) for l in prune]
+    return cfg, cu, ids, x, wbs, keeps, tables
+
+
+def _run_shadows(cfg, cu, ids, x, wbs, keeps, tables):
+    blocks = [P.BlockWeights({k: bf(v) for k, v in w.items()}, cfg.dim, cfg.heads, cfg.mlp_dim,
+                             cfg.ln_eps) for w in wbs]
+    sr = ShadowRollout(blocks, cfg.batch, cfg.n_tokens, cfg.prune_blocks, dev())
+    xo, cuo, ido = sr.forward(bf(x), i32(cu), i32(ids), [f32(t) for t in tables],
+                              [i32(k) for k in keeps])
+    torch.cuda.synchronize()
+    assert int(sr.status.item()) == 0
+    assert P.dora_read_status(P.dora_workspace_status(sr.ws)) == 0
+    return sr, xo, cuo.cpu().numpy(), ido.cpu().numpy()
+
+
+def test_shadow_rollout_matches_oracle_prefixes():
+    """Rollout, Native and the shadows of prefixes 0 and 2 in one packed
+    batch: the integer trajectory of every sequence (boundaries, ids) bit for
+    bit against the oracle's forward of each prefix run on its own."""
+    cfg, cu, ids, x, wbs, keeps, tables = _shadow_case()
+    sr, xo, cuo, ido = _run_shadows(cfg, cu, ids, x, wbs, keeps, tables)
+    b = cfg.batch
+    prune = {l: (tables[j], keeps[j]) for j, l in enumerate(cfg.prune_blocks)}
+    ref = O.shadow_forwards(O.bf16_to_f64(x), cu, ids, [O.decode_weights(w) for w in wbs],
+                            cfg.heads, cfg.ln_eps, prune)
+    groups = [("rollout", cfg.prune_blocks[-1]), ("native", -1)] + \
+        [(l, l) for l in cfg.prune_blocks[:-1]]
+    assert len(cuo) == b * len(groups) + 1
+    for name, key in groups:
+        g0 = sr.groups[name]
+        r = ref[key]
+        lens = np.diff(cuo)[g0:g0 + b]
+        assert np.array_equal(lens, np.diff(r["cu"])), name
+        rows = np.concatenate([np.arange(cuo[g0 + i], cuo[g0 + i + 1]) for i in range(b)])
+        assert np.array_equal(ido[rows], r["ids"]), name
+
+
+def test_shadow_rollout_blocks_match_oracle():
+    """Each block of the batched forward (rollout pruned, Native and shadows
+    kept whole, branches after the pruning blocks) against the oracle block
+    fed the same bf16 input: rows within the block tolerance, boundaries,
+    ids and branched copies bit for bit."""
+    cfg, cu, ids, x, wbs, keeps, tables = _shadow_case()
+    blocks = [P.BlockWeights({k: bf(v) for k, v in w.items()}, cfg.dim, cfg.heads, cfg.mlp_dim,
+                             cfg.ln_eps) for w in wbs]
+    sr = ShadowRollout(blocks, cfg.batch, cfg.n_tokens, cfg.prune_blocks, dev())
+    b = cfg.batch
+
+    def state(stop):
+        xs, cs, i_s = sr.forward(bf(x), i32(cu), i32(ids), [f32(t) for t in tables],
+                                 [i32(k) for k in keeps], stop=stop)
+        torch.cuda.synchronize()
+        cs = cs.cpu().numpy()
+        t = int(cs[-1])
+        return bits(xs)[:t], cs, i_s.cpu().numpy()[:t]
+
+    x_in, cu_in, ids_in = state(0)
+    assert np.array_equal(cu_in, np.concatenate([cu, cu[-1] + cu[1:]]))   # Native copies
+    for l in range(cfg.depth):
+        x_out, cu_out, ids_out = state(l + 1)
+        wf = O.decode_weights(wbs[l])
+        if l in cfg.prune_blocks:
+            j = cfg.prune_blocks.index(l)
+            scores = np.zeros(len(ids_in))
+            scores[:cu_in[b]] = O.gather_scores(tables[j], cu_in[:b + 1], ids_in[:cu_in[b]])
+            kc = np.concatenate([keeps[j], np.diff(cu_in)[b:]])
+            r = O.pruned_block(O.bf16_to_f64(x_in), cu_in, ids_in, wf, cfg.heads, cfg.ln_eps,
+                               scores, kc)
+            rx, rcu, rids = r["x_out"], r["cu_out"], r["ids_out"]
+            if l in cfg.prune_blocks[:-1]:               # the rollout's images branch off
+                rows = np.arange(rcu[0], rcu[b])
+                rx = np.concatenate([rx, rx[rows]])
+                rids = np.concatenate([rids, rids[rows]])
+                rcu = np.concatenate([rcu, rcu[-1] + rcu[1:b + 1]])
+        else:
+            r = O.pruned_block(O.bf16_to_f64(x_in), cu_in, ids_in, wf, cfg.heads, cfg.ln_eps)
+            rx, rcu, rids = r["x_out"], cu_in, ids_in
+        assert np.array_equal(cu_out, rcu), l
+        assert np.array_equal(ids_out, rids), l
+        assert_close(O.bf16_to_f64(x_out), rx, f"batched shadow forward, block {l}")
+        if l in cfg.prune_blocks[:-1]:                   # branched rows are exact copies
+            t0 = int(rcu[-b - 1])
+            assert np.array_equal(x_out[t0:], x_out[rcu[0]:rcu[b]])
+        x_in, cu_in, ids_in = x_out, cu_out, ids_out
+
+
+def test_shadow_equals_the_prefix_run_alone_bit_for_bit():
+    """A shadow riding in the big batch has the bits of the same prefix run as
+    a rollout on its own (rows never interact across sequences)."""
+    cfg, cu, ids, x, wbs, keeps, tables = _shadow_case()
+    sr, xo, cuo, _ = _run_shadows(cfg, cu, ids, x, wbs, keeps, tables)
+    b = cfg.batch
+    g0 = sr.groups[0]
+    shadow_rows = bits(xo)[cuo[g0]:cuo[g0 + b]]
+    alone = S.get_config("cfg1", batch=b, depth=cfg.depth, prune_blocks=(0,))
+    _, xa, cua, _ = _run_shadows(alone, cu, ids, x, wbs, keeps[:1], tables[:1])
+    assert np.array_equal(bits(xa)[cua[0]:cua[b]], shadow_rows)
+
+
+def test_shadow_costs_match_oracle_on_the_logits():
+    cfg, cu, ids, x, wbs, keeps, tables = _shadow_case()
+    sr, xo, cuo, _ = _run_shadows(cfg, cu, ids, x, wbs, keeps, tables)
+    wh = S.embed_head_weights(cfg, 13)
+    w_head = np.zeros((1024, cfg.dim), np.uint16)
+    w_head[:1000] = wh["w_head"]
+    b_head = np.zeros(1024, np.uint16)
+    b_head[:1000] = wh["b_head"]
+    logits, cost = sr.head_and_costs(xo, i32(cuo), bf(wh["norm_w"]), bf(wh["norm_b"]), 1e-6,
+                                     bf(w_head), bf(b_head))
+    torch.cuda.synchronize()
+    assert int(sr.status.item()) == 0
+    lg = f64(logits)
+    c = cost.cpu().numpy().astype(np.float64)
+    b = cfg.batch
+    ref_logits = O.classifier_head(f64(xo), cuo, O.bf16_to_f64(wh["norm_w"]),
+                                   O.bf16_to_f64(wh["norm_b"]), 1e-6, O.bf16_to_f64(w_head),
+                                   O.bf16_to_f64(b_head))
+    assert_close(lg, ref_logits, "shadow logits")
+    for s in range(len(c)):
+        ref = O.kd_cost(lg[b + s % b, :1000], lg[s, :1000], 3.0)
+        assert abs(c[s] - ref) <= 1e-4 * (1 + ref), (s, c[s], ref)
+    assert np.all(c[b:2 * b] == 0.0)                     # Native against itself
+    assert np.all(c[:b] > 0) and np.all(c[2 * b:] > 0)
