@@ -594,15 +594,18 @@ int dora_fold_layerscale(const dora_bf16* w, const dora_bf16* b, const dora_bf16
  * dora_pl_sample -- the ordered removal sequence (i_1..i_k) of each image,
  * drawn without replacement from the Plackett-Luce distribution of its scores
  * as the Gumbel-top-k: the k_i largest keys s_j + g_j (fp32 sum; -0 == +0,
- * NaN above +inf, equal keys by lower j) in decreasing order.  gumbel fp32
- * [t_cap] row-aligned standard Gumbel noise, drawn by the caller; k int32
- * [batch] (device); order int32 [batch, k_cap] out: order[i, t] = j of the
- * (t+1)-th removal, -1 for t >= k_i.  k_i outside [0, min(n_i, k_cap)] is
- * clamped and raises DORA_ERR_DEVICE_BAD_COUNT.
+ * NaN above +inf, equal keys by higher j first) in decreasing order.  The
+ * tie rule is dora_select_keep's, so the sampled set is exactly what the
+ * block deletes when it is given the keys as its scores: keys_out fp32
+ * [t_cap] (nullable) receives s + g on every visual row (the CLS row: s).
+ * gumbel fp32 [t_cap] row-aligned standard Gumbel noise, drawn by the
+ * caller; k int32 [batch] (device); order int32 [batch, k_cap] out:
+ * order[i, t] = j of the (t+1)-th removal, -1 for t >= k_i.  k_i outside
+ * [0, min(n_i, k_cap)] is clamped and raises DORA_ERR_DEVICE_BAD_COUNT.
  */
 int dora_pl_sample(const float* scores, const float* gumbel, const int32_t* cu, int32_t batch,
                    int32_t t_cap, const int32_t* k, int32_t k_cap, int32_t* order,
-                   int32_t* status, dora_stream_t stream);
+                   float* keys_out, int32_t* status, dora_stream_t stream);
 
 /*
  * dora_pl_logprob -- logp fp32 [batch]: log pi_S(i | k) = sum_t [s_{i_t} -

@@ -553,11 +553,13 @@ def pl_sample_gumbel(scores: np.ndarray, gumbel: np.ndarray, k: int) -> np.ndarr
     Gumbel-top-k of the scores: the k largest keys s_j + g_j in decreasing
     order, g_j standard Gumbel noise supplied by the caller.  The keys are
     formed in fp32 (the precision the decision is taken in on both sides);
-    ties go to the lower index, -0 equals +0 and NaN ranks above +inf."""
+    -0 equals +0, NaN ranks above +inf, and equal keys go to the higher index
+    first -- the tie rule of select_keep, so the first k entries are exactly
+    the tokens that deterministic selection on the keys s + g deletes."""
     s = np.asarray(scores, dtype=np.float32)
     g = np.asarray(gumbel, dtype=np.float32)
     keys = score_order_key((s + g).astype(np.float32))
-    order = sorted(range(len(s)), key=lambda j: (-int(keys[j]), j))
+    order = sorted(range(len(s)), key=lambda j: (-int(keys[j]), -j))
     return np.array(order[:k], dtype=np.int64)
 
 

@@ -80,7 +80,7 @@ _SIGS = {
     "dora_classifier_head_lc1": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _f32, _vp,
                                                 _vp, _i32, _vp, _vp, _sz, _vp]),
     "dora_fold_layerscale": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp]),
-    "dora_pl_sample": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _i32, _vp, _vp, _vp]),
+    "dora_pl_sample": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _i32, _vp, _vp, _vp, _vp]),
     "dora_pl_logprob": (ctypes.c_int, [_vp, _vp, _i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp,
                                        _vp]),
     "dora_branch": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _vp, _i32, _vp, _vp, _vp,
@@ -726,19 +726,21 @@ def dora_classifier_head(x, cu, norm_w, norm_b, eps, w_head, b_head, logits, wor
 # fidelity cost
 # ---------------------------------------------------------------------------
 
-def dora_pl_sample(scores, gumbel, cu, k, order, status=None, stream=None):
-    """Gumbel-top-k removal sequences: order int32 [B, k_cap] (-1 past k_i)."""
+def dora_pl_sample(scores, gumbel, cu, k, order, keys_out=None, status=None, stream=None):
+    """Gumbel-top-k removal sequences: order int32 [B, k_cap] (-1 past k_i);
+    keys_out (fp32, row-aligned) receives the perturbed keys s + g."""
     _req(scores, torch.float32, "scores")
     _req(gumbel, torch.float32, "gumbel")
     _req(cu, torch.int32, "cu")
     _req(k, torch.int32, "k")
     _req(order, torch.int32, "order")
+    _req(keys_out, torch.float32, "keys_out", optional=True)
     b = cu.numel() - 1
     if order.dim() != 2 or order.shape[0] != b or k.numel() != b:
         raise ValueError("order must be [B, k_cap] and k [B]")
     _check(load_library().dora_pl_sample(_ptr(scores), _ptr(gumbel), _ptr(cu), b, scores.numel(),
-                                         _ptr(k), order.shape[1], _ptr(order), _ptr(status),
-                                         _stream(stream)), "dora_pl_sample")
+                                         _ptr(k), order.shape[1], _ptr(order), _ptr(keys_out),
+                                         _ptr(status), _stream(stream)), "dora_pl_sample")
     return order
 
 

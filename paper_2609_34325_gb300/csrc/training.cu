@@ -36,13 +36,16 @@ __device__ __forceinline__ uint32_t order_key(float v) {
 
 // ---------------------------------------------------------------------------
 // Gumbel-top-k: one CTA per image.  Visual token j's rank is the number of
-// tokens whose key s + g (fp32) is larger, or equal with a lower index; ranks
-// below k_i give order[i, rank] = j.  Entries k_i..k_cap-1 are -1.
+// tokens whose key s + g (fp32) is larger, or equal with a higher index (the
+// deployment selection's tie rule, so the first k_i are what it deletes given
+// the keys); ranks below k_i give order[i, rank] = j, entries k_i..k_cap-1
+// are -1, and the keys go to keys_out (row-aligned, nullable).
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads)
     pl_sample_kernel(const float* __restrict__ scores, const float* __restrict__ gumbel,
                      const int32_t* __restrict__ cu, int t_cap, const int32_t* __restrict__ kreq,
-                     int k_cap, int32_t* __restrict__ order, int32_t* status) {
+                     int k_cap, int32_t* __restrict__ order, float* __restrict__ keys_out,
+                     int32_t* status) {
   __shared__ uint32_t keys[kMaxVisual];
   const int img = blockIdx.x;
   const int lo = cu[img], hi = cu[img + 1];
@@ -59,15 +62,20 @@ __global__ void __launch_bounds__(kThreads)
     k = k < 0 ? 0 : (k > n ? n : k);
     k = k > k_cap ? k_cap : k;
   }
-  for (int j = threadIdx.x; j < n; j += blockDim.x)
-    keys[j] = order_key(scores[lo + 1 + j] + gumbel[lo + 1 + j]);
+  for (int j = threadIdx.x; j < n; j += blockDim.x) {
+    const float key = scores[lo + 1 + j] + gumbel[lo + 1 + j];
+    keys[j] = order_key(key);
+    if (keys_out != nullptr) keys_out[lo + 1 + j] = key;
+  }
+  if (keys_out != nullptr && threadIdx.x == 0 && hi > lo && lo >= 0 && lo < t_cap)
+    keys_out[lo] = scores[lo];
   __syncthreads();
   for (int j = threadIdx.x; j < n; j += blockDim.x) {
     const uint32_t kj = keys[j];
     int rank = 0;
     for (int u = 0; u < n; ++u) {
       const uint32_t ku = keys[u];
-      rank += (ku > kj) | ((ku == kj) & (u < j));
+      rank += (ku > kj) | ((ku == kj) & (u > j));
     }
     if (rank < k) out[rank] = j;
   }
@@ -340,7 +348,7 @@ extern "C" {
 
 int dora_pl_sample(const float* scores, const float* gumbel, const int32_t* cu, int32_t batch,
                    int32_t t_cap, const int32_t* k, int32_t k_cap, int32_t* order,
-                   int32_t* status, dora_stream_t stream) {
+                   float* keys_out, int32_t* status, dora_stream_t stream) {
   if (batch < 0 || batch > (1 << 24) || t_cap < 0 || k_cap < 1 || k_cap > train::kMaxVisual)
     return DORA_ERR_INVALID_ARG;
   if (scores == nullptr || gumbel == nullptr || cu == nullptr || k == nullptr || order == nullptr)
@@ -349,7 +357,7 @@ int dora_pl_sample(const float* scores, const float* gumbel, const int32_t* cu, 
   if (e != DORA_OK) return e;
   if (batch == 0) return DORA_OK;
   train::pl_sample_kernel<<<batch, train::kThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      scores, gumbel, cu, t_cap, k, k_cap, order, status);
+      scores, gumbel, cu, t_cap, k, k_cap, order, keys_out, status);
   return cudaGetLastError() == cudaSuccess ? DORA_OK : DORA_ERR_CUDA;
 }
 

@@ -22,8 +22,9 @@ import contextlib
 
 import torch
 
-from . import (alloc_workspace, dora_branch, dora_classifier_head,
-               dora_classifier_head_lc1, dora_gather_scores, dora_kd_cost, dora_pruned_block)
+from . import (alloc_workspace, dora_branch, dora_classifier_head, dora_classifier_head_lc1,
+               dora_gather_scores, dora_kd_cost, dora_pl_logprob, dora_pl_sample,
+               dora_pruned_block)
 
 
 class ShadowRollout:
@@ -60,6 +61,20 @@ class ShadowRollout:
         # every sequence compares with its image's Native logits
         self.image_of = torch.arange(self.nseq, dtype=torch.int32, device=dev) % batch
         self.head_ws = None
+        # training rollouts (App. A.3): per pruning block the selector scores,
+        # the rollout's boundaries, the sampled removal order and its
+        # log-probability
+        npb = len(self.prune)
+        self.k_cap = n_tokens - 1
+        self.keys = torch.zeros(t, dtype=torch.float32, device=dev)
+        self.gum = torch.zeros(batch * n_tokens, dtype=torch.float32, device=dev)
+        self.s_hist = [torch.zeros(batch * n_tokens, dtype=torch.float32, device=dev)
+                       for _ in range(npb)]
+        self.cu_hist = [torch.zeros(batch + 1, dtype=torch.int32, device=dev) for _ in range(npb)]
+        self.order = torch.full((npb, batch, self.k_cap), -1, dtype=torch.int32, device=dev)
+        self.logp = torch.zeros(npb, batch, dtype=torch.float32, device=dev)
+        self.grad = [torch.zeros(batch * n_tokens, dtype=torch.float32, device=dev)
+                     for _ in range(npb)]
         # sequence layout after the forward: rollout, Native, then one group
         # of `batch` shadows per branching block
         self.groups = {"rollout": 0, "native": batch}
@@ -77,19 +92,25 @@ class ShadowRollout:
                     n += 2
         return n
 
-    def forward(self, x0, cu0, ids0, tables, keeps, stream=None, stop=None):
+    def forward(self, x0, cu0, ids0, tables, keeps, stream=None, stop=None, gumbel=None,
+                removals=None):
         """Rollout + Native + shadows through every block.  x0 bf16 [B N, d],
         cu0 int32 [B + 1], ids0 int32 [B N]; tables[j] fp32 [B, stride]
         deletion-score tables keyed by original token id and keeps[j] int32
-        [B] keep counts for pruning block j.  Returns (x, cu, ids) of the whole
+        [B] keep counts for pruning block j.  A training rollout also passes
+        gumbel[j] (fp32 [B, stride] standard Gumbel noise keyed, like the
+        scores, by original token id) and removals[j] (int32 [B], k = rows -
+        keep counts): the removal order
+        is then sampled (dora_pl_sample) and the block deletes the sampled set
+        by taking the perturbed keys as its scores.  Returns (x, cu, ids) of the whole
         packed batch (sequence order: rollout, Native, shadow groups).  With
         ``stop`` the batch is returned after the first ``stop`` blocks (and
         their branches)."""
         with torch.cuda.stream(stream) if stream is not None else contextlib.nullcontext():
             return self._forward(x0, cu0, ids0, tables, keeps, stream,
-                                 self.depth if stop is None else stop)
+                                 self.depth if stop is None else stop, gumbel, removals)
 
-    def _forward(self, x0, cu0, ids0, tables, keeps, stream, stop):
+    def _forward(self, x0, cu0, ids0, tables, keeps, stream, stop, gumbel, removals):
         b = self.b
         rows = x0.shape[0]
         x, mv, ids = self.x[0], None, self.ids[0]
@@ -107,11 +128,23 @@ class ShadowRollout:
             if l in self.prune:
                 j = self.prune.index(l)
                 self.keep[:b].copy_(keeps[j])
-                dora_gather_scores(tables[j], ids, cu[:b + 1], self.scores, status=self.status,
-                                   stream=stream)
+                sc = self.scores
+                if gumbel is not None:
+                    sj = self.s_hist[j]
+                    dora_gather_scores(tables[j], ids, cu[:b + 1], sj, status=self.status,
+                                       stream=stream)
+                    dora_gather_scores(gumbel[j], ids, cu[:b + 1], self.gum, status=self.status,
+                                       stream=stream)
+                    self.cu_hist[j].copy_(cu[:b + 1])
+                    dora_pl_sample(sj, self.gum, self.cu_hist[j], removals[j], self.order[j],
+                                   keys_out=self.keys, status=self.status, stream=stream)
+                    sc = self.keys
+                else:
+                    dora_gather_scores(tables[j], ids, cu[:b + 1], sc, status=self.status,
+                                       stream=stream)
                 cu_out, idn = self.cu[1 - q], self.ids[1 - q]
                 dora_pruned_block(x, cu[:nseq + 1], w, self.n_tokens, out, self.ws, ids_in=ids,
-                                  scores=self.scores, keep_counts=self.keep[:nseq],
+                                  scores=sc, keep_counts=self.keep[:nseq],
                                   cu_out=cu_out[:nseq + 1], ids_out=idn, kept_idx=self.kept,
                                   x_in_moments=mv, x_out_moments=mv_out, stream=stream)
                 if l in self.branch_at:
@@ -126,6 +159,16 @@ class ShadowRollout:
             x, mv, p = out, mv_out, 1 - p
         self.nseq_out = nseq
         return x, cu[:nseq + 1], ids
+
+    def logprob(self, removals, dlogp=None, stream=None):
+        """Plackett-Luce log-probabilities [pruning blocks, B] of the sampled
+        removal orders of the last training forward, and their gradients with
+        respect to the selector scores (times dlogp [B], e.g. advantages)."""
+        for j in range(len(self.prune)):
+            dora_pl_logprob(self.s_hist[j], self.cu_hist[j], removals[j], self.order[j],
+                            self.logp[j], grad=self.grad[j], dlogp=dlogp, status=self.status,
+                            stream=stream)
+        return self.logp, self.grad
 
     def head_and_costs(self, x, cu, norm_w, norm_b, eps, w_head, b_head, lc1=False, tau=3.0,
                        stream=None):

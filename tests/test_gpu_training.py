@@ -344,3 +344,52 @@ def test_shadow_costs_match_oracle_on_the_logits():
         assert abs(c[s] - ref) <= 1e-4 * (1 + ref), (s, c[s], ref)
     assert np.all(c[b:2 * b] == 0.0)                     # Native against itself
     assert np.all(c[:b] > 0) and np.all(c[2 * b:] > 0)
+
+
+def test_training_rollout_deletes_its_sampled_sets():
+    """Training mode: at each pruning block the removal order is sampled
+    (Gumbel-top-k of the gathered scores) and the block deletes exactly the
+    sampled set -- the rollout's trajectory equals the oracle forward whose
+    score tables are the fp32 keys s + g; the orders' log-probabilities and
+    gradients match the oracle's on the same scores."""
+    cfg, cu, ids, x, wbs, keeps, tables = _shadow_case(seed=17)
+    rng = np.random.default_rng(17)
+    gtabs = [_gumbel(rng, t.size).reshape(t.shape) for t in tables]
+    _, befores = S.keep_schedule(cfg, 17)
+    removals = [np.asarray(bf_) - np.asarray(k) for bf_, k in zip(befores, keeps)]
+    blocks = [P.BlockWeights({k: bf(v) for k, v in w.items()}, cfg.dim, cfg.heads, cfg.mlp_dim,
+                             cfg.ln_eps) for w in wbs]
+    sr = ShadowRollout(blocks, cfg.batch, cfg.n_tokens, cfg.prune_blocks, dev())
+    xo, cuo, ido = sr.forward(bf(x), i32(cu), i32(ids), [f32(t) for t in tables],
+                              [i32(k) for k in keeps], gumbel=[f32(g) for g in gtabs],
+                              removals=[i32(r) for r in removals])
+    adv = rng.uniform(-1, 1, cfg.batch)
+    logp, grads = sr.logprob([i32(r) for r in removals], dlogp=f32(adv))
+    torch.cuda.synchronize()
+    assert int(sr.status.item()) == 0
+    b = cfg.batch
+    keyed = {l: ((tables[j] + gtabs[j]).astype(np.float32), keeps[j])
+             for j, l in enumerate(cfg.prune_blocks)}
+    ref = O.forward(O.bf16_to_f64(x), cu, ids, [O.decode_weights(w) for w in wbs], cfg.heads,
+                    cfg.ln_eps, keyed)
+    cuo = cuo.cpu().numpy()
+    assert np.array_equal(np.diff(cuo)[:b], np.diff(ref["cu"]))
+    assert np.array_equal(ido.cpu().numpy()[:cuo[b]], ref["ids"])
+    orders = sr.order.cpu().numpy()
+    lp = logp.cpu().numpy()
+    for j, l in enumerate(cfg.prune_blocks):
+        cuj = sr.cu_hist[j].cpu().numpy()
+        sj = sr.s_hist[j].cpu().numpy()
+        gj = grads[j].cpu().numpy()
+        kept = ref["kept"][l]
+        for i in range(b):
+            lo, hi = int(cuj[i]), int(cuj[i + 1])
+            k = int(removals[j][i])
+            seq = orders[j, i, :k]
+            kept_local = set((kept[(kept > lo) & (kept < hi)] - lo - 1).tolist())
+            assert set(seq.tolist()) == set(range(hi - lo - 1)) - kept_local, (l, i)
+            s = sj[lo + 1:hi].astype(np.float64)
+            r = O.pl_logprob(s, seq)
+            assert abs(lp[j, i] - r) <= 1e-5 * (abs(r) + k * (1 + np.abs(s).max())), (l, i)
+            gref = adv[i] * O.pl_logprob_grad(s, seq)
+            assert np.all(np.abs(gj[lo + 1:hi] - gref) <= 2e-4 * (1 + np.abs(gref)))

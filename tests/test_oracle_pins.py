@@ -753,13 +753,30 @@ def test_gumbel_top_k_is_a_plackett_luce_sample():
 def test_gumbel_top_k_order_rules():
     s = np.array([0.5, 2.0, -1.0, 2.0, 0.0, -0.0, np.nan], dtype=np.float32)
     z = np.zeros(7, dtype=np.float32)
-    # NaN first, equal keys by lower index, -0 == +0
-    assert O.pl_sample_gumbel(s, z, 7).tolist() == [6, 1, 3, 0, 4, 5, 2]
-    assert O.pl_sample_gumbel(s[:6], z[:6], 2).tolist() == [1, 3]
+    # NaN first, equal keys by higher index (as deployment deletes), -0 == +0
+    assert O.pl_sample_gumbel(s, z, 7).tolist() == [6, 3, 1, 0, 5, 4, 2]
+    assert O.pl_sample_gumbel(s[:6], z[:6], 2).tolist() == [3, 1]
     # keys are fp32 sums: 1 + 2^-24 rounds to 1, so index order decides
     a = np.array([1.0, 1.0], dtype=np.float32)
-    g = np.array([2.0 ** -24, 0.0], dtype=np.float32)
-    assert O.pl_sample_gumbel(a, g[::-1].copy(), 2).tolist() == [0, 1]
+    g = np.array([0.0, 2.0 ** -24], dtype=np.float32)
+    assert O.pl_sample_gumbel(a, g, 2).tolist() == [1, 0]
+
+
+def test_sampled_set_is_what_selection_deletes_on_the_keys():
+    """The first k of the Gumbel-top-k order are exactly the tokens that the
+    deterministic selection removes when given the keys s + g (ties
+    included), so a training rollout deletes its sampled set."""
+    rng = np.random.default_rng(8)
+    for trial in range(200):
+        n = int(rng.integers(1, 30))
+        s = rng.integers(-3, 4, n).astype(np.float32)
+        g = (rng.integers(-2, 3, n) * 0.5).astype(np.float32)
+        k = int(rng.integers(0, n + 1))
+        removed = set(O.pl_sample_gumbel(s, g, k).tolist())
+        keys = np.concatenate([[0.0], s + g]).astype(np.float32)   # CLS row first
+        kept, _, st = O.select_keep(keys, np.array([0, n + 1]), np.array([n + 1 - k]))
+        assert st == 0
+        assert removed == set(range(n)) - set((kept[1:] - 1).tolist())
 
 
 def test_kd_cost_pins():
