@@ -496,6 +496,44 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
                     "(actor at the pruning blocks, configured keep counts) -> LayerNorm + "
                     "classifier; dense = the same without deletion or actor"}
 
+        # one training rollout step (App. A.3, App. B.2): the forward with
+        # Plackett-Luce sampled deletions at the pruning blocks, the Native
+        # forward and the complete-prefix shadows of every pruning block but
+        # the last riding in the same packed batch, the classifier on every
+        # sequence, the fidelity costs, and the log-probabilities of the
+        # sampled orders with their gradients
+        from paper_2609_34325_gb300.shadow import ShadowRollout
+        sr = ShadowRollout(blocks, cfg.batch, cfg.n_tokens, cfg.prune_blocks, dev)
+        grng = np.random.default_rng(args.seed + 31)
+        gtabs = [[torch.from_numpy((-np.log(-np.log(grng.random(t.shape)))).astype(np.float32))
+                  .to(dev) for t in s_["tables"]] for s_ in hw.sets]
+        rem = [[torch.from_numpy((np.asarray(b_) - np.asarray(k_)).astype(np.int32)).to(dev)
+                for b_, k_ in zip(s_["befores"], s_["keeps"])] for s_ in hw.sets]
+        adv = torch.from_numpy(grng.uniform(-1, 1, cfg.batch).astype(np.float32)).to(dev)
+        L0 = lanes[0]
+
+        def train_step(i):
+            r = i % nsets
+            xo, cuo, _ = sr.forward(sets[r]["x"], L0["cu0"], L0["ids0"], sets[r]["tables"],
+                                    sets[r]["keeps"], gumbel=gtabs[r], removals=rem[r],
+                                    stream=stream)
+            sr.head_and_costs(xo, cuo, E["norm_w"], E["norm_b"], 1e-6, w_head, b_head, lc1=lc1,
+                              stream=stream)
+            sr.logprob(rem[r], dlogp=adv, stream=stream)
+
+        tsecs, _ = timed(train_step, args.steps, max(args.warmup, 3))
+        sst = int(sr.status.item())
+        bst = P.dora_read_status(P.dora_workspace_status(sr.ws))
+        result["training_step"] = {
+            "value": round(cfg.batch * args.steps * world / tsecs, 1), "unit": UNIT,
+            "ms_per_step": round(1000 * tsecs / args.steps, 4),
+            "sequences": sr.nseq_out, "device_status": max(sst, bst),
+            "what": "rollout with Plackett-Luce sampled deletions (Gumbel-top-k, noise an input) "
+                    f"at {'/'.join(map(str, cfg.prune_blocks))}, Native forward and the "
+                    "complete-prefix shadows branched after each pruning block but the last, "
+                    "all in one packed batch through the same kernels; classifier on every "
+                    "sequence, fidelity costs (tau = 3), log-probabilities and their gradients"}
+
     # context: torch eager dense forward of the same shapes and weights
     # (cuBLAS linears, scaled_dot_product_attention), not this library
     try:
