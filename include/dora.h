@@ -630,7 +630,8 @@ int dora_pl_logprob(const float* scores, const int32_t* cu, int32_t batch, int32
  * n_branch]: cu followed by the appended sequences' ends (cu_out == cu is
  * allowed when it has the room); len_out int32 [n_branch] (nullable): their
  * lengths, which are also their keep counts at every later block.  Rows past
- * t_cap are not written (DORA_ERR_DEVICE_SEQLEN, the sequence gets length 0).
+ * t_cap are not written: the first appended sequence that does not fit, and
+ * every one after it, gets length 0 (DORA_ERR_DEVICE_SEQLEN).
  */
 int dora_branch(dora_bf16* x, int32_t* ids, float* x_moments, const int32_t* cu, int32_t batch,
                 int32_t t_cap, int32_t dim, const int32_t* src, int32_t n_branch,

@@ -94,6 +94,69 @@ __global__ void patchify_any_kernel(const uint16_t* __restrict__ img, int batch,
   }
 }
 
+// Even patch side (DINOv2's 14): one thread writes one 4-byte pixel pair of
+// the K-padded patch matrix, consecutive threads consecutive pairs of a
+// token row, so every store is coalesced; the pair (an even pair never
+// straddles two patches) is read from the image, pad pairs are zero.  All
+// counts fit in 32 bits (checked by the caller).
+__global__ void patchify_even_kernel(const uint32_t* __restrict__ img, int batch, int ch, int h,
+                                     int w, int p, int kpad, uint32_t* __restrict__ out) {
+  const int gw = w / p, gh = h / p, p2 = p / 2, row2 = p * p2, k2 = ch * row2, w2 = w / 2;
+  const int kp2 = kpad / 2;
+  const int total = batch * gh * gw * kp2;
+  for (int s = blockIdx.x * blockDim.x + threadIdx.x; s < total; s += gridDim.x * blockDim.x) {
+    const int q = s % kp2, tok = s / kp2;
+    uint32_t v = 0u;
+    if (q < k2) {
+      const int c = q / row2, rem = q - c * row2, dy = rem / p2, e = rem - dy * p2;
+      const int gx = tok % gw, t2 = tok / gw, gy = t2 % gh, b = t2 / gh;
+      v = __ldg(img + (static_cast<size_t>((b * ch + c) * h + gy * p + dy) * w2 + gx * p2 + e));
+    }
+    out[s] = v;
+  }
+}
+
+// The same relayout with the patch side and channel count fixed at compile
+// time (DINOv2-B/14 on RGB), staged through shared memory: one block per
+// band of patches (image b, patch row gy).  The band's CH x P image rows are
+// read with coalesced 16-byte loads, then its gw token rows are written with
+// coalesced 16-byte stores, each 8-column piece gathered from shared memory
+// (column c P^2 + dy P + dx, zero past CH P^2).  Needs w % 8 == 0.
+template <int P, int CH>
+__global__ void __launch_bounds__(256)
+    patchify_band_kernel(const uint4* __restrict__ img, int gh, int gw, int h, int w,
+                         uint4* __restrict__ out) {
+  extern __shared__ uint16_t band[];                   // [CH][P][w]
+  constexpr int kK = CH * P * P, kKp8 = (kK + 63) / 64 * 8;
+  const int gy = blockIdx.x % gh, b = blockIdx.x / gh;
+  const int w8 = w / 8;
+  uint4* band4 = reinterpret_cast<uint4*>(band);
+  for (int i = threadIdx.x; i < CH * P * w8; i += blockDim.x) {
+    const int x8 = i % w8, r = i / w8, dy = r % P, c = r / P;
+    band4[i] = __ldg(img + (static_cast<size_t>((b * CH + c) * h + gy * P + dy) * w8 + x8));
+  }
+  __syncthreads();
+  uint4* dst = out + static_cast<size_t>(blockIdx.x) * gw * kKp8;
+  for (int i = threadIdx.x; i < gw * kKp8; i += blockDim.x) {
+    const int gx = i / kKp8, c8 = i - gx * kKp8;
+    uint32_t v[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      uint32_t pr = 0u;
+#pragma unroll
+      for (int hlf = 0; hlf < 2; ++hlf) {
+        const int col = c8 * 8 + 2 * e + hlf;
+        if (col < kK) {
+          const int c = col / (P * P), rem = col - c * (P * P), dy = rem / P, dx = rem - dy * P;
+          pr |= static_cast<uint32_t>(band[(c * P + dy) * w + gx * P + dx]) << (16 * hlf);
+        }
+      }
+      v[e] = pr;
+    }
+    dst[i] = make_uint4(v[0], v[1], v[2], v[3]);
+  }
+}
+
 // w [d, k] -> [d, kpad] with zero columns k..kpad-1 (the GEMM's B for K-padded patches).
 __global__ void pad_cols_kernel(const uint16_t* __restrict__ w, int d, int k, int kpad,
                                 uint16_t* __restrict__ out) {
@@ -159,13 +222,15 @@ __global__ void cls_ln_kernel(const uint16_t* __restrict__ x, const int32_t* __r
   }
 }
 
-// LC1 readout of one image per CTA (16 warps): rows lo..hi-1 of x are layer-
+// LC1 readout of one image per CTA (8 warps): rows lo..hi-1 of x are layer-
 // normalised (fp32, biased variance, row held in registers: dim <= 2048); the
-// CLS row goes to u[i, 0:d], the others are summed per warp in shared memory
-// and their mean goes to u[i, d:2d] (zero for an image without visual rows).
-constexpr int kLc1Warps = 16;
+// CLS row goes to u[i, 0:d], the others are summed per lane in registers and
+// their mean goes to u[i, d:2d] (zero for an image without visual rows).
+constexpr int kLc1Warps = 8;
 constexpr int kLc1MaxDim = 2048;
 
+// kChunks = 16-byte pieces of a row per lane (dim <= 256 kChunks).
+template <int kChunks>
 __global__ void __launch_bounds__(kLc1Warps * 32)
     lc1_pool_kernel(const uint16_t* __restrict__ x, const int32_t* __restrict__ cu, int t_cap,
                     int dim, const uint16_t* __restrict__ gam, const uint16_t* __restrict__ bet,
@@ -181,20 +246,37 @@ __global__ void __launch_bounds__(kLc1Warps * 32)
     for (int c = threadIdx.x; c < 2 * dim; c += blockDim.x) ur[c] = 0;
     return;
   }
-  for (int c = lane; c < dim; c += 32) acc[warp * dim + c] = 0.f;
-  __syncwarp();
-  constexpr int kChunks = kLc1MaxDim / 8 / 32;
-  for (int j = lo + warp; j < hi; j += kLc1Warps) {
+  // Each lane owns the columns of its chunks c8 = lane + 32 i in every row,
+  // so the visual rows' normalised values x^ = (x - mean) rstd are summed in
+  // its registers; the affine map is applied once at the end, to the mean
+  // (mean of g x^ + b = g mean(x^) + b).  Each warp walks rows lo + warp,
+  // lo + warp + 8, ...; the next row's loads are issued before the current
+  // row is reduced.
+  float accr[kChunks][8];
+#pragma unroll
+  for (int i = 0; i < kChunks; ++i)
+#pragma unroll
+    for (int e = 0; e < 8; ++e) accr[i][e] = 0.f;
+  uint4 nxt[kChunks];
+  auto load_row = [&](int j, uint4 (&q)[kChunks]) {
     const uint4* xr = reinterpret_cast<const uint4*>(x + static_cast<size_t>(j) * dim);
-    uint4 q[kChunks];
-    float s = 0.f;
 #pragma unroll
     for (int i = 0; i < kChunks; ++i) {
       const int c8 = lane + 32 * i;
-      q[i] = c8 < d8 ? xr[c8] : make_uint4(0, 0, 0, 0);
+      q[i] = (j < hi && c8 < d8) ? xr[c8] : make_uint4(0, 0, 0, 0);
+    }
+  };
+  load_row(lo + warp, nxt);
+  for (int j = lo + warp; j < hi; j += kLc1Warps) {
+    uint4 q[kChunks];
+#pragma unroll
+    for (int i = 0; i < kChunks; ++i) q[i] = nxt[i];
+    load_row(j + kLc1Warps, nxt);
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < kChunks; ++i)
       s += lo_f(q[i].x) + hi_f(q[i].x) + lo_f(q[i].y) + hi_f(q[i].y) + lo_f(q[i].z) +
            hi_f(q[i].z) + lo_f(q[i].w) + hi_f(q[i].w);
-    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
     const float mean = s / dim;
@@ -212,37 +294,51 @@ __global__ void __launch_bounds__(kLc1Warps * 32)
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v2 += __shfl_xor_sync(0xffffffffu, v2, o);
     const float rstd = rsqrtf(v2 / dim + eps);
+    if (j == lo) {                                       // CLS row: LN(x) itself
 #pragma unroll
-    for (int i = 0; i < kChunks; ++i) {
-      const int c8 = lane + 32 * i;
-      if (c8 >= d8) continue;
-      const uint32_t wv[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
-      const uint4 g4 = reinterpret_cast<const uint4*>(gam)[c8];
-      const uint4 b4 = reinterpret_cast<const uint4*>(bet)[c8];
-      const uint32_t gv[4] = {g4.x, g4.y, g4.z, g4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
-      float n[8];
+      for (int i = 0; i < kChunks; ++i) {
+        const int c8 = lane + 32 * i;
+        if (c8 >= d8) continue;
+        const uint32_t wv[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
+        const uint4 g4 = reinterpret_cast<const uint4*>(gam)[c8];
+        const uint4 b4 = reinterpret_cast<const uint4*>(bet)[c8];
+        const uint32_t gv[4] = {g4.x, g4.y, g4.z, g4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
+        uint32_t o[4];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        n[2 * e] = (lo_f(wv[e]) - mean) * rstd * lo_f(gv[e]) + lo_f(bv[e]);
-        n[2 * e + 1] = (hi_f(wv[e]) - mean) * rstd * hi_f(gv[e]) + hi_f(bv[e]);
+        for (int e = 0; e < 4; ++e)
+          o[e] = pack2((lo_f(wv[e]) - mean) * rstd * lo_f(gv[e]) + lo_f(bv[e]),
+                       (hi_f(wv[e]) - mean) * rstd * hi_f(gv[e]) + hi_f(bv[e]));
+        reinterpret_cast<uint4*>(ur)[c8] = make_uint4(o[0], o[1], o[2], o[3]);
       }
-      if (j == lo) {
-        reinterpret_cast<uint4*>(ur)[c8] = make_uint4(pack2(n[0], n[1]), pack2(n[2], n[3]),
-                                                      pack2(n[4], n[5]), pack2(n[6], n[7]));
-      } else {
-        float* a = acc + warp * dim + c8 * 8;
+    } else {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) a[e] += n[e];
+      for (int i = 0; i < kChunks; ++i) {
+        const uint32_t wv[4] = {q[i].x, q[i].y, q[i].z, q[i].w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          accr[i][2 * e] += (lo_f(wv[e]) - mean) * rstd;
+          accr[i][2 * e + 1] += (hi_f(wv[e]) - mean) * rstd;
+        }
       }
     }
   }
+#pragma unroll
+  for (int i = 0; i < kChunks; ++i) {
+    const int c8 = lane + 32 * i;
+    if (c8 >= d8) continue;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[warp * dim + c8 * 8 + e] = accr[i][e];
+  }
   __syncthreads();
-  const float inv = hi - lo > 1 ? 1.f / static_cast<float>(hi - lo - 1) : 0.f;
+  const int n_vis = hi - lo - 1;
+  const float inv = n_vis > 0 ? 1.f / static_cast<float>(n_vis) : 0.f;
   for (int c = threadIdx.x; c < dim; c += blockDim.x) {
     float t = 0.f;
 #pragma unroll
     for (int wp = 0; wp < kLc1Warps; ++wp) t += acc[wp * dim + c];
-    const __nv_bfloat16 hv = __float2bfloat16_rn(t * inv);
+    const float g = __uint_as_float(static_cast<uint32_t>(gam[c]) << 16);
+    const float b = __uint_as_float(static_cast<uint32_t>(bet[c]) << 16);
+    const __nv_bfloat16 hv = __float2bfloat16_rn(n_vis > 0 ? t * inv * g + b : 0.f);
     ur[dim + c] = *reinterpret_cast<const uint16_t*>(&hv);
   }
 }
@@ -332,9 +428,28 @@ int dora_patch_embed(const dora_bf16* images, int32_t batch, int32_t channels, i
     // and a zero-padded copy of the weights in the workspace
     uint16_t* wp = reinterpret_cast<uint16_t*>(ws + 256 + embed::up256(tok * kpad * 2) +
                                                embed::up256(tok * dim * 2));
-    const long long segs = tok * (kpad / 8);
-    embed::patchify_any_kernel<<<embed::grid_for(segs), 256, 0, stream>>>(
-        images, batch, channels, height, width, patch, kpad, reinterpret_cast<uint4*>(patches));
+    const long long items = tok * (kpad / 2);
+    const int band_smem = 3 * 14 * width * 2;
+    if (patch == 14 && channels == 3 && width % 8 == 0 && band_smem <= 160 * 1024 &&
+        static_cast<long long>(batch) * (height / patch) < (1LL << 31)) {
+      auto kern = embed::patchify_band_kernel<14, 3>;
+      if (band_smem > 48 * 1024 &&
+          cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, band_smem) !=
+              cudaSuccess)
+        return DORA_ERR_CUDA;
+      kern<<<static_cast<unsigned>(batch * (height / patch)), 256, band_smem, stream>>>(
+          reinterpret_cast<const uint4*>(images), height / patch, width / patch, height, width,
+          reinterpret_cast<uint4*>(patches));
+    } else if (patch % 2 == 0 && items < (1LL << 31) &&
+               static_cast<long long>(batch) * channels * height * width / 2 < (1LL << 31)) {
+      embed::patchify_even_kernel<<<embed::grid_for(items), 256, 0, stream>>>(
+          reinterpret_cast<const uint32_t*>(images), batch, channels, height, width, patch, kpad,
+          reinterpret_cast<uint32_t*>(patches));
+    } else {
+      const long long segs = tok * (kpad / 8);
+      embed::patchify_any_kernel<<<embed::grid_for(segs), 256, 0, stream>>>(
+          images, batch, channels, height, width, patch, kpad, reinterpret_cast<uint4*>(patches));
+    }
     if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
     if (kpad != k) {
       embed::pad_cols_kernel<<<embed::grid_for(static_cast<long long>(dim) * kpad), 256, 0,
@@ -430,15 +545,18 @@ int dora_classifier_head_lc1(const dora_bf16* x, const int32_t* cu, int32_t batc
   int32_t* status = reinterpret_cast<int32_t*>(ws);
   uint16_t* u = reinterpret_cast<uint16_t*>(ws + 256);
   const int smem = embed::kLc1Warps * dim * 4;
-  static bool attr_set[64] = {false};
-  if (dev < 64 && !attr_set[dev]) {
-    if (cudaFuncSetAttribute(embed::lc1_pool_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             embed::kLc1Warps * embed::kLc1MaxDim * 4) != cudaSuccess)
-      return DORA_ERR_CUDA;
-    attr_set[dev] = true;
-  }
-  embed::lc1_pool_kernel<<<batch, embed::kLc1Warps * 32, smem, stream>>>(
-      x, cu, t_cap, dim, norm_w, norm_b, eps, u, status);
+  const int chunks = (dim / 8 + 31) / 32;
+  auto kern = chunks <= 1   ? embed::lc1_pool_kernel<1>
+              : chunks <= 2 ? embed::lc1_pool_kernel<2>
+              : chunks <= 3 ? embed::lc1_pool_kernel<3>
+              : chunks <= 4 ? embed::lc1_pool_kernel<4>
+                            : embed::lc1_pool_kernel<8>;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+          cudaSuccess)
+    return DORA_ERR_CUDA;
+  kern<<<batch, embed::kLc1Warps * 32, smem, stream>>>(x, cu, t_cap, dim, norm_w, norm_b, eps, u,
+                                                      status);
   if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
   LinearEpi ep;
   ep.bias = b_head;

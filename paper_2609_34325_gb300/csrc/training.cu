@@ -238,27 +238,74 @@ __global__ void __launch_bounds__(kThreads)
 // (in place), with their ids and row moments; cu[batch + 1 + s] and the
 // appended sequences' lengths (len_out) written by the single scan CTA.
 // ---------------------------------------------------------------------------
-__global__ void branch_cu_kernel(const int32_t* __restrict__ cu, int batch,
-                                 const int32_t* __restrict__ src, int nb, int t_cap,
-                                 int32_t* __restrict__ cu_out, int32_t* __restrict__ len_out,
-                                 int32_t* status) {
-  // a serial scan: nb is the number of sequences branched at one block
-  if (threadIdx.x != 0) return;
-  int32_t end = cu[batch];
+constexpr int kScanThreads = 1024;
+
+__global__ void __launch_bounds__(kScanThreads)
+    branch_cu_kernel(const int32_t* __restrict__ cu, int batch, const int32_t* __restrict__ src,
+                     int nb, int t_cap, int32_t* __restrict__ cu_out,
+                     int32_t* __restrict__ len_out, int32_t* status) {
+  // one CTA: the appended lengths in chunks of 1024, a block-wide exclusive
+  // scan per chunk carried across chunks (64-bit sums)
+  __shared__ long long warp_sum[kScanThreads / 32];
+  __shared__ int warp_fit[kScanThreads / 32];
+  __shared__ long long carry;
+  __shared__ int last_fit;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (cu_out != cu)
-    for (int i = 0; i <= batch; ++i) cu_out[i] = cu[i];
-  for (int s = 0; s < nb; ++s) {
-    const int b = src[s];
-    int len = 0;
-    if (b >= 0 && b < batch) len = cu[b + 1] - cu[b];
-    else record_status(status, DORA_ERR_DEVICE_BAD_COUNT);
-    if (len < 0 || end + len > t_cap) {
-      record_status(status, DORA_ERR_DEVICE_SEQLEN);
-      len = 0;
+    for (int i = threadIdx.x; i <= batch; i += blockDim.x) cu_out[i] = cu[i];
+  if (threadIdx.x == 0) {
+    carry = cu[batch];
+    last_fit = cu[batch] < t_cap ? cu[batch] : t_cap;
+  }
+  __syncthreads();
+  for (int base = 0; base < nb; base += kScanThreads) {
+    const int s = base + threadIdx.x;
+    long long len = 0;
+    if (s < nb) {
+      const int b = src[s];
+      if (b >= 0 && b < batch) len = cu[b + 1] - cu[b];
+      else record_status(status, DORA_ERR_DEVICE_BAD_COUNT);
+      if (len < 0) len = 0;
     }
-    end += len;
-    cu_out[batch + 1 + s] = end;
-    if (len_out != nullptr) len_out[s] = len;
+    long long inc = len;                                 // inclusive warp scan
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const long long o = __shfl_up_sync(0xffffffffu, inc, off);
+      if (lane >= off) inc += o;
+    }
+    if (lane == 31) warp_sum[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+      long long w = warp_sum[lane];
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const long long o = __shfl_up_sync(0xffffffffu, w, off);
+        if (lane >= off) w += o;
+      }
+      warp_sum[lane] = w;                                // inclusive over warps
+    }
+    __syncthreads();
+    const long long end = carry + (warp > 0 ? warp_sum[warp - 1] : 0) + inc;
+    const bool fits = end <= t_cap;
+    // the ends only grow: the last one that fits is the largest fitting end
+    const int fm = __reduce_max_sync(0xffffffffu, (s < nb && fits) ? static_cast<int>(end) : 0);
+    if (lane == 0) warp_fit[warp] = fm;
+    __syncthreads();                                     // carry and warp_fit are read
+    if (threadIdx.x == 0) {
+      int m = last_fit;
+      for (int w = 0; w < kScanThreads / 32; ++w) m = warp_fit[w] > m ? warp_fit[w] : m;
+      last_fit = m;
+    }
+    __syncthreads();
+    if (s < nb) {
+      // the first sequence that does not fit in t_cap, and every one after
+      // it, gets length 0 (its end is the last end that fits)
+      if (!fits && len > 0) record_status(status, DORA_ERR_DEVICE_SEQLEN);
+      cu_out[batch + 1 + s] = fits ? static_cast<int32_t>(end) : last_fit;
+      if (len_out != nullptr) len_out[s] = fits ? static_cast<int32_t>(len) : 0;
+    }
+    if (threadIdx.x == kScanThreads - 1) carry = end;
+    __syncthreads();
   }
 }
 
@@ -388,8 +435,8 @@ int dora_branch(dora_bf16* x, int32_t* ids, float* x_moments, const int32_t* cu,
   const int e = device_or_error();
   if (e != DORA_OK) return e;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  train::branch_cu_kernel<<<1, 32, 0, stream>>>(cu, batch, src, n_branch, t_cap, cu_out, len_out,
-                                                 status);
+  train::branch_cu_kernel<<<1, train::kScanThreads, 0, stream>>>(cu, batch, src, n_branch, t_cap,
+                                                                  cu_out, len_out, status);
   if (cudaGetLastError() != cudaSuccess) return DORA_ERR_CUDA;
   if (n_branch == 0) return DORA_OK;
   train::branch_rows_kernel<<<152 * 8, 256, 0, stream>>>(

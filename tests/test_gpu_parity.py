@@ -1025,7 +1025,8 @@ def test_block_with_actor_equals_actor_then_block(given_counts):
                                              (2, 4, 32, 32, 8, 128),
                                              (2, 3, 224, 224, 14, 768),    # DINOv2: K 588 -> 640
                                              (3, 1, 42, 28, 7, 128),       # K 49 -> 64
-                                             (1, 4, 24, 40, 4, 64)])       # generic path, K 64
+                                             (1, 4, 24, 40, 4, 64),        # even path, K 64
+                                             (2, 3, 36, 48, 6, 64)])       # even, K 108 -> 128
 def test_patch_embed_matches_oracle(b, c, h, w, patch, d):
     rng = np.random.default_rng(b * 100 + d)
     g = (h // patch) * (w // patch)
@@ -1119,7 +1120,8 @@ def test_dinov2_block_with_layerscale():
     assert_close(f64(r["x_out"][:t_out]), ref["x_out"], "dinov2 block")
 
 
-@pytest.mark.parametrize("name,dim", [("cfg6", 768), ("cfg1", 192), ("cfg4", 1024)])
+@pytest.mark.parametrize("name,dim", [("cfg6", 768), ("cfg1", 192), ("cfg4", 1024),
+                                      ("cfg1", 2048)])
 def test_classifier_head_lc1_matches_oracle(name, dim):
     cfg = S.get_config(name, batch=24)
     keeps, _ = S.keep_schedule(cfg, 17)
