@@ -48,6 +48,8 @@ NCU_TRAFFIC = {
     # profiles/gemm_tcgen05_deit_base_b256.md: mean over the 48 GEMM launches
     # of one forward step
     ("cfg3", "b34dcbc477c16fbd82653b7888b9deb4fa8716d95e482f5d9899e205d6137ff3"): 188246208,
+    # the same capture on the DINOv2-B/14 workload (bench.py --config cfg6)
+    ("cfg6", "b34dcbc477c16fbd82653b7888b9deb4fa8716d95e482f5d9899e205d6137ff3"): 270655605,
 }
 
 
