@@ -153,3 +153,21 @@ def test_dinov2_entry_points_host_checks(lib):
     # the 14-pixel patch workspace holds the K-padded (588 -> 640) patches and weight copy
     n = lib.dora_embed_workspace_size(2, 3, 224, 224, 14, 768)
     assert n >= 256 + 2 * 256 * 640 * 2 + 2 * 256 * 768 * 2 + 768 * 640 * 2
+
+
+def test_training_entry_points_host_checks(lib):
+    # Plackett-Luce: k_cap outside [1, 2048], missing buffers
+    assert lib.dora_pl_sample(16, 16, 16, 4, 100, 16, 0, 16, None, None, None) == 1
+    assert lib.dora_pl_sample(16, 16, 16, 4, 100, 16, 4096, 16, None, None, None) == 1
+    assert lib.dora_pl_sample(16, None, 16, 4, 100, 16, 8, 16, None, None, None) == 1
+    assert lib.dora_pl_logprob(16, 16, 4, 100, 16, 16, 0, 16, None, None, None, None) == 1
+    assert lib.dora_pl_logprob(16, 16, 4, 100, 16, 16, 8, None, None, None, None, None) == 1
+    # branch: dim % 8, misaligned rows, sources missing
+    assert lib.dora_branch(16, None, None, 16, 4, 100, 12, 16, 2, 16, None, None, None) == 1
+    assert lib.dora_branch(24, None, None, 16, 4, 100, 16, 16, 2, 16, None, None, None) == 1
+    assert lib.dora_branch(16, None, None, 16, 4, 100, 16, None, 2, 16, None, None, None) == 1
+    # fidelity cost: row pitch below the class count, tau <= 0
+    assert lib.dora_kd_cost(16, 16, None, 8, 4, 1000, 999, ctypes.c_float(3.0), 16, None,
+                            None) == 1
+    assert lib.dora_kd_cost(16, 16, None, 8, 4, 1000, 1024, ctypes.c_float(0.0), 16, None,
+                            None) == 1
