@@ -8,8 +8,9 @@ to the rollout up to and including block l, so it is branched off the
 rollout's output of block l (``dora_branch``: the image's surviving rows
 copied as a new sequence of the same packed batch) and from then on rides in
 the same kernels as the rollout with its keep count equal to its length.  The
-Native copies are branched before block 0; no shadow is branched at the last
-pruning block, whose prefix is the rollout itself.  Every GEMM row and every
+Native copies are branched just before the first pruning block (until then
+the rollout is the Native forward, so those blocks run once); no shadow is
+branched at the last pruning block, whose prefix is the rollout itself.  Every GEMM row and every
 attention sequence is computed independently of the others in the batch, so
 a shadow computed here has the same bits as the same prefix run alone.
 
@@ -118,13 +119,15 @@ class ShadowRollout:
         ids[:rows].copy_(ids0)
         cu = self.cu[0]
         cu[:b + 1].copy_(cu0)
-        # Native copies: whole images, never pruned
-        dora_branch(x, cu[:b + 1], self.src, cu[:2 * b + 1], ids=ids,
-                    len_out=self.keep[b:2 * b], status=self.status, stream=stream)
-        nseq, p, q = 2 * b, 0, 0
+        nseq, p, q = b, 0, 0
         for l, w in enumerate(self.blocks[:stop]):
             out = self.x[1 - p]
             mv_out = self.mv[1 - p] if l + 1 < self.depth else None
+            if l == self.prune[0]:
+                # Native copies: whole images, never pruned from here on
+                dora_branch(x, cu[:b + 1], self.src, cu[:2 * b + 1], ids=ids, x_moments=mv,
+                            len_out=self.keep[b:2 * b], status=self.status, stream=stream)
+                nseq = 2 * b
             if l in self.prune:
                 j = self.prune.index(l)
                 self.keep[:b].copy_(keeps[j])

@@ -278,10 +278,15 @@ def test_shadow_rollout_blocks_match_oracle():
         return bits(xs)[:t], cs, i_s.cpu().numpy()[:t]
 
     x_in, cu_in, ids_in = state(0)
-    assert np.array_equal(cu_in, np.concatenate([cu, cu[-1] + cu[1:]]))   # Native copies
+    assert np.array_equal(cu_in, cu)
     for l in range(cfg.depth):
         x_out, cu_out, ids_out = state(l + 1)
         wf = O.decode_weights(wbs[l])
+        if l == cfg.prune_blocks[0]:                     # the Native copies branch off here
+            rows = np.arange(cu_in[0], cu_in[b])
+            x_in = np.concatenate([x_in, x_in[rows]])
+            ids_in = np.concatenate([ids_in, ids_in[rows]])
+            cu_in = np.concatenate([cu_in, cu_in[-1] + cu_in[1:b + 1]])
         if l in cfg.prune_blocks:
             j = cfg.prune_blocks.index(l)
             scores = np.zeros(len(ids_in))
