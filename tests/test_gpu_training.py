@@ -398,3 +398,53 @@ def test_training_rollout_deletes_its_sampled_sets():
             assert abs(lp[j, i] - r) <= 1e-5 * (abs(r) + k * (1 + np.abs(s).max())), (l, i)
             gref = adv[i] * O.pl_logprob_grad(s, seq)
             assert np.all(np.abs(gj[lo + 1:hi] - gref) <= 2e-4 * (1 + np.abs(gref)))
+
+
+def test_branch_scan_across_chunks_and_overflow():
+    """More appended sequences than one 1024-wide scan chunk: boundaries carried
+    across chunks bit for bit; the first sequence past t_cap and every later
+    one get length 0 with the status set."""
+    rng = np.random.default_rng(14)
+    lens = rng.integers(0, 6, 300)
+    cu = O.cu_from_counts(lens)
+    src = rng.integers(0, 300, 2500).astype(np.int32)
+    want = np.concatenate([cu, cu[-1] + np.cumsum(lens[src])])
+    d = 64
+    t_cap = int(want[-1]) + 3
+    x = S.f32_to_bf16_bits(rng.standard_normal((t_cap, d)))
+    xt = bf(x)
+    cu_out = torch.zeros(301 + len(src), dtype=torch.int32, device=dev())
+    st = _status()
+    P.dora_branch(xt, i32(cu), i32(src), cu_out, status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert np.array_equal(cu_out.cpu().numpy(), want)
+    rows = np.concatenate([np.arange(cu[s], cu[s + 1]) for s in src]).astype(np.int64)
+    assert np.array_equal(bits(xt)[int(cu[-1]):int(want[-1])], x[rows])
+    # room for the sequences up to index 1500 only
+    cap = int(want[301 + 1500])
+    lens_out = torch.zeros(len(src), dtype=torch.int32, device=dev())
+    st = _status()
+    P.dora_branch(bf(x[:cap]), i32(cu), i32(src), cu_out, len_out=lens_out, status=st)
+    torch.cuda.synchronize()
+    got = cu_out.cpu().numpy()
+    fits = want[301:] <= cap
+    assert np.array_equal(got[301:][fits], want[301:][fits])
+    assert np.all(got[301:][~fits] == cap) and got[-1] == cap
+    lo = lens_out.cpu().numpy()
+    assert np.array_equal(lo[fits], lens[src][fits]) and np.all(lo[~fits] == 0)
+    assert int(st.item()) == (O.DORA_ERR_DEVICE_SEQLEN if (lens[src][~fits] > 0).any() else 0)
+
+
+def test_pl_sample_and_logprob_at_the_largest_image():
+    """2048 visual tokens (the kernels' shared-memory limit), k up to 2048."""
+    cu = O.cu_from_counts([2049, 2049, 300])
+    t = int(cu[-1])
+    rng = np.random.default_rng(15)
+    scores = (rng.standard_normal(t) * 3).astype(np.float32)
+    gumbel = _gumbel(rng, t)
+    k = np.array([2048, 1000, 150])
+    got, st = _run_sample(scores, gumbel, cu, k, 2048)
+    assert st == 0
+    assert np.array_equal(got, _oracle_orders(scores, gumbel, cu, k, 2048))
+    _check_logprob(scores, cu, got.astype(np.int32), k, np.ones(3))
