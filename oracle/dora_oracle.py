@@ -622,3 +622,18 @@ def shadow_forwards(x: np.ndarray, cu: np.ndarray, ids: np.ndarray, blocks: list
                          {b: v for b, v in prune.items() if b <= l}, head_dim)
     return out
 
+
+def step_rewards(costs: np.ndarray, removals: np.ndarray, blocks, depth: int, n0: int,
+                 a: float) -> np.ndarray:
+    """Local rewards of one image's actions (App. B.3): at the l-th acting
+    block r_l = 25 Delta C_l - a (D_l - D_{l-1}), Delta C_l = k_l (L - l) /
+    (L N0) (Eq. 4's per-block term), D_{-1} = 0.  costs[j] and removals[j]
+    belong to blocks[j] (increasing)."""
+    out = np.zeros(len(blocks))
+    prev = 0.0
+    for j, l in enumerate(blocks):
+        dc = removals[j] * (depth - l) / (depth * n0)
+        out[j] = 25.0 * dc - a * (costs[j] - prev)
+        prev = costs[j]
+    return out
+

@@ -812,3 +812,27 @@ def test_shadow_prefixes_end_at_native_and_rollout():
     assert np.array_equal(sh[2]["x"], roll["x"])
     assert np.array_equal(sh[0]["kept"][0], roll["kept"][0])
     assert np.array_equal(sh[0]["cu"], O.cu_from_counts(keeps[0]))
+
+
+def test_step_rewards_telescope():
+    """Sum over an episode of the local rewards = 25 C - a D_final (App. B.3),
+    with C from the definition C = (1 / L N0) sum_l (N0 - N_l^post) and the
+    per-block counts written out."""
+    rng = np.random.default_rng(10)
+    depth, n0 = 12, 196
+    blocks = [1, 3, 6, 9]
+    k = rng.integers(0, 40, len(blocks))
+    d = np.cumsum(rng.uniform(-0.2, 0.5, len(blocks)))
+    a = 30.0
+    r = O.step_rewards(d, k, blocks, depth, n0, a)
+    post, n = [], n0
+    for l in range(depth):
+        if l in blocks:
+            n -= k[blocks.index(l)]
+        post.append(n)
+    c = sum(n0 - p for p in post) / (depth * n0)
+    assert abs(r.sum() - (25 * c - a * d[-1])) < 1e-12
+    # a gate-off step (k = 0, D unchanged) earns nothing
+    k0, d0 = k.copy(), d.copy()
+    k0[2], d0[2] = 0, d0[1]
+    assert O.step_rewards(d0, k0, blocks, depth, n0, a)[2] == 0.0
