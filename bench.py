@@ -512,6 +512,8 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
         rem = [[torch.from_numpy((np.asarray(b_) - np.asarray(k_)).astype(np.int32)).to(dev)
                 for b_, k_ in zip(s_["befores"], s_["keeps"])] for s_ in hw.sets]
         adv = torch.from_numpy(grng.uniform(-1, 1, cfg.batch).astype(np.float32)).to(dev)
+        rem2 = [torch.stack(r_) for r_ in rem]
+        rwd = torch.zeros(len(cfg.prune_blocks), cfg.batch, dtype=torch.float32, device=dev)
         L0 = lanes[0]
 
         def train_step(i):
@@ -522,6 +524,7 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
             sr.head_and_costs(xo, cuo, E["norm_w"], E["norm_b"], 1e-6, w_head, b_head, lc1=lc1,
                               stream=stream)
             sr.logprob(rem[r], dlogp=adv, stream=stream)
+            sr.rewards(rem2[r], 30.0, rwd, stream=stream)
 
         tsecs, _ = timed(train_step, args.steps, max(args.warmup, 3))
         sst = int(sr.status.item())
@@ -534,7 +537,8 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream):
                     f"at {'/'.join(map(str, cfg.prune_blocks))}, Native forward and the "
                     "complete-prefix shadows branched after each pruning block but the last, "
                     "all in one packed batch through the same kernels; classifier on every "
-                    "sequence, fidelity costs (tau = 3), log-probabilities and their gradients"}
+                    "sequence, fidelity costs (tau = 3), local rewards (a = 30), "
+                    "log-probabilities and their gradients"}
 
     # context: torch eager dense forward of the same shapes and weights
     # (cuBLAS linears, scaled_dot_product_attention), not this library

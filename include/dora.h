@@ -649,6 +649,22 @@ int dora_kd_cost(const dora_bf16* z_native, const dora_bf16* z, const int32_t* s
                  int32_t shadows, int32_t batch, int32_t classes, int32_t ld, float tau,
                  float* cost, int32_t* status, dora_stream_t stream);
 
+/*
+ * dora_step_rewards -- local rewards of each image's actions (App. B.3):
+ * r_j = 25 k_j (L - l_j) / (L N0) - a (D_j - D_{j-1}), D_{-1} = 0, for the
+ * pruning blocks l_j = blocks[j] (int32 [n_blocks], device, increasing),
+ * removals int32 [n_blocks, batch] (device; k = 0 at a gate-off step), L =
+ * depth, N0 = n0 visual tokens, a the fidelity coefficient.  cost fp32 is the
+ * fidelity-cost array of a batched shadow forward, [(n_blocks + 1) batch] in
+ * sequence order: rollout (its D is that of the last pruning block), Native,
+ * then the shadows of pruning blocks 0..n_blocks-2.  reward fp32 [n_blocks,
+ * batch]; ret fp32 [batch] (nullable): the episode sum, which telescopes to
+ * 25 C - a D_final.
+ */
+int dora_step_rewards(const float* cost, const int32_t* removals, const int32_t* blocks,
+                      int32_t n_blocks, int32_t batch, int32_t depth, int32_t n0, float a,
+                      float* reward, float* ret, dora_stream_t stream);
+
 /* Synchronises the current device and copies the status word at `status_dev`
  * (a device int32, e.g. dora_workspace_status(ws)) to *code.  Test/debug
  * only: it blocks the host. */

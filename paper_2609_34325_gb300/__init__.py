@@ -25,7 +25,7 @@ __all__ = [
     "dora_merge_moments", "ActorWeights", "dora_actor", "dora_actor_workspace_size",
     "alloc_actor_workspace", "dora_pruned_block_actor", "dora_patch_embed",
     "dora_classifier_head", "dora_classifier_head_lc1", "dora_fold_layerscale",
-    "dora_pl_sample", "dora_pl_logprob", "dora_branch", "dora_kd_cost",
+    "dora_pl_sample", "dora_pl_logprob", "dora_branch", "dora_kd_cost", "dora_step_rewards",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -86,6 +86,8 @@ _SIGS = {
     "dora_branch": (ctypes.c_int, [_vp, _vp, _vp, _vp, _i32, _i32, _i32, _vp, _i32, _vp, _vp, _vp,
                                    _vp]),
     "dora_kd_cost": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _i32, _f32, _vp, _vp, _vp]),
+    "dora_step_rewards": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _i32, _f32, _vp, _vp,
+                                         _vp]),
     "dora_classifier_head": (ctypes.c_int, [_vp, _vp, _i32, _i32, _i32, _vp, _vp, _f32, _vp, _vp,
                                             _i32, _vp, _vp, _sz, _vp]),
     "dora_pruned_block_actor": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _i32, _vp, _vp, _vp,
@@ -801,4 +803,22 @@ def dora_kd_cost(z_native, z, cost, classes, shadow_image=None, tau=3.0, status=
                                        z_native.shape[0], int(classes), z.shape[1], float(tau),
                                        _ptr(cost), _ptr(status), _stream(stream)), "dora_kd_cost")
     return cost
+
+
+def dora_step_rewards(cost, removals, blocks, depth, n0, a, reward, ret=None, stream=None):
+    """Local rewards [P, B] (and episode sums [B]) from a batched shadow
+    forward's fidelity costs (rollout, Native, shadows) and the removal
+    counts [P, B] at the pruning blocks (device int32 [P])."""
+    _req(cost, torch.float32, "cost")
+    _req(removals, torch.int32, "removals")
+    _req(blocks, torch.int32, "blocks")
+    _req(reward, torch.float32, "reward")
+    _req(ret, torch.float32, "ret", optional=True)
+    p, b = removals.shape
+    if blocks.numel() != p or tuple(reward.shape) != (p, b) or cost.numel() < (p + 1) * b:
+        raise ValueError("removals and reward must be [P, B], blocks [P], cost >= (P + 1) B")
+    _check(load_library().dora_step_rewards(_ptr(cost), _ptr(removals), _ptr(blocks), p, b,
+                                            int(depth), int(n0), float(a), _ptr(reward),
+                                            _ptr(ret), _stream(stream)), "dora_step_rewards")
+    return reward
 

@@ -376,6 +376,32 @@ __global__ void kd_cost_kernel(const uint16_t* __restrict__ zn, const uint16_t* 
   if (lane == 0) cost[sh] = tau2 * kl;
 }
 
+// ---------------------------------------------------------------------------
+// Local rewards: one thread per image.  D_j of pruning block j < P - 1 is the
+// cost of its shadow, cost[(2 + j) B + i]; the last pruning block's prefix is
+// the whole rollout, cost[i]; D_{-1} = 0.
+// ---------------------------------------------------------------------------
+__global__ void step_rewards_kernel(const float* __restrict__ cost,
+                                    const int32_t* __restrict__ removals,
+                                    const int32_t* __restrict__ blocks, int n_blocks, int batch,
+                                    int depth, int n0, float a, float* __restrict__ reward,
+                                    float* __restrict__ ret) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= batch) return;
+  const float inv = 25.f / (static_cast<float>(depth) * static_cast<float>(n0));
+  float prev = 0.f, total = 0.f;
+  for (int j = 0; j < n_blocks; ++j) {
+    const float d = j + 1 < n_blocks ? cost[static_cast<size_t>(2 + j) * batch + i] : cost[i];
+    const float dc = static_cast<float>(removals[static_cast<size_t>(j) * batch + i]) *
+                     static_cast<float>(depth - blocks[j]) * inv;
+    const float r = dc - a * (d - prev);
+    reward[static_cast<size_t>(j) * batch + i] = r;
+    total += r;
+    prev = d;
+  }
+  if (ret != nullptr) ret[i] = total;
+}
+
 }  // namespace train
 }  // namespace dora
 
@@ -457,6 +483,21 @@ int dora_kd_cost(const dora_bf16* z_native, const dora_bf16* z, const int32_t* s
   const int blocks = (shadows * 32 + 255) / 256;
   train::kd_cost_kernel<<<blocks, 256, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
       z_native, z, shadow_image, shadows, batch, classes, ld, 1.f / tau, tau * tau, cost, status);
+  return cudaGetLastError() == cudaSuccess ? DORA_OK : DORA_ERR_CUDA;
+}
+
+int dora_step_rewards(const float* cost, const int32_t* removals, const int32_t* blocks,
+                      int32_t n_blocks, int32_t batch, int32_t depth, int32_t n0, float a,
+                      float* reward, float* ret, dora_stream_t stream) {
+  if (n_blocks < 1 || batch < 1 || depth < 1 || n0 < 1 || !(a == a))
+    return DORA_ERR_INVALID_ARG;
+  if (cost == nullptr || removals == nullptr || blocks == nullptr || reward == nullptr)
+    return DORA_ERR_INVALID_ARG;
+  const int e = device_or_error();
+  if (e != DORA_OK) return e;
+  train::step_rewards_kernel<<<(batch + 255) / 256, 256, 0,
+                               reinterpret_cast<cudaStream_t>(stream)>>>(
+      cost, removals, blocks, n_blocks, batch, depth, n0, a, reward, ret);
   return cudaGetLastError() == cudaSuccess ? DORA_OK : DORA_ERR_CUDA;
 }
 

@@ -25,7 +25,7 @@ import torch
 
 from . import (alloc_workspace, dora_branch, dora_classifier_head, dora_classifier_head_lc1,
                dora_gather_scores, dora_kd_cost, dora_pl_logprob, dora_pl_sample,
-               dora_pruned_block)
+               dora_pruned_block, dora_step_rewards)
 
 
 class ShadowRollout:
@@ -172,6 +172,15 @@ class ShadowRollout:
                             self.logp[j], grad=self.grad[j], dlogp=dlogp, status=self.status,
                             stream=stream)
         return self.logp, self.grad
+
+    def rewards(self, removals, a, reward, ret=None, stream=None):
+        """Local rewards [P, B] of the last training forward's actions from the
+        fidelity costs of head_and_costs (App. B.3); removals int32 [P, B]."""
+        if not hasattr(self, "_blocks_dev"):
+            self._blocks_dev = torch.tensor(self.prune, dtype=torch.int32,
+                                            device=self.cost.device)
+        return dora_step_rewards(self.cost, removals, self._blocks_dev, self.depth,
+                                 self.n_tokens - 1, a, reward, ret=ret, stream=stream)
 
     def head_and_costs(self, x, cu, norm_w, norm_b, eps, w_head, b_head, lc1=False, tau=3.0,
                        stream=None):

@@ -171,3 +171,10 @@ def test_training_entry_points_host_checks(lib):
                             None) == 1
     assert lib.dora_kd_cost(16, 16, None, 8, 4, 1000, 1024, ctypes.c_float(0.0), 16, None,
                             None) == 1
+
+
+def test_step_rewards_host_checks(lib):
+    assert lib.dora_step_rewards(16, 16, 16, 0, 4, 12, 196, ctypes.c_float(30.0), 16, None,
+                                 None) == 1
+    assert lib.dora_step_rewards(16, None, 16, 3, 4, 12, 196, ctypes.c_float(30.0), 16, None,
+                                 None) == 1

@@ -448,3 +448,30 @@ def test_pl_sample_and_logprob_at_the_largest_image():
     assert st == 0
     assert np.array_equal(got, _oracle_orders(scores, gumbel, cu, k, 2048))
     _check_logprob(scores, cu, got.astype(np.int32), k, np.ones(3))
+
+
+def test_step_rewards_from_the_shadow_costs():
+    """Local rewards (App. B.3) from the batched forward's fidelity costs,
+    against the oracle's rewards on the same costs; the episode sums."""
+    cfg, cu, ids, x, wbs, keeps, tables = _shadow_case()
+    sr, xo, cuo, _ = _run_shadows(cfg, cu, ids, x, wbs, keeps, tables)
+    wh = S.embed_head_weights(cfg, 13)
+    w_head = np.zeros((1024, cfg.dim), np.uint16)
+    w_head[:1000] = wh["w_head"]
+    _, cost = sr.head_and_costs(xo, i32(cuo), bf(wh["norm_w"]), bf(wh["norm_b"]), 1e-6,
+                                bf(w_head), None)
+    _, befores = S.keep_schedule(cfg, 13)
+    rem = np.stack([np.asarray(b_) - np.asarray(k) for b_, k in zip(befores, keeps)])
+    b, npb = cfg.batch, len(cfg.prune_blocks)
+    reward = torch.zeros(npb, b, dtype=torch.float32, device=dev())
+    ret = torch.zeros(b, dtype=torch.float32, device=dev())
+    sr.rewards(i32(rem), 30.0, reward, ret=ret)
+    torch.cuda.synchronize()
+    c = cost.cpu().numpy().astype(np.float64)
+    r = reward.cpu().numpy().astype(np.float64)
+    for i in range(b):
+        d = [c[(2 + j) * b + i] for j in range(npb - 1)] + [c[i]]
+        ref = O.step_rewards(np.array(d), rem[:, i], cfg.prune_blocks, cfg.depth,
+                             cfg.n_vis0, 30.0)
+        assert np.allclose(r[:, i], ref, rtol=1e-5, atol=1e-5), (i, r[:, i], ref)
+        assert abs(ret[i].item() - ref.sum()) <= 1e-5 * (1 + abs(ref.sum()))
