@@ -35,6 +35,9 @@ class ShadowRollout:
 
     def __init__(self, blocks: list, batch: int, n_tokens: int, prune_blocks, device,
                  classes: int = 1000):
+        if not prune_blocks or list(prune_blocks) != sorted(set(prune_blocks)) or \
+                prune_blocks[-1] >= len(blocks) or prune_blocks[0] < 0:
+            raise ValueError("prune_blocks must be increasing block indices, at least one")
         self.blocks = blocks
         self.b = batch
         self.n_tokens = n_tokens
