@@ -178,3 +178,10 @@ def test_step_rewards_host_checks(lib):
                                  None) == 1
     assert lib.dora_step_rewards(16, None, 16, 3, 4, 12, 196, ctypes.c_float(30.0), 16, None,
                                  None) == 1
+
+
+def test_shadow_rollout_rejects_bad_schedules():
+    from paper_2609_34325_gb300.shadow import ShadowRollout
+    for prune in ((), (2, 1), (0, 5), (-1, 2), (1, 1)):
+        with pytest.raises(ValueError):
+            ShadowRollout([object()] * 3, 4, 197, prune, "cpu")
