@@ -12,13 +12,16 @@
 // Design (one persistent CTA per SM, CTAs paired in clusters of two):
 //   The two CTAs of a cluster work on vertically adjacent output tiles
 //   (M-tiles 2p and 2p+1 of the same N-tile), so they need the same W tile.
-//   warp 0     TMA producer: the CTA's own 128x64 X tile, plus one half of the
-//              shared BNx64 W tile multicast into both CTAs, per stage of a
-//              4-stage shared-memory ring (128-byte swizzle).  Each W byte is
-//              read from L2 once per pair.
-//   warp 1     MMA issuer: one thread issues tcgen05.mma (M=128, N=BN, K=16)
-//              into one of two TMEM accumulators (2 x BN fp32 columns), so
-//              the epilogue of tile t overlaps the main loop of tile t+1.
+//   warp 0     TMA producer: the CTA's own 128x64 X tile and its part of the
+//              BNx64 W tile, per stage of a shared-memory ring (128-byte
+//              swizzle).  256-wide tiles run as a CTA pair (below), each CTA
+//              loading half of W; narrower tiles load the whole W tile in each
+//              CTA (both CTAs of a cluster read the same W tile, so the second
+//              read is an L2 hit).
+//   warp 1     MMA issuer: one thread issues tcgen05.mma (M=128, N=BN, K=16,
+//              or M=256 across the pair) into one of two TMEM accumulators
+//              (2 x BN fp32 columns), so the epilogue of tile t overlaps the
+//              main loop of tile t+1.
 //   epilogue warps (2 .. 1 + kEpiWarps): tcgen05.ld the accumulator (each
 //              thread owns one row; the warps of a TMEM lane quarter split the
 //              columns), release it once in registers, add bias, GELU or
@@ -51,7 +54,7 @@ constexpr int kSmemLimit = 227 * 1024;
 // Pair mode: one MMA of M = 256 spans both CTAs of the cluster, each holding
 // its own 128 rows of X and one half of the W tile, so a stage is 32 KB
 // instead of 48; the shared memory read per MMA drops by a third.  Otherwise
-// one MMA per CTA, with W halves multicast.
+// one MMA per CTA on a whole W tile of its own.
 // Epilogue warps: a multiple of 4 (one per TMEM lane quarter); the ALU-heavy
 // plain GELU epilogue gets 16, the others 8 with two staging buffers per warp
 // (the residual epilogue one per chunk).  The stages fill what shared memory is left.
@@ -256,8 +259,8 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
     for (int i = 0; i < kStages; ++i) {
       mbar_init(&s.full[i], 1);
       // pair mode: the first CTA's MMAs release both CTAs' stages; otherwise
-      // both CTAs' MMAs release a stage (its W halves came from both)
-      mbar_init(&s.empty[i], kPair ? 1 : kCluster);
+      // each CTA's own MMAs release its stage
+      mbar_init(&s.empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s.acc_full[i], 1);
@@ -283,7 +286,7 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
     else tmem_alloc(&s.tmem_base, kTmemCols);
   }
   tc_fence_before();
-  cluster_sync();              // peers' barriers are initialised before any multicast
+  cluster_sync();              // peers' barriers are initialised before any remote signal
   tc_fence_after();
   // the set-up above overlaps the previous kernel; global memory waits for it
   pdl_wait();
@@ -318,10 +321,11 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
             tma_load_2d_pair(s.a[st], &tmA, &s.full[st], 0, kb * BK, mt * BM);
             tma_load_2d_pair(s.b[st], &tmB, &s.full[st], 0, kb * BK, nt * BN + rank * kHalfB);
           } else {
+            // the X tile and both halves of the W tile (the map's box is BN/2 rows)
             mbar_arrive_expect_tx(&s.full[st], (BM + BN) * BK * 2);
             tma_load_2d(s.a[st], &tmA, &s.full[st], kb * BK, mt * BM);
-            tma_load_2d_multicast(s.b[st] + rank * kHalfB * BK, &tmB, &s.full[st], kb * BK,
-                                  nt * BN + rank * kHalfB, kPairMask);
+            tma_load_2d(s.b[st], &tmB, &s.full[st], kb * BK, nt * BN);
+            tma_load_2d(s.b[st] + kHalfB * BK, &tmB, &s.full[st], kb * BK, nt * BN + kHalfB);
           }
           ++it;
         }
@@ -385,7 +389,7 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k)
             mma_bf16_ss(d, ad + 2 * k, bd + 2 * k, idesc, (kb | k) != 0 ? 1u : 0u);
-          mma_commit_multicast(&s.empty[st], kPairMask);   // both CTAs' W halves free
+          mma_commit(&s.empty[st]);                        // this CTA's stage free
           ++it;
         }
         if (ok) mma_commit(&s.acc_full[acc]);
@@ -608,7 +612,6 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
       if (!kPair || rank == 0)
         for (int it = s.consumed; it < s.issued; ++it)
           mbar_wait_limited(&s.full[it % kStages], (it / kStages) & 1, 100ull * 1000 * 1000);
-      __nanosleep(50000);      // the peer's last multicast halves
     }
     __syncthreads();
   }

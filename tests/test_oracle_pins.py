@@ -535,6 +535,90 @@ def test_actor_budget_masked_argmax_brute_force():
     assert O.actor_budget(rng.standard_normal(128), 50, n0, wt)[0] == 2
 
 
+def _gelu_lib(x: float) -> float:
+    """Exact GELU from PyTorch's float64 routine (independent of the oracle's)."""
+    return float(torch.nn.functional.gelu(torch.tensor(x, dtype=torch.float64)))
+
+
+def test_actor_budget_logits_closed_form():
+    """Appendix A.1 budget head: logits = W2 GELU(W1 LN(Z_CLS) + b1) + b2.
+    Z_CLS = mu + sigma s with s alternating +-1 over the 128 channels has row
+    mean mu and biased variance sigma^2 exactly, so LN(Z_CLS)_c = g_c s_c
+    sigma / sqrt(sigma^2 + eps) + beta_c in closed form.  W1 = I and a one-hot
+    W2 (logit m reads hidden unit m mod 128 with weight (m + 1) / 10) expose
+    every logit.  The large mean (mu = 500) makes a missing LayerNorm fail,
+    and the hidden values near +-1 separate GELU from SiLU and ReLU."""
+    n0 = 196
+    w = _actor_w(64, n0=n0)
+    grid = O.budget_grid(n0)
+    m = len(grid)
+    mu, sigma = 500.0, 0.75
+    s = np.array([1.0 if c % 2 == 0 else -1.0 for c in range(128)])
+    z = mu + sigma * s
+    w1 = np.eye(128)
+    w2 = np.zeros((m, 128))
+    for j in range(m):
+        w2[j, j % 128] = (j + 1) / 10
+    wb = dict(w, bud_w1=w1, bud_w2=w2)
+    k, logits = O.actor_budget(z, 120, n0, wb)
+    scale = sigma / math.sqrt(sigma * sigma + O.ACTOR_EPS)
+    for j in range(m):
+        c = j % 128
+        u = w["bud_ln_w"][c] * s[c] * scale + w["bud_ln_b"][c]
+        ref = (j + 1) / 10 * _gelu_lib(u + w["bud_b1"][c]) + w["bud_b2"][j]
+        assert abs(logits[j] - ref) < 1e-12, (j, logits[j], ref)
+    assert k == int(grid[int(np.argmax(np.where(grid <= 116, logits, -np.inf)))])
+
+
+def test_actor_encoder_feed_forward_closed_form():
+    """Appendix A.1 shared encoder, feed-forward sublayer: with the attention
+    output layer zeroed, Z = X + W_fc2 GELU(W_fc1 LN2(X) + b_fc1) + b_fc2,
+    pre-LayerNorm.  X is built with a closed-form row mean and variance:
+    W_in reads key entry 0 with sign s_c (alternating +-1) and key entry 1
+    with weight 1, so X_jc = s_c sigma_j + mu_j (+ h_0 on CLS through W_h),
+    and LN2(X)_jc = g_c s_c sigma_j / sqrt(sigma_j^2 + eps) + beta_c.  Hidden
+    unit r reads LN2 column r mod 128; output c mixes hidden units c and
+    128 + c as 1.5 GELU(.) - 0.5 GELU(.).  The large row means make a missing
+    or post-placed LayerNorm fail; the hidden values separate GELU from SiLU
+    and ReLU."""
+    d, n = 64, 5
+    w = _actor_w(d)
+    s = np.array([1.0 if c % 2 == 0 else -1.0 for c in range(128)])
+    w_in = np.zeros((128, d))
+    w_in[:, 0] = s
+    w_in[:, 1] = 1.0
+    w_h = np.zeros((128, 3))
+    w_h[:, 0] = 1.0
+    fc1 = np.zeros((256, 128))
+    for r in range(256):
+        fc1[r, r % 128] = 1.0
+    fc2 = np.zeros((128, 256))
+    for c in range(128):
+        fc2[c, c] = 1.5
+        fc2[c, 128 + c] = -0.5
+    we = dict(w, enc_w_in=w_in, enc_b_in=np.zeros(128), enc_w_h=w_h,
+              enc_w_o=np.zeros_like(w["enc_w_o"]), enc_b_o=np.zeros_like(w["enc_b_o"]),
+              enc_w_fc1=fc1, enc_w_fc2=fc2)
+    e_c = np.zeros(128)
+    h = np.array([7.0, 0.2, 0.1])
+    sig = [0.5, 1.0, 1.7, 2.5, 0.9, 3.0]
+    mus = [40.0 + 25.0 * j for j in range(n + 1)]
+    keys = np.zeros((n + 1, d))
+    for j in range(n + 1):
+        keys[j, 0], keys[j, 1] = sig[j], mus[j]
+    z = O.actor_encoder(keys, e_c, h, we)
+    g, beta = w["enc_ln2_w"], w["enc_ln2_b"]
+    b1, b2 = w["enc_b_fc1"], w["enc_b_fc2"]
+    for j in range(n + 1):
+        mu = mus[j] + (h[0] if j == 0 else 0.0)
+        scale = sig[j] / math.sqrt(sig[j] ** 2 + O.ACTOR_EPS)
+        for c in range(128):
+            x = s[c] * sig[j] + mu
+            u = g[c] * s[c] * scale + beta[c]
+            ref = x + 1.5 * _gelu_lib(u + b1[c]) - 0.5 * _gelu_lib(u + b1[128 + c]) + b2[c]
+            assert abs(z[j, c] - ref) < 1e-11, (j, c, z[j, c], ref)
+
+
 def test_actor_selector_closed_form():
     """Eq. 2 with a one-hot first layer: s_j = silu(Z_j[0] + 2 k / N_l) + 0.25."""
     w = _actor_w(64)
