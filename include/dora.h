@@ -382,7 +382,9 @@ int32_t* dora_workspace_status(void* workspace);
  *    a DeiT-Base-shape block with pre-folded weights, 1,600 without).
  *  - The first call on a device looks up the device address of the scratch
  *    array (cudaGetSymbolAddress) with that device current; make that first
- *    call before any stream capture on the device.
+ *    call before any stream capture on the device.  The address is kept for
+ *    the life of the process, so a cudaDeviceReset after that first call is
+ *    not supported: the kept address may no longer be the array's.
  *  - No cudaMalloc, cudaFree or other allocating routine is called.
  *  - Every call on a device shares the same scratch, which keeps the previous
  *    call's contents: the status word in it is cleared at the start of each
@@ -547,7 +549,7 @@ int dora_classifier_head(const dora_bf16* x, const int32_t* cu, int32_t batch, i
                          size_t workspace_bytes, dora_stream_t stream);
 
 /*
- * DINOv2 backbones (App. E.2: register-free DINOv2-B/14 with its LC1 readout
+ * DINOv2 backbones (App. E.3: register-free DINOv2-B/14 with its LC1 readout
  * and LayerScale kept).
  *
  * dora_classifier_head_lc1 -- logits bf16 [batch, classes] = u_i W_head^T +

@@ -35,7 +35,7 @@ block of Eq. 1 (Sec. 3.1), in float64, from bf16/fp32 inputs decoded exactly:
                     log-probability (App. A.3) and the shadows' fidelity cost
                     (App. B.2).
 * ``lc1_readout``, ``classifier_head_lc1``, LayerScale in the block halves
-                    the DINOv2-B/14 backbone (App. E.2): LayerScale on both
+                    the DINOv2-B/14 backbone (App. E.3): LayerScale on both
                     residual branches and the LC1 readout.
 
 Readings where the paper is silent:
@@ -516,7 +516,7 @@ def classifier_head(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.nd
 
 def lc1_readout(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.ndarray,
                 eps: float) -> np.ndarray:
-    """DINOv2's LC1 readout (App. E.2, baseline implementations): the final
+    """DINOv2's LC1 readout (App. E.3, baseline implementations): the final
     LayerNorm applied to every token, then each image's normalised CLS row
     concatenated with the mean of its normalised surviving visual rows
     ([B, 2 d]; an image without visual tokens contributes a zero mean)."""
@@ -537,7 +537,7 @@ def lc1_readout(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.ndarra
 
 def classifier_head_lc1(x: np.ndarray, cu: np.ndarray, ln_w: np.ndarray, ln_b: np.ndarray,
                         eps: float, w_head: np.ndarray, b_head: np.ndarray) -> np.ndarray:
-    """Class logits from the LC1 features (App. E.2): the linear layer
+    """Class logits from the LC1 features (App. E.3): the linear layer
     w_head [classes, 2 d] applied to lc1_readout's [B, 2 d] rows."""
     return linear(lc1_readout(x, cu, ln_w, ln_b, eps), w_head, b_head)
 

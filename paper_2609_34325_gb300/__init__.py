@@ -635,7 +635,13 @@ def dora_pruned_block_actor(x_in, cu_in, weights: BlockWeights, max_seqlen, x_ou
 
 def dora_patch_embed(images, w_pe, b_pe, cls, pos, patch, x0, workspace=None, stream=None):
     """Packed tokens x0 [B * (g + 1), d] from images [B, C, H, W]: strided patch
-    convolution (w_pe [d, C * patch^2]), CLS first, position embeddings added."""
+    convolution (w_pe [d, C * patch^2]), CLS first, position embeddings added.
+
+    The C entry point never allocates.  This wrapper does when ``workspace``
+    is None: it then makes a zero-filled uint8 tensor of
+    ``dora_embed_workspace_size`` bytes with torch on every such call.  The
+    workspace used is returned; pass it back on later calls to keep a loop
+    free of allocations."""
     for n, t in (("images", images), ("w_pe", w_pe), ("cls", cls), ("pos", pos), ("x0", x0)):
         _req(t, torch.bfloat16, n)
     _req(b_pe, torch.bfloat16, "b_pe", optional=True)
@@ -674,7 +680,12 @@ def dora_fold_layerscale(w, b, gamma, w_out=None, b_out=None, stream=None):
 def dora_classifier_head_lc1(x, cu, norm_w, norm_b, eps, w_head, b_head, logits, workspace=None,
                              stream=None):
     """logits [B, classes] from DINOv2's LC1 features [LN(CLS), mean LN(visual
-    rows)] of each image (w_head [classes, 2 d], classes a multiple of 32)."""
+    rows)] of each image (w_head [classes, 2 d], classes a multiple of 32).
+
+    With ``workspace`` None a zero-filled workspace of
+    ``dora_head_lc1_workspace_size`` bytes is allocated with torch on that
+    call; the workspace used is returned for reuse (the C entry point itself
+    never allocates)."""
     for n, t in (("x", x), ("norm_w", norm_w), ("norm_b", norm_b), ("w_head", w_head),
                  ("logits", logits)):
         _req(t, torch.bfloat16, n)
@@ -700,7 +711,12 @@ def dora_classifier_head_lc1(x, cu, norm_w, norm_b, eps, w_head, b_head, logits,
 def dora_classifier_head(x, cu, norm_w, norm_b, eps, w_head, b_head, logits, workspace=None,
                          stream=None):
     """logits [B, classes] = LayerNorm(x[cu[i]]) W_head^T + b_head per image
-    (classes a multiple of 32: pad the head with zero rows)."""
+    (classes a multiple of 32: pad the head with zero rows).
+
+    With ``workspace`` None a zero-filled workspace of
+    ``dora_head_workspace_size`` bytes is allocated with torch on that call;
+    the workspace used is returned for reuse (the C entry point itself never
+    allocates)."""
     for n, t in (("x", x), ("norm_w", norm_w), ("norm_b", norm_b), ("w_head", w_head),
                  ("logits", logits)):
         _req(t, torch.bfloat16, n)

@@ -56,10 +56,7 @@ constexpr int kEpiWarp0 = 12;   // epilogue warps 12-15
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleLog2 = 8.f;    // raise the reference maximum past 2^8
 constexpr uint32_t kSleepNs = 200000;  // waiting threads sleep instead of spinning
-#ifndef ATTN_SP_BUFS
-#define ATTN_SP_BUFS 3
-#endif
-constexpr int kSpBufs = ATTN_SP_BUFS;   // S/P buffers, used by steps in turn
+constexpr int kSpBufs = 3;      // S/P buffers, used by steps in turn
 __device__ __forceinline__ uint32_t tmem_sp(int b) { return 128u * static_cast<uint32_t>(b); }
 __device__ __forceinline__ uint32_t tmem_o(int b) {
   return 128u * kSpBufs + 64u * static_cast<uint32_t>(b);

@@ -6,7 +6,7 @@
 //                     added, into the packed token layout of the blocks;
 //   classifier head   the final LayerNorm on each image's CLS row and the
 //                     linear layer to the class logits (tcgen05 GEMM);
-//   LC1 head          DINOv2's readout (App. E.2): the final LayerNorm on every
+//   LC1 head          DINOv2's readout (App. E.3): the final LayerNorm on every
 //                     surviving token, normalised CLS ++ the mean of the
 //                     normalised visual rows of each image, then the linear
 //                     layer on the 2 d features;

@@ -63,26 +63,17 @@ struct Cfg {
   static constexpr bool kPair = PAIR;
   static constexpr int kBRows = kPair ? BN / 2 : BN;   // W rows held per CTA
   static constexpr bool kLn = EPI == kEpiLn || EPI == kEpiLnGelu;
-#ifndef GEMM_LNGELU_WARPS
-#define GEMM_LNGELU_WARPS 16
-#endif
-  static constexpr int kEpiWarps =
-      EPI == DORA_EPI_BIAS_GELU ? 16 : (EPI == kEpiLnGelu ? GEMM_LNGELU_WARPS : 8);
+  // the two GELU epilogues are ALU-bound: 16 warps; the others 8
+  static constexpr int kEpiWarps = (EPI == DORA_EPI_BIAS_GELU || EPI == kEpiLnGelu) ? 16 : 8;
   static constexpr int kColGroups = kEpiWarps / 4;
   static constexpr int kCols = BN / kColGroups;         // columns per epilogue warp
   static constexpr int kChunks = kCols / 32;
   // chunks per TMEM load: two (64 registers) unless 16 warps cap registers at 96
-#ifndef GEMM_GELU16_BATCH
-#define GEMM_GELU16_BATCH 1
-#endif
-  static constexpr int kBatch =
-      kEpiWarps == 16 ? GEMM_GELU16_BATCH : (kChunks < 2 ? kChunks : 2);
+  static constexpr int kBatch = kEpiWarps == 16 ? 1 : (kChunks < 2 ? kChunks : 2);
   static constexpr bool kResTma = EPI == DORA_EPI_BIAS_RESIDUAL;
-#ifndef GEMM_LN_BUFS
-#define GEMM_LN_BUFS 1
-#endif
-  static constexpr int kBufs =
-      kResTma ? kChunks : (kEpiWarps == 16 ? 1 : (kLn ? GEMM_LN_BUFS : 2));
+  // staging buffers per epilogue warp: one per chunk for the residual (its
+  // TMA load lands there), one with 16 warps or the folded LayerNorm, else two
+  static constexpr int kBufs = kResTma ? kChunks : ((kEpiWarps == 16 || kLn) ? 1 : 2);
   // folded LayerNorm: each epilogue warp's c and d columns, staged per tile
   static constexpr int kCdCols = kLn ? kCols : 1;
   static constexpr int kThreads = 64 + 32 * kEpiWarps;

@@ -450,16 +450,35 @@ def test_pl_sample_and_logprob_at_the_largest_image():
     _check_logprob(scores, cu, got.astype(np.int32), k, np.ones(3))
 
 
+def _kd_first_order_bound(zn, z, dzn, dz, tau=3.0):
+    """First-order bound on the change of D = tau^2 KL(softmax(zn/tau) ||
+    softmax(z/tau)) when the logits move by at most dzn (Native) and dz
+    (shadow) in every entry: dD/dz_c = tau (p_c - pn_c) and dD/dzn_c =
+    tau pn_c (log(pn_c / p_c) - D / tau^2)."""
+    lpn = O.log_softmax(zn / tau)
+    lp = O.log_softmax(z / tau)
+    pn, p = np.exp(lpn), np.exp(lp)
+    d = tau * tau * float(np.sum(pn * (lpn - lp)))
+    return (tau * float(np.abs(p - pn).sum()) * dz
+            + tau * float(np.sum(pn * np.abs(lpn - lp - d / (tau * tau)))) * dzn)
+
+
 def test_step_rewards_from_the_shadow_costs():
     """Local rewards (App. B.3) from the batched forward's fidelity costs,
-    against the oracle's rewards on the same costs; the episode sums."""
+    against the oracle's rewards on the same costs.  The costs are taken by
+    the sequence groups of the batch, whose prefixes are pinned against the
+    oracle's forwards elsewhere; each image's episode sum is checked against
+    the telescoping identity 25 C - a D_final with C from the count schedule
+    (Eq. 4) and D_final the rollout's own cost; and the first shadow's cost
+    against the oracle's complete-prefix shadow (App. B.2) run end to end in
+    fp64, within the first-order bound of the measured logit error."""
     cfg, cu, ids, x, wbs, keeps, tables = _shadow_case()
     sr, xo, cuo, _ = _run_shadows(cfg, cu, ids, x, wbs, keeps, tables)
     wh = S.embed_head_weights(cfg, 13)
     w_head = np.zeros((1024, cfg.dim), np.uint16)
     w_head[:1000] = wh["w_head"]
-    _, cost = sr.head_and_costs(xo, i32(cuo), bf(wh["norm_w"]), bf(wh["norm_b"]), 1e-6,
-                                bf(w_head), None)
+    logits, cost = sr.head_and_costs(xo, i32(cuo), bf(wh["norm_w"]), bf(wh["norm_b"]), 1e-6,
+                                     bf(w_head), None)
     _, befores = S.keep_schedule(cfg, 13)
     rem = np.stack([np.asarray(b_) - np.asarray(k) for b_, k in zip(befores, keeps)])
     b, npb = cfg.batch, len(cfg.prune_blocks)
@@ -469,9 +488,30 @@ def test_step_rewards_from_the_shadow_costs():
     torch.cuda.synchronize()
     c = cost.cpu().numpy().astype(np.float64)
     r = reward.cpu().numpy().astype(np.float64)
+    comp = S.compression_from_counts(cfg, keeps, befores)
+    g_roll = sr.groups["rollout"]
     for i in range(b):
-        d = [c[(2 + j) * b + i] for j in range(npb - 1)] + [c[i]]
+        d = [c[sr.groups[l] + i] for l in cfg.prune_blocks[:-1]] + [c[g_roll + i]]
         ref = O.step_rewards(np.array(d), rem[:, i], cfg.prune_blocks, cfg.depth,
                              cfg.n_vis0, 30.0)
         assert np.allclose(r[:, i], ref, rtol=1e-5, atol=1e-5), (i, r[:, i], ref)
         assert abs(ret[i].item() - ref.sum()) <= 1e-5 * (1 + abs(ref.sum()))
+        tele = 25.0 * comp[i] - 30.0 * c[g_roll + i]
+        assert abs(ret[i].item() - tele) <= 1e-5 * (1 + abs(tele)), (i, ret[i].item(), tele)
+    # the first shadow's cost against the oracle's own complete-prefix forward
+    prune = {l: (tables[j], keeps[j]) for j, l in enumerate(cfg.prune_blocks)}
+    l0 = cfg.prune_blocks[0]
+    fw = O.shadow_forwards(O.bf16_to_f64(x), cu, ids, [O.decode_weights(w) for w in wbs],
+                           cfg.heads, cfg.ln_eps, {l0: prune[l0]})
+    head = (O.bf16_to_f64(wh["norm_w"]), O.bf16_to_f64(wh["norm_b"]), 1e-6,
+            O.bf16_to_f64(w_head[:1000]), np.zeros(1000))
+    zn = O.classifier_head(fw[-1]["x"], fw[-1]["cu"], *head)
+    zs = O.classifier_head(fw[l0]["x"], fw[l0]["cu"], *head)
+    lg = f64(logits)[:, :1000]
+    g_nat, g_sh = sr.groups["native"], sr.groups[l0]
+    for i in range(b):
+        dzn = float(np.abs(lg[g_nat + i] - zn[i]).max())
+        dz = float(np.abs(lg[g_sh + i] - zs[i]).max())
+        want = O.kd_cost(zn[i], zs[i], 3.0)
+        tol = 2.0 * _kd_first_order_bound(zn[i], zs[i], dzn, dz) + 1e-4 * (1 + want)
+        assert abs(c[g_sh + i] - want) <= tol, (i, c[g_sh + i], want, tol)

@@ -717,7 +717,7 @@ def test_classifier_reads_only_cls_rows():
 
 
 # ---------------------------------------------------------------------------
-# DINOv2 pieces: LayerScale and the LC1 readout (App. E.2; Table 3)
+# DINOv2 pieces: LayerScale and the LC1 readout (App. E.3; Table 3)
 # ---------------------------------------------------------------------------
 
 def test_layerscale_zero_leaves_the_residual_stream():

@@ -51,11 +51,15 @@ def _outputs(t, b, dim):
                 kept_idx=torch.zeros(t, dtype=torch.int32, device=dev))
 
 
-def test_noalloc_matches_workspace_entry_on_consecutive_calls():
-    cfg = S.get_config("cfg1")                       # 8 x 197 tokens, D=192: ~7 MB scratch
+def _check_consecutive_calls(cfg, seeds):
+    """Calls in a row through the scratch-array entry point against the
+    workspace entry point on the same inputs: the same kernels run on the same
+    data, so every output must match bit for bit.  The first call is also
+    checked against the fp64 oracle within the block tolerance."""
     t = cfg.batch * cfg.n_tokens
-    for seed, prune in ((31, True), (32, True), (33, False)):   # calls in a row
+    for n, (seed, prune) in enumerate(seeds):
         x, cu, ids, w, kw = _inputs(cfg, seed, prune)
+        assert P.dora_workspace_size(t, cfg.batch, w) <= P.NOALLOC_SCRATCH_BYTES
         ref = _outputs(t, cfg.batch, cfg.dim)
         ws = P.alloc_workspace(t, cfg.batch, w)
         P.dora_pruned_block(x, cu, w, cfg.n_tokens, ref["x_out"], ws, ids_in=ids,
@@ -68,6 +72,7 @@ def test_noalloc_matches_workspace_entry_on_consecutive_calls():
                                     kept_idx=got["kept_idx"], status=status, **kw)
         torch.cuda.synchronize()
         assert int(status.item()) == 0
+        assert P.dora_read_status(P.dora_workspace_status(ws)) == 0
         if prune:
             t_out = int(ref["cu_out"][-1].item())
             assert torch.equal(got["cu_out"], ref["cu_out"])
@@ -75,8 +80,30 @@ def test_noalloc_matches_workspace_entry_on_consecutive_calls():
             assert torch.equal(got["ids_out"][:t_out], ref["ids_out"][:t_out])
         else:
             t_out = t
-        assert_close(got["x_out"][:t_out].float().cpu().numpy(),
-                     ref["x_out"][:t_out].float().cpu().numpy(), f"noalloc seed {seed}")
+        assert torch.equal(got["x_out"][:t_out], ref["x_out"][:t_out]), f"seed {seed}"
+        if n == 0:
+            cu_h, ids_h = S.initial_layout(cfg)
+            wb = S.block_weights(cfg, 0, seed, random_affine=True)
+            sc = kp = None
+            if prune:
+                keeps, _ = S.keep_schedule(cfg, seed)
+                sc = O.gather_scores(S.score_table(cfg, 0, seed), cu_h, ids_h)
+                kp = keeps[0]
+            o = O.pruned_block(O.bf16_to_f64(S.activations_bf16(cfg, seed)), cu_h, ids_h,
+                               O.decode_weights(wb), cfg.heads, cfg.ln_eps, sc, kp)
+            assert np.array_equal(got["cu_out"].cpu().numpy(), o["cu_out"])
+            assert_close(got["x_out"][:t_out].float().cpu().numpy(), o["x_out"],
+                         f"noalloc vs oracle, seed {seed}")
+
+
+def test_noalloc_matches_workspace_entry_on_consecutive_calls():
+    # DeiT-Tiny shape, 8 x 197 tokens, D = 192: about 7 MB of scratch
+    _check_consecutive_calls(S.get_config("cfg1"), ((31, True), (32, True), (33, False)))
+
+
+def test_noalloc_matches_workspace_entry_deit_small_sub_batch():
+    # DeiT-Small shape, 16 of its 64 images (3152 rows, D = 384): about 26 MB
+    _check_consecutive_calls(S.get_config("cfg2", batch=16), ((41, True), (42, True)))
 
 
 def test_noalloc_rejects_blocks_larger_than_its_scratch():
