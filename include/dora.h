@@ -118,6 +118,31 @@ int dora_compact(const dora_bf16* x, int32_t dim, const int32_t* kept_idx, const
                  int32_t* ids_out, int32_t* status, dora_stream_t stream);
 
 /*
+ * dora_select_compact -- dora_select_keep and the compaction of the kept
+ * rows in one launch (Sec. 3.2 "Sampling and deployment" and Appendix A.3
+ * for the kept set; Sec. 3.1 pruning operator and Sec. 3.5 "Inference" for
+ * the packed buffer).
+ *
+ * Arguments as dora_select_keep, plus:
+ * x          bf16 [t_in_cap, dim] rows to gather from (16-byte aligned;
+ *            dim % 8 == 0, dim <= 2048).
+ * ids_in     nullable int32 [t_in_cap]; ids_out nullable out int32 (given
+ *            together): ids_out[r] = ids_in[kept_idx[r]].
+ * mv_in      nullable fp32 [t_in_cap, 2]; mv_out nullable out (given
+ *            together, 8-byte aligned): mv_out[r] = mv_in[kept_idx[r]].
+ * packed     out bf16 [capacity >= t_in_cap, dim]: packed[r] =
+ *            x[kept_idx[r]], bit for bit.
+ * kept_idx, cu_out and status are written exactly as dora_select_keep
+ * writes them, except that an image whose rows do not lie inside
+ * [0, t_in_cap) keeps nothing and raises DORA_ERR_DEVICE_SEQLEN.
+ */
+int dora_select_compact(const float* scores, const int32_t* cu_in, const int32_t* keep_counts,
+                        int32_t batch, int32_t max_seqlen, const dora_bf16* x, int32_t dim,
+                        int32_t t_in_cap, const int32_t* ids_in, const float* mv_in,
+                        int32_t* kept_idx, int32_t* cu_out, dora_bf16* packed,
+                        int32_t* ids_out, float* mv_out, int32_t* status, dora_stream_t stream);
+
+/*
  * dora_compact_ln -- dora_compact fused with the LayerNorm' that follows the
  * deletion in Eq. 1: also writes ln_out[r] = LayerNorm(packed[r]) with affine
  * ln_w, ln_b (bf16 [dim]) and epsilon eps (biased variance, fp32 statistics).

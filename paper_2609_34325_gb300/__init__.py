@@ -16,7 +16,7 @@ import torch
 __all__ = [
     "DoraError", "load_library", "library_path", "EPI_BIAS", "EPI_BIAS_GELU",
     "EPI_BIAS_RESIDUAL", "EXPORTED_SYMBOLS", "dora_status_string", "dora_version",
-    "dora_select_keep", "dora_compact", "dora_compact_ln", "dora_layernorm", "dora_linear",
+    "dora_select_keep", "dora_select_compact", "dora_compact", "dora_compact_ln", "dora_layernorm", "dora_linear",
     "dora_varlen_attn", "dora_gather_scores", "BlockWeights", "dora_workspace_size",
     "dora_pruned_block", "dora_workspace_status", "dora_read_status", "alloc_workspace",
     "dora_pruned_block_noalloc", "NOALLOC_SCRATCH_BYTES", "dora_row_stats",
@@ -40,6 +40,8 @@ _SIGS = {
     "dora_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "dora_version": (ctypes.c_int, []),
     "dora_select_keep": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp]),
+    "dora_select_compact": (ctypes.c_int, [_vp, _vp, _vp, _i32, _i32, _vp, _i32, _i32, _vp, _vp,
+                                           _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
     "dora_compact": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _vp, _vp]),
     "dora_compact_ln": (ctypes.c_int, [_vp, _i32, _vp, _vp, _i32, _i32, _vp, _vp, _vp, _f32,
                                        _vp, _vp, _vp, _vp, _vp]),
@@ -181,6 +183,36 @@ def dora_select_keep(scores, cu_in, keep_counts, max_seqlen, kept_idx, cu_out, s
     _check(load_library().dora_select_keep(_ptr(scores), _ptr(cu_in), _ptr(keep_counts), batch,
                                            int(max_seqlen), _ptr(kept_idx), _ptr(cu_out),
                                            _ptr(status), _stream(stream)), "dora_select_keep")
+
+
+def dora_select_compact(scores, cu_in, keep_counts, max_seqlen, x, kept_idx, cu_out, packed,
+                        ids_in=None, ids_out=None, mv_in=None, mv_out=None, status=None,
+                        stream=None):
+    """dora_select_keep and the compaction of the kept rows in one launch:
+    kept_idx and cu_out as dora_select_keep writes them, packed[r] =
+    x[kept_idx[r]], and (when given) ids_out[r] = ids_in[kept_idx[r]],
+    mv_out[r] = mv_in[kept_idx[r]]."""
+    _req(scores, torch.float32, "scores")
+    _req(x, torch.bfloat16, "x")
+    _req(packed, torch.bfloat16, "packed")
+    for n, t in (("cu_in", cu_in), ("keep_counts", keep_counts), ("kept_idx", kept_idx),
+                 ("cu_out", cu_out)):
+        _req(t, torch.int32, n)
+    for n, t in (("ids_in", ids_in), ("ids_out", ids_out), ("status", status)):
+        _req(t, torch.int32, n, optional=True)
+    _req(mv_in, torch.float32, "mv_in", optional=True)
+    _req(mv_out, torch.float32, "mv_out", optional=True)
+    t_in_cap, dim = x.shape
+    if packed.shape[0] < t_in_cap or packed.shape[1] != dim:
+        raise ValueError("packed must hold at least as many rows as x")
+    for n, t in (("mv_in", mv_in), ("mv_out", mv_out)):
+        if t is not None and t.numel() < t_in_cap * 2:
+            raise ValueError(f"{n} must hold [t_in_cap, 2] floats")
+    _check(load_library().dora_select_compact(
+        _ptr(scores), _ptr(cu_in), _ptr(keep_counts), cu_in.numel() - 1, int(max_seqlen),
+        _ptr(x), dim, t_in_cap, _ptr(ids_in), _ptr(mv_in), _ptr(kept_idx), _ptr(cu_out),
+        _ptr(packed), _ptr(ids_out), _ptr(mv_out), _ptr(status), _stream(stream)),
+        "dora_select_compact")
 
 
 def dora_compact(x, kept_idx, cu_out, packed, ids_in=None, ids_out=None, status=None,

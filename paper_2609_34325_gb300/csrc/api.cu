@@ -136,6 +136,28 @@ int dora_select_keep(const float* scores, const int32_t* cu_in, const int32_t* k
                                         cu_out, status, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+int dora_select_compact(const float* scores, const int32_t* cu_in, const int32_t* keep_counts,
+                        int32_t batch, int32_t max_seqlen, const dora_bf16* x, int32_t dim,
+                        int32_t t_in_cap, const int32_t* ids_in, const float* mv_in,
+                        int32_t* kept_idx, int32_t* cu_out, dora_bf16* packed,
+                        int32_t* ids_out, float* mv_out, int32_t* status, dora_stream_t stream) {
+  DORA_CHECK_ARG(batch >= 0 && batch <= (1 << 24) && t_in_cap >= 0);
+  DORA_CHECK_ARG(max_seqlen >= 0 && max_seqlen <= kMaxSeqlenSelect);
+  DORA_CHECK_ARG(cu_in && keep_counts && cu_out);
+  DORA_CHECK_ARG(batch == 0 || (scores && kept_idx));
+  DORA_CHECK_ARG(dim > 0 && dim % 8 == 0 && dim <= kMaxDimRow);
+  DORA_CHECK_ARG(t_in_cap == 0 || (x && packed));
+  DORA_CHECK_ARG(aligned16(x) && aligned16(packed));
+  DORA_CHECK_ARG((ids_in == nullptr) == (ids_out == nullptr));
+  DORA_CHECK_ARG((mv_in == nullptr) == (mv_out == nullptr));
+  DORA_CHECK_ARG(aligned8(mv_in) && aligned8(mv_out));
+  DORA_CHECK_DEVICE();
+  return cuda_status(launch_select_compact(scores, cu_in, keep_counts, batch, max_seqlen,
+                                           x, dim, t_in_cap, ids_in, mv_in, kept_idx, cu_out,
+                                           packed, ids_out, mv_out, status,
+                                           reinterpret_cast<cudaStream_t>(stream)));
+}
+
 static int compact_common(const dora_bf16* x, int32_t dim, const int32_t* kept_idx,
                           const int32_t* cu_out, int32_t batch, int32_t t_in_cap,
                           const int32_t* ids_in, const dora_bf16* ln_w, const dora_bf16* ln_b,
@@ -522,11 +544,9 @@ static int pruned_block_impl(const dora_bf16* x_in, const int32_t* cu_in, const 
   const uint16_t* hk = hattn;
   const int32_t* rows_mid = rows_in;
   if (scores) {
-    if (launch_select_keep(scores, cu_in, keep_counts, batch, max_seqlen, kept, cu_out, status,
-                           stream) != cudaSuccess)
-      return DORA_ERR_CUDA;
-    if (launch_compact(hattn, d, kept, cu_out, batch, t_cap, ids_in, nullptr, nullptr, 0.f, hkeep,
-                       ids_out, nullptr, mv, mv2, status, stream) != cudaSuccess)
+    if (launch_select_compact(scores, cu_in, keep_counts, batch, max_seqlen, hattn, d, t_cap,
+                              ids_in, mv, kept, cu_out, hkeep, ids_out, mv2, status,
+                              stream) != cudaSuccess)
       return DORA_ERR_CUDA;
     hk = hkeep;
     rows_mid = cu_out + batch;

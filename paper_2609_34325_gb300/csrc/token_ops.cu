@@ -84,40 +84,85 @@ __device__ __forceinline__ uint32_t score_key(float s) {
 }
 
 // Tokens image i keeps after clamping; every CTA evaluates it identically.
-__device__ __forceinline__ int clamped_keep(int n, int m, int max_seqlen) {
-  if (n > max_seqlen || n <= 0) return 0;
+// An image whose rows do not lie inside [0, t_cap) keeps nothing.
+__device__ __forceinline__ int clamped_keep(int lo, int n, int m, int max_seqlen, int t_cap) {
+  if (n > max_seqlen || n <= 0 || lo < 0 || lo > t_cap - n) return 0;
   return m < 1 ? 1 : (m > n ? n : m);
 }
 
 // ---------------------------------------------------------------------------
-// K1: per-image deterministic top-k deletion
+// K1: per-image deterministic top-k deletion, optionally fused with the
+// compaction of the kept rows
 // ---------------------------------------------------------------------------
-// One CTA per image.  Each visual candidate j counts how many candidates
-// precede it in the order (score key, index); it is kept when that rank is
-// below m - 1.  Kept flags are then scanned to write ascending indices.
+// Work of one CTA (kSelectThreads threads) for image i = blockIdx.x / splits:
+//  1. its output offset, the sum of the clamped keep counts of images < i;
+//  2. the image's candidate keys (ordered uint32 of the deletion scores) in
+//     shared memory;
+//  3. radix select, 8 bits a pass from the top: the key T of the
+//     (m-1)-th smallest candidate and how many candidates equal to T are
+//     kept (the lowest-indexed ones: ties are broken by index);
+//  4. one block-wide scan over contiguous index segments of the packed
+//     counts (candidates below T, candidates equal to T), which gives every
+//     kept token its output position in index order;
+//  5. the kept list in shared memory (and, by the image's first CTA, in
+//     kept_idx and cu_out).
+// With CPL > 0, the `splits` CTAs of the image then copy its kept rows
+// (16-byte vector loads and stores, one warp per row, two rows in flight a
+// warp), their ids and their row moments: every CTA selects (the scores are
+// read from L2 after the first), and the row copies are spread over all of
+// them.  Selection and compaction are one launch, and no kept_idx round trip
+// through global memory stands between them.  CPL is the number of 16-byte
+// chunks of a row per lane (registers sized to the row); 0 = selection only.
+constexpr int kRadixBins = 256;
+static_assert(kSelectThreads == kRadixBins, "one histogram bin per thread");
+
+template <int CPL>
 __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
     const float* __restrict__ scores, const int32_t* __restrict__ cu_in,
-    const int32_t* __restrict__ keep_counts, int32_t batch, int32_t max_seqlen,
-    int32_t* __restrict__ kept_idx, int32_t* __restrict__ cu_out, int32_t* status) {
+    const int32_t* __restrict__ keep_counts, int32_t batch, int32_t max_seqlen, int32_t t_cap,
+    int32_t splits, int32_t* __restrict__ kept_idx, int32_t* __restrict__ cu_out,
+    const uint4* __restrict__ x, int32_t chunks, const int32_t* __restrict__ ids_in,
+    const float2* __restrict__ mv_in, uint4* __restrict__ packed, int32_t* __restrict__ ids_out,
+    float2* __restrict__ mv_out, int32_t* status) {
   pdl_trigger();
   pdl_wait();
-  extern __shared__ uint32_t keys[];            // [max_seqlen]
+  extern __shared__ uint32_t keys[];            // [max_seqlen] keys, then [max_seqlen] kept rows
+  int32_t* kept_rows = reinterpret_cast<int32_t*>(keys + max_seqlen);
   __shared__ int scratch[33];
-  const int i = blockIdx.x;
+  __shared__ int hist[kRadixBins];
+  __shared__ uint32_t sel_prefix;
+  __shared__ int sel_rank;
+  const int i = blockIdx.x / splits;
+  const int part = blockIdx.x - i * splits;
   const int tid = threadIdx.x;
+  const int lane = tid & 31;
+  // rows of the input (and capacity of the outputs): t_cap, or cu_in[batch]
+  // when the caller gives none
+  const int cap = t_cap >= 0 ? t_cap : cu_in[batch];
 
-  // output offset of this image: sum of the clamped keep counts before it
-  int part = 0;
-  for (int t = tid; t < i; t += blockDim.x)
-    part += clamped_keep(cu_in[t + 1] - cu_in[t], keep_counts[t], max_seqlen);
-  const int off = block_sum(part, scratch);
-
-  const int lo = cu_in[i];
-  const int n = cu_in[i + 1] - lo;
-  const int m = keep_counts[i];
-  const int me = clamped_keep(n, m, max_seqlen);
-  if (tid == 0) {
-    if (n > max_seqlen) record_status(status, DORA_ERR_DEVICE_SEQLEN);
+  // 1. output offset of this image; the image's own bounds and keep count
+  // come in the same round of loads (the thread that reads entry i shares them)
+  __shared__ int own[3];
+  int acc = 0;
+  for (int t = tid; t <= i; t += blockDim.x) {
+    const int l0 = cu_in[t], l1 = cu_in[t + 1], kt = keep_counts[t];
+    if (t < i) {
+      acc += clamped_keep(l0, l1 - l0, kt, max_seqlen, cap);
+    } else {
+      own[0] = l0;
+      own[1] = l1 - l0;
+      own[2] = kt;
+    }
+  }
+  const int off = block_sum(acc, scratch);   // its barriers publish own[]
+  const int lo = own[0];
+  const int n = own[1];
+  const int m = own[2];
+  const int me = clamped_keep(lo, n, m, max_seqlen, cap);
+  if (part == 0 && tid == 0) {
+    // rows outside the input, or (boundaries not increasing) outputs past it
+    if (n > max_seqlen || (n > 0 && (lo < 0 || lo > cap - n)) || off > cap - me)
+      record_status(status, DORA_ERR_DEVICE_SEQLEN);
     else if (n < 0 || (n > 0 && me != m) || (n == 0 && m != 0))
       record_status(status, DORA_ERR_DEVICE_BAD_COUNT);
     cu_out[i + 1] = off + me;
@@ -125,39 +170,126 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
   }
   if (me == 0) return;
 
+  // 2. candidate keys
   for (int j = tid; j < n; j += blockDim.x) keys[j] = score_key(scores[lo + j]);
   __syncthreads();
 
-  // Each thread owns a contiguous segment of candidate indices so that the
-  // flag scan below preserves index order.
+  // 3. threshold key T and the number of candidates equal to T that are kept
+  const int need = me - 1;                       // visual tokens kept
+  uint32_t thr;
+  int ties_keep;
+  if (need == 0) {
+    thr = 0u;                                    // no candidate is below key 0 ...
+    ties_keep = 0;                               // ... and none equal to it is kept
+  } else if (need == n - 1) {
+    thr = 0xFFFFFFFFu;                           // every candidate is kept
+    ties_keep = n;
+  } else {
+    uint32_t prefix = 0u, hi_mask = 0u;
+    int rank = need;                             // 1-based rank among the remaining
+#pragma unroll 1
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      hist[tid] = 0;
+      __syncthreads();
+      // warp-uniform trip count: every lane reaches the match below
+      for (int base = 0; base < n; base += blockDim.x) {
+        const int j = base + tid;
+        const uint32_t k = (j >= 1 && j < n) ? keys[j] : 0u;
+        const bool in = j >= 1 && j < n && ((k ^ prefix) & hi_mask) == 0u;
+        const uint32_t digit = in ? ((k >> shift) & 0xFFu) : 0x100u;
+        const uint32_t peers = __match_any_sync(0xffffffffu, digit);
+        if (in && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], __popc(peers));
+      }
+      __syncthreads();
+      const int c = hist[tid];
+      const int below = block_exclusive_scan(c, scratch);
+      if (below < rank && rank <= below + c) {
+        sel_prefix = prefix | (static_cast<uint32_t>(tid) << shift);
+        sel_rank = rank - below;
+      }
+      __syncthreads();
+      prefix = sel_prefix;
+      rank = sel_rank;
+      hi_mask |= 0xFFu << shift;
+    }
+    thr = prefix;
+    ties_keep = rank;
+  }
+
+  // 4. output positions: each thread owns a contiguous segment of indices;
+  // CLS (index 0) counts as a token below the threshold
   const int per = (n + blockDim.x - 1) / blockDim.x;
   const int j0 = tid * per;
   const int j1 = min(n, j0 + per);
-  uint32_t keepmask = 0;     // bit q set when index j0 + q is kept (per <= 32)
-  int cnt = 0;
-  const int need = me - 1;   // visual tokens to keep
+  int below = 0, equal = 0;
   for (int j = j0; j < j1; ++j) {
-    bool kept;
     if (j == 0) {
-      kept = true;           // CLS
+      ++below;
     } else {
-      const uint32_t kj = keys[j];
-      int rank = 0;
-      for (int t = 1; t < n; ++t) {
-        const uint32_t kt = keys[t];
-        rank += (kt < kj) | ((kt == kj) & (t < j));
-      }
-      kept = rank < need;
-    }
-    if (kept) {
-      keepmask |= 1u << (j - j0);
-      ++cnt;
+      const uint32_t k = keys[j];
+      below += k < thr;
+      equal += k == thr;
     }
   }
-  const int pos = block_exclusive_scan(cnt, scratch);
-  int w = off + pos;
-  for (int j = j0; j < j1; ++j)
-    if (keepmask & (1u << (j - j0))) kept_idx[w++] = lo + j;
+  const int pre = block_exclusive_scan((equal << 16) | below, scratch);   // both < 2^16
+  int ties_before = pre >> 16;
+  int pos = (pre & 0xFFFF) + min(ties_before, ties_keep);
+  // 5. the kept list
+  for (int j = j0; j < j1; ++j) {
+    bool kept = j == 0;
+    if (!kept) {
+      const uint32_t k = keys[j];
+      if (k == thr) kept = ties_before++ < ties_keep;
+      else kept = k < thr;
+    }
+    if (kept) {
+      if (part == 0 && off + pos < cap) kept_idx[off + pos] = lo + j;
+      if constexpr (CPL > 0) kept_rows[pos] = lo + j;
+      ++pos;
+    }
+  }
+  if constexpr (CPL > 0) {
+    __syncthreads();
+    // rows r = part * 8 + warp, + splits * 8, ... of this image: two per pass
+    const int warps = blockDim.x >> 5;
+    const int stride = splits * warps;
+    const int rows = min(me, cap - off);        // outputs past the capacity are dropped
+    int r = part * warps + (tid >> 5);
+    for (; r < rows; r += 2 * stride) {
+      const int r2 = r + stride;
+      const bool two = r2 < rows;
+      const int s1 = kept_rows[r];
+      const int s2 = two ? kept_rows[r2] : s1;
+      const uint4* src1 = x + static_cast<size_t>(s1) * chunks;
+      const uint4* src2 = x + static_cast<size_t>(s2) * chunks;
+      uint4 v1[CPL], v2[CPL];
+#pragma unroll
+      for (int q = 0; q < CPL; ++q) {
+        const int c = lane + 32 * q;
+        if (c < chunks) {
+          v1[q] = __ldg(src1 + c);
+          if (two) v2[q] = __ldg(src2 + c);
+        }
+      }
+      uint4* dst1 = packed + static_cast<size_t>(off + r) * chunks;
+      uint4* dst2 = packed + static_cast<size_t>(off + r2) * chunks;
+#pragma unroll
+      for (int q = 0; q < CPL; ++q) {
+        const int c = lane + 32 * q;
+        if (c < chunks) {
+          dst1[c] = v1[q];
+          if (two) dst2[c] = v2[q];
+        }
+      }
+      if (lane == 0) {
+        if (ids_out != nullptr) ids_out[off + r] = ids_in[s1];
+        if (mv_out != nullptr) mv_out[off + r] = mv_in[s1];
+      } else if (lane == 1 && two) {
+        if (ids_out != nullptr) ids_out[off + r2] = ids_in[s2];
+        if (mv_out != nullptr) mv_out[off + r2] = mv_in[s2];
+      }
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -537,20 +669,92 @@ static int row_grid(int64_t rows) {
   return static_cast<int>(g);
 }
 
+// Shared memory of the selection: keys and the kept list, [max_seqlen] each.
+static cudaError_t select_smem(const void* kern, int32_t max_seqlen, size_t* smem) {
+  *smem = static_cast<size_t>(max_seqlen) * 2 * sizeof(uint32_t);
+  if (*smem > 48 * 1024)
+    return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(*smem));
+  return cudaSuccess;
+}
+
 cudaError_t launch_select_keep(const float* scores, const int32_t* cu_in,
                                const int32_t* keep_counts, int32_t batch, int32_t max_seqlen,
                                int32_t* kept_idx, int32_t* cu_out, int32_t* status,
                                cudaStream_t stream) {
   if (batch == 0) return cudaSuccess;
-  const size_t smem = static_cast<size_t>(max_seqlen) * sizeof(uint32_t);
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(select_keep_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
-    if (e != cudaSuccess) return e;
+  size_t smem = 0;
+  cudaError_t e = select_smem(reinterpret_cast<const void*>(select_keep_kernel<0>),
+                              max_seqlen, &smem);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(select_keep_kernel<0>, dim3(batch), dim3(kSelectThreads), smem, stream,
+                    scores, cu_in, keep_counts, batch, max_seqlen, -1, 1, kept_idx,
+                    cu_out, static_cast<const uint4*>(nullptr), 0,
+                    static_cast<const int32_t*>(nullptr), static_cast<const float2*>(nullptr),
+                    static_cast<uint4*>(nullptr), static_cast<int32_t*>(nullptr),
+                    static_cast<float2*>(nullptr), status);
+}
+
+// CTAs per image of the fused kernel: about kSelectCtas CTAs in all (a
+// measured sweep at 256 x 197, 64 x 577 and 1024 x 197 tokens put the best
+// split near 512 CTAs), at most kSelectMaxSplits, and no more than one per
+// 16 tokens of the longest image.
+int select_compact_splits(int32_t batch, int32_t max_seqlen) {
+  if (batch <= 0) return 1;
+  int s = (kSelectCtas + batch - 1) / batch;
+  const int by_rows = (max_seqlen + 15) / 16;
+  if (s > by_rows) s = by_rows;
+  return s < 1 ? 1 : (s > kSelectMaxSplits ? kSelectMaxSplits : s);
+}
+
+template <int CPL>
+static cudaError_t select_compact_cpl(const float* scores, const int32_t* cu_in,
+                                      const int32_t* keep_counts, int32_t batch,
+                                      int32_t max_seqlen, const uint16_t* x, int32_t chunks,
+                                      int32_t t_in_cap, const int32_t* ids_in,
+                                      const float* mv_in, int32_t* kept_idx, int32_t* cu_out,
+                                      uint16_t* packed, int32_t* ids_out, float* mv_out,
+                                      int32_t* status, cudaStream_t stream) {
+  size_t smem = 0;
+  cudaError_t e = select_smem(reinterpret_cast<const void*>(select_keep_kernel<CPL>),
+                              max_seqlen, &smem);
+  if (e != cudaSuccess) return e;
+  const int splits = select_compact_splits(batch, max_seqlen);
+  const long long grid = static_cast<long long>(batch) * splits;
+  if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
+  return launch_pdl(select_keep_kernel<CPL>, dim3(static_cast<unsigned>(grid)),
+                    dim3(kSelectThreads), smem, stream, scores, cu_in, keep_counts, batch,
+                    max_seqlen, t_in_cap, splits, kept_idx, cu_out,
+                    reinterpret_cast<const uint4*>(x), chunks, ids_in,
+                    reinterpret_cast<const float2*>(mv_in), reinterpret_cast<uint4*>(packed),
+                    ids_out, reinterpret_cast<float2*>(mv_out), status);
+}
+
+cudaError_t launch_select_compact(const float* scores, const int32_t* cu_in,
+                                  const int32_t* keep_counts, int32_t batch, int32_t max_seqlen,
+                                  const uint16_t* x, int32_t dim, int32_t t_in_cap,
+                                  const int32_t* ids_in, const float* mv_in, int32_t* kept_idx,
+                                  int32_t* cu_out, uint16_t* packed, int32_t* ids_out,
+                                  float* mv_out, int32_t* status, cudaStream_t stream) {
+  if (batch == 0) return cudaSuccess;
+  const int chunks = dim / 8;
+  switch ((chunks + 31) / 32) {
+    case 1: return select_compact_cpl<1>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
+                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         mv_out, status, stream);
+    case 2: return select_compact_cpl<2>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
+                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         mv_out, status, stream);
+    case 3: return select_compact_cpl<3>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
+                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         mv_out, status, stream);
+    case 4: return select_compact_cpl<4>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
+                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         mv_out, status, stream);
+    default: return select_compact_cpl<kMaxChunksPerLane>(
+        scores, cu_in, keep_counts, batch, max_seqlen, x, chunks, t_in_cap, ids_in, mv_in,
+        kept_idx, cu_out, packed, ids_out, mv_out, status, stream);
   }
-  return launch_pdl(select_keep_kernel, dim3(batch), dim3(kSelectThreads), smem, stream, scores,
-                    cu_in, keep_counts, batch, max_seqlen, kept_idx, cu_out, status);
 }
 
 cudaError_t launch_compact(const uint16_t* x, int32_t dim, const int32_t* kept_idx,

@@ -33,12 +33,27 @@ constexpr int kSelectThreads = 256;
 constexpr int kRowThreads = 256;          // 8 rows per CTA, one warp per row
 constexpr int kMaxChunksPerLane = 8;      // 16-byte chunks per lane: dim <= 2048
 constexpr int kMaxDimRow = 32 * 8 * kMaxChunksPerLane;
-constexpr int kMaxSeqlenSelect = 32 * kSelectThreads;   // one 32-bit mask per thread
+// selection: keys and kept list of one image in shared memory (64 KB at the
+// limit); the per-thread segment counts are packed into 16-bit halves
+constexpr int kMaxSeqlenSelect = 32 * kSelectThreads;
+constexpr int kSelectCtas = 512;          // fused compaction: CTAs in all, split over the images
+constexpr int kSelectMaxSplits = 8;
 
 cudaError_t launch_select_keep(const float* scores, const int32_t* cu_in,
                                const int32_t* keep_counts, int32_t batch, int32_t max_seqlen,
                                int32_t* kept_idx, int32_t* cu_out, int32_t* status,
                                cudaStream_t stream);
+
+// Selection fused with the compaction of the kept rows (ids_in/ids_out and
+// mv_in/mv_out nullable in pairs): the same kept_idx and cu_out as
+// launch_select_keep, then packed[r] = x[kept_idx[r]], ids and row moments.
+int select_compact_splits(int32_t batch, int32_t max_seqlen);
+cudaError_t launch_select_compact(const float* scores, const int32_t* cu_in,
+                                  const int32_t* keep_counts, int32_t batch, int32_t max_seqlen,
+                                  const uint16_t* x, int32_t dim, int32_t t_in_cap,
+                                  const int32_t* ids_in, const float* mv_in, int32_t* kept_idx,
+                                  int32_t* cu_out, uint16_t* packed, int32_t* ids_out,
+                                  float* mv_out, int32_t* status, cudaStream_t stream);
 
 // ln_out (LayerNorm' of the kept rows) is nullable; so is mv_out, which
 // receives mv_in[kept_idx[r]] (row moments, below) for every packed row r.

@@ -56,6 +56,15 @@ def test_host_validation_without_gpu(lib):
     assert lib.dora_linear(16, 128, None, 128, 16, 128, None, None, 2, 16, None, None) == 1
     assert lib.dora_linear(16, 128, None, 128, 16, 128, None, None, 7, 16, None, None) == 1
     assert lib.dora_compact(16, 12, 16, 16, 1, 10, None, 16, None, None, None) == 1
+    # dora_select_compact: dim % 8, ids given without ids_out, mv_out misaligned
+    assert lib.dora_select_compact(16, 16, 16, 1, 197, 16, 12, 197, None, None, 16, 16, 16,
+                                   None, None, None, None) == 1
+    assert lib.dora_select_compact(16, 16, 16, 1, 197, 16, 64, 197, 16, None, 16, 16, 16,
+                                   None, None, None, None) == 1
+    assert lib.dora_select_compact(16, 16, 16, 1, 197, 16, 64, 197, None, 16, 16, 16, 16,
+                                   None, 12, None, None) == 1
+    assert lib.dora_select_compact(16, 16, 16, 1, 1 << 20, 16, 64, 197, None, None, 16, 16, 16,
+                                   None, None, None, None) == 1
     assert lib.dora_layernorm(16, 4, None, 4096, 16, 16, 1e-6, 16, None) == 1
     assert lib.dora_gather_scores(16, 0, 16, 16, 1, 16, None, None) == 1
     assert lib.dora_read_status(None, None) == 1

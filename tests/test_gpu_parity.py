@@ -197,6 +197,184 @@ def test_compact_empty_output():
 
 
 # ---------------------------------------------------------------------------
+# selection fused with the compaction (one launch)
+# ---------------------------------------------------------------------------
+
+def _run_select_compact(scores, cu, keeps, max_seqlen, x, ids=None, mv=None, t_cap=None,
+                        extra=0):
+    """dora_select_compact with sentinel-filled outputs of t_cap + extra rows."""
+    t_cap = int(cu[-1]) if t_cap is None else t_cap
+    b = len(cu) - 1
+    dim = x.shape[1]
+    rows = max(t_cap + extra, 1)
+    kept = torch.full((rows,), SENT, dtype=torch.int32, device=dev())
+    cu_out = torch.full((b + 1,), SENT, dtype=torch.int32, device=dev())
+    packed = torch.zeros(rows, dim, dtype=torch.bfloat16, device=dev())
+    packed.view(torch.int16).fill_(SENT)
+    ids_out = mv_out = None
+    if ids is not None:
+        ids_out = torch.full((rows,), SENT, dtype=torch.int32, device=dev())
+    if mv is not None:
+        mv_out = torch.full((rows, 2), float(SENT), dtype=torch.float32, device=dev())
+    st = _status()
+    xd = bf(x[:t_cap]) if t_cap > 0 else torch.zeros(0, dim, dtype=torch.bfloat16, device=dev())
+    P.dora_select_compact(f32(scores), i32(cu), i32(keeps), max_seqlen, xd, kept, cu_out, packed,
+                          ids_in=None if ids is None else i32(ids[:t_cap]), ids_out=ids_out,
+                          mv_in=None if mv is None else f32(mv[:t_cap]), mv_out=mv_out, status=st)
+    torch.cuda.synchronize()
+    return dict(kept=kept.cpu().numpy(), cu=cu_out.cpu().numpy(), packed=bits(packed),
+                ids=None if ids_out is None else ids_out.cpu().numpy(),
+                mv=None if mv_out is None else mv_out.cpu().numpy(), status=int(st.item()))
+
+
+def _check_select_compact(scores, cu, keeps, x, ids=None, mv=None, max_seqlen=None):
+    lens = np.diff(cu)
+    ms = int(lens.max()) if max_seqlen is None else max_seqlen
+    g = _run_select_compact(scores, cu, keeps, ms, x, ids, mv)
+    rk, rcu, rst = O.select_keep(scores, cu, keeps)
+    t_out = int(rcu[-1])
+    assert np.array_equal(g["cu"], rcu)
+    assert np.array_equal(g["kept"][:t_out], rk)
+    assert np.all(g["kept"][t_out:] == SENT)
+    assert g["status"] == rst
+    ref_packed, ref_ids = O.compact(x, rk, ids if ids is not None else np.zeros(len(x), np.int32))
+    assert np.array_equal(g["packed"][:t_out], ref_packed)
+    assert np.all(g["packed"][t_out:].view(np.int16) == SENT)
+    if ids is not None:
+        assert np.array_equal(g["ids"][:t_out], ref_ids)
+        assert np.all(g["ids"][t_out:] == SENT)
+    if mv is not None:
+        assert np.array_equal(g["mv"][:t_out].view(np.uint32), mv[rk].view(np.uint32))
+        assert np.all(g["mv"][t_out:] == SENT)
+    return t_out
+
+
+def _row_inputs(rng, t, dim):
+    x = rng.integers(0, 65536, size=(t, dim), dtype=np.uint16)      # any bit pattern
+    ids = rng.integers(0, 1 << 20, size=t).astype(np.int32)
+    mv = rng.standard_normal((t, 2)).astype(np.float32)
+    return x, ids, mv
+
+
+@pytest.mark.parametrize("name", CFGS)
+def test_select_compact_configs(name):
+    """Kept rows, ids, row moments, kept_idx and boundaries of one launch,
+    bit for bit against the oracle's selection and compaction, on the first
+    two pruning steps of every workload."""
+    cfg = S.get_config(name)
+    cu, ids = S.initial_layout(cfg)
+    keeps, _ = S.keep_schedule(cfg, 3)
+    rng = np.random.default_rng(30)
+    lcu, lids = cu, ids
+    for j, blk in enumerate(cfg.prune_blocks[:2]):
+        scores = O.gather_scores(S.score_table(cfg, blk, 3), lcu, lids)
+        x, _, mv = _row_inputs(rng, int(lcu[-1]), cfg.dim)
+        _check_select_compact(scores, lcu, keeps[j], x, lids, mv, cfg.n_tokens)
+        rk, rcu, _ = O.select_keep(scores, lcu, keeps[j])
+        lcu, lids = rcu, lids[rk]
+
+
+@pytest.mark.parametrize("dim", [64, 192, 384, 768, 1024, 2048])
+@pytest.mark.parametrize("kind", ["uniform", "ties", "special", "allequal"])
+def test_select_compact_edges(kind, dim):
+    """Lengths 1..577 around the 16/32/128/256 boundaries, ties, signed
+    zeros, NaN and infinities, keep one / all / random, every row width class
+    (1 to 8 16-byte chunks a lane); ids and moments given or not."""
+    rng = np.random.default_rng(43)
+    lens = _edge_lengths()
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    if kind == "uniform":
+        s = rng.random(t).astype(np.float32)
+    elif kind == "ties":
+        s = rng.choice(np.array([0.0, 0.25, 0.5], np.float32), size=t)
+    elif kind == "allequal":
+        s = np.full(t, 0.125, np.float32)
+    else:
+        pal = np.array([0.0, -0.0, np.nan, -np.nan, np.inf, -np.inf, 1.0, -1.0, 1e-38, -1e-38],
+                       dtype=np.float32)
+        s = rng.choice(pal, size=t)
+    x, ids, mv = _row_inputs(rng, t, dim)
+    for n, mode in enumerate(("one", "all", "random")):
+        if mode == "one":
+            keeps = np.ones_like(lens)
+        elif mode == "all":
+            keeps = lens.copy()
+        else:
+            keeps = np.array([rng.integers(1, k + 1) for k in lens])
+        with_side = n != 1
+        _check_select_compact(s, cu, keeps, x, ids if with_side else None,
+                              mv if with_side else None)
+
+
+def test_select_compact_bad_counts_and_max_seqlen():
+    rng = np.random.default_rng(44)
+    lens = np.array([5, 0, 9, 3, 12])
+    cu = O.cu_from_counts(lens)
+    s = rng.random(int(cu[-1])).astype(np.float32)
+    x, ids, mv = _row_inputs(rng, int(cu[-1]), 192)
+    keeps = np.array([0, 0, 20, 3, -4])
+    _check_select_compact(s, cu, keeps, x, ids, mv)
+    lens = np.array([10, 40, 10])
+    cu = O.cu_from_counts(lens)
+    x, ids, mv = _row_inputs(rng, 60, 192)
+    g = _run_select_compact(rng.random(60).astype(np.float32), cu, np.array([5, 5, 5]), 32, x,
+                            ids, mv)
+    assert g["status"] == O.DORA_ERR_DEVICE_SEQLEN
+    assert g["cu"].tolist() == [0, 5, 5, 10]               # the long image keeps nothing
+    assert np.all(g["packed"][10:].view(np.int16) == SENT)
+
+
+def test_select_compact_overlapping_boundaries_stay_in_capacity():
+    """Boundaries that are not increasing ([0, 100, 50, 150]: the second
+    image has negative length, the third overlaps the first) keep the outputs
+    inside the input's 150 rows: rows past them are dropped and the status
+    says so."""
+    rng = np.random.default_rng(45)
+    cu = np.array([0, 100, 50, 150], np.int32)
+    s = rng.random(150).astype(np.float32)
+    x, ids, mv = _row_inputs(rng, 150, 128)
+    keeps = np.array([90, 0, 80])
+    g = _run_select_compact(s, cu, keeps, 100, x, ids, mv, t_cap=150, extra=64)
+    # the first error recorded wins: the negative length or the overflow
+    assert g["status"] in (O.DORA_ERR_DEVICE_BAD_COUNT, O.DORA_ERR_DEVICE_SEQLEN)
+    assert g["cu"].tolist() == [0, 90, 90, 170]
+    assert np.all(g["kept"][150:] == SENT)
+    assert np.all(g["packed"][150:].view(np.int16) == SENT)
+    assert np.all(g["ids"][150:] == SENT) and np.all(g["mv"][150:] == SENT)
+    # the first image's 90 rows are exact
+    rk, _, _ = O.select_keep(s[:100], np.array([0, 100]), np.array([90]))
+    assert np.array_equal(g["kept"][:90], rk)
+    assert np.array_equal(g["packed"][:90], x[rk])
+
+
+def test_select_compact_large_batch_b1024():
+    rng = np.random.default_rng(46)
+    lens = rng.integers(1, 198, size=1024)
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    s = rng.random(t).astype(np.float32)
+    x, ids, mv = _row_inputs(rng, t, 768)
+    keeps = np.array([rng.integers(1, n + 1) for n in lens])
+    _check_select_compact(s, cu, keeps, x, ids, mv, 197)
+
+
+def test_select_compact_longest_images():
+    """Images of 8192 tokens (the selection's shared-memory limit), every
+    image the same length and a mix."""
+    rng = np.random.default_rng(47)
+    lens = np.array([8192, 1, 8192, 4097])
+    cu = O.cu_from_counts(lens)
+    t = int(cu[-1])
+    s = rng.random(t).astype(np.float32)
+    pick = rng.random(t) < 0.4                        # ties and NaN among random scores
+    s[pick] = rng.choice(np.array([0.0, 0.5, 1.0, np.nan], np.float32), size=int(pick.sum()))
+    x, ids, mv = _row_inputs(rng, t, 64)
+    keeps = np.array([4000, 1, 8192, 17])
+    _check_select_compact(s, cu, keeps, x, ids, mv, 8192)
+
+
+# ---------------------------------------------------------------------------
 # LayerNorm
 # ---------------------------------------------------------------------------
 
