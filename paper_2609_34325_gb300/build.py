@@ -17,6 +17,11 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libdora.so")
+# The timeout-path test library: the same objects, except that the attention
+# kernel's bounded waits give up after 5 ms and its first CTA withholds its
+# first K/V load, so a wait runs out (tests/test_gpu_timeout.py).
+TIMEOUT_TEST_LIB_PATH = os.path.join(HERE, "libdora_timeout_test.so")
+TIMEOUT_TEST_FLAGS = ["-DDORA_TEST_WITHHOLD_KV_LOAD", "-DDORA_TEST_WAIT_LIMIT_NS=5000000ull"]
 SOURCES = ["token_ops.cu", "gemm_tcgen05.cu", "attn_tcgen05.cu", "api.cu", "noalloc.cu",
            "actor.cu", "embed_head.cu", "training.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -41,10 +46,13 @@ def _deps() -> list:
 
 
 def up_to_date() -> bool:
-    if not os.path.exists(LIB_PATH):
-        return False
-    t = os.path.getmtime(LIB_PATH)
-    return all(os.path.getmtime(f) <= t for f in _deps())
+    for lib in (LIB_PATH, TIMEOUT_TEST_LIB_PATH):
+        if not os.path.exists(lib):
+            return False
+        t = os.path.getmtime(lib)
+        if not all(os.path.getmtime(f) <= t for f in _deps()):
+            return False
+    return True
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags: list | None = None) -> str:
@@ -56,9 +64,10 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list | None =
     common = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE,
                      "-I", CSRC, "--expt-relaxed-constexpr"] + list(extra_flags or [])
 
-    def compile_one(src: str) -> str:
-        obj = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + ".o")
-        cmd = [nvcc] + common + ["-c", os.path.join(CSRC, src), "-o", obj]
+    def compile_one(job) -> str:
+        src, tag, flags = job
+        obj = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + tag + ".o")
+        cmd = [nvcc] + common + flags + ["-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed on {src}:\n{' '.join(cmd)}\n{r.stdout}\n{r.stderr}")
@@ -66,15 +75,24 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list | None =
             print(r.stdout, r.stderr)
         return obj
 
-    with ThreadPoolExecutor(len(SOURCES)) as ex:
-        objs = list(ex.map(compile_one, SOURCES))
-    tmp = LIB_PATH + ".tmp"
-    cmd = [nvcc] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs + [
-        "-Xlinker", "-rpath," + _cuda_lib_dir(nvcc)]
-    r = subprocess.run(cmd, capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError(f"link failed:\n{' '.join(cmd)}\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB_PATH)
+    jobs = [(src, "", []) for src in SOURCES] + [("attn_tcgen05.cu", "_timeout_test",
+                                                  TIMEOUT_TEST_FLAGS)]
+    with ThreadPoolExecutor(len(jobs)) as ex:
+        objs = list(ex.map(compile_one, jobs))
+    main_objs = objs[:len(SOURCES)]
+    test_objs = [objs[-1] if s == "attn_tcgen05.cu" else o for s, o in zip(SOURCES, main_objs)]
+
+    def link(objs_, path):
+        tmp = path + ".tmp"
+        cmd = [nvcc] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + objs_ + [
+            "-Xlinker", "-rpath," + _cuda_lib_dir(nvcc)]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"link failed:\n{' '.join(cmd)}\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, path)
+
+    link(test_objs, TIMEOUT_TEST_LIB_PATH)
+    link(main_objs, LIB_PATH)
     return LIB_PATH
 
 

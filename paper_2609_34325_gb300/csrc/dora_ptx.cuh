@@ -13,8 +13,14 @@
 namespace dora {
 
 // A bounded wait gives up after this many nanoseconds of %globaltimer and
-// reports DORA_ERR_TIMEOUT instead of spinning forever.
+// reports DORA_ERR_TIMEOUT instead of spinning forever.  The timeout-path test
+// library builds the attention kernel with a limit of a few milliseconds
+// (DORA_TEST_WAIT_LIMIT_NS); the product library never defines it.
+#ifdef DORA_TEST_WAIT_LIMIT_NS
+constexpr uint64_t kWaitLimitNs = DORA_TEST_WAIT_LIMIT_NS;
+#else
 constexpr uint64_t kWaitLimitNs = 1000ull * 1000ull * 1000ull;   // 1 s
+#endif
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
