@@ -18,12 +18,14 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libdora.so")
 # The timeout-path test library: the same objects, except that the attention
-# kernel's bounded waits give up after 5 ms and its first CTA withholds its
+# kernels' bounded waits give up after 5 ms and their first CTA withholds its
 # first K/V load, so a wait runs out (tests/test_gpu_timeout.py).
 TIMEOUT_TEST_LIB_PATH = os.path.join(HERE, "libdora_timeout_test.so")
 TIMEOUT_TEST_FLAGS = ["-DDORA_TEST_WITHHOLD_KV_LOAD", "-DDORA_TEST_WAIT_LIMIT_NS=5000000ull"]
-SOURCES = ["token_ops.cu", "gemm_tcgen05.cu", "attn_tcgen05.cu", "api.cu", "noalloc.cu",
-           "actor.cu", "embed_head.cu", "training.cu"]
+SOURCES = ["token_ops.cu", "gemm_tcgen05.cu", "attn_tcgen05.cu", "attn_exchange_tcgen05.cu",
+           "api.cu", "noalloc.cu", "actor.cu", "embed_head.cu", "training.cu"]
+# the attention translation units, rebuilt with the test flags for the timeout-path library
+ATTN_SOURCES = ("attn_tcgen05.cu", "attn_exchange_tcgen05.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -75,12 +77,13 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list | None =
             print(r.stdout, r.stderr)
         return obj
 
-    jobs = [(src, "", []) for src in SOURCES] + [("attn_tcgen05.cu", "_timeout_test",
-                                                  TIMEOUT_TEST_FLAGS)]
+    jobs = [(src, "", []) for src in SOURCES] + [(src, "_timeout_test", TIMEOUT_TEST_FLAGS)
+                                                  for src in ATTN_SOURCES]
     with ThreadPoolExecutor(len(jobs)) as ex:
         objs = list(ex.map(compile_one, jobs))
     main_objs = objs[:len(SOURCES)]
-    test_objs = [objs[-1] if s == "attn_tcgen05.cu" else o for s, o in zip(SOURCES, main_objs)]
+    test_attn = dict(zip(ATTN_SOURCES, objs[len(SOURCES):]))
+    test_objs = [test_attn.get(s, o) for s, o in zip(SOURCES, main_objs)]
 
     def link(objs_, path):
         tmp = path + ".tmp"
