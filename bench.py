@@ -40,16 +40,17 @@ METRIC = "pruned ViT forward images/sec on 1 GB300; varlen-attn % bf16 peak; com
 UNIT = "images/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
-# DRAM traffic per GEMM launch from an ncu capture (dram__bytes_read.sum +
-# dram__bytes_write.sum), keyed by the workload and the sha256 of the kernel
-# source it was taken on; reported as null once the source changes and for a
-# workload without a capture.
-NCU_TRAFFIC = {
-    # profiles/gemm_tcgen05_deit_base_b256.md: mean over the 48 GEMM launches
-    # of one forward step
-    ("cfg3", "b34dcbc477c16fbd82653b7888b9deb4fa8716d95e482f5d9899e205d6137ff3"): 188246208,
-    # the same capture on the DINOv2-B/14 workload (bench.py --config cfg6)
-    ("cfg6", "b34dcbc477c16fbd82653b7888b9deb4fa8716d95e482f5d9899e205d6137ff3"): 270655605,
+# DRAM traffic of the GEMM (dram__bytes_read.sum + dram__bytes_write.sum)
+# from an ncu capture of the linear micro-benchmark (50432 rows, D = 768, MLP
+# 3072: one launch of each linear, inputs far above L2), keyed by the sha256 of
+# the kernel source it was taken on: bytes per row of each linear.  The bench
+# scales it to its own launches by their row counts (weights are read once a
+# launch, a small share), so it is reported for the DeiT-B shape only, and as
+# null once the source changes.
+NCU_GEMM_BYTES_PER_ROW = {
+    # profiles/gemm_tcgen05_deit_base_b256.md
+    "34028c7f64f651efea1ca44f9acc035d375b0841fc63cfcd50bdad42358a173f": {
+        "gemm_qkv": 5141.4, "gemm_proj": 4038.9, "gemm_fc1": 6640.8, "gemm_fc2": 9156.8},
 }
 
 
@@ -824,7 +825,7 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
                        dict(bytes=2.0 * T * d + 8.0 * T))
             launch("gemm_qkv", lambda: P.dora_linear_ln(x, mvi, cfg.ln_eps, *fl["qkv"], qkv,
                                                    m_dev=rows, stream=stream),
-                   dict(flops=2.0 * T * 3 * d * d,
+                   dict(flops=2.0 * T * 3 * d * d, rows=T,
                         bytes=2.0 * (T * d + 3 * d * d + 3 * T * d) + 8.0 * T + 24.0 * d))
             launch("attention", lambda: P.dora_varlen_attn(qkv, cu, cfg.n_tokens, cfg.heads, o,
                                                           stream=stream),
@@ -834,7 +835,7 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
                    lambda: P.dora_linear_residual_stats(o, w["w_proj"], x, hattn, sm,
                                                         bias=w["b_proj"], m_dev=rows,
                                                         stream=stream),
-                   dict(flops=2.0 * T * d * d, bytes=2.0 * (3 * T * d + d * d) + sb * T))
+                   dict(flops=2.0 * T * d * d, rows=T, bytes=2.0 * (3 * T * d + d * d) + sb * T))
             launch("merge_moments", lambda: P.dora_merge_moments(sm, mv, rows_dev=rows,
                                                                 stream=stream),
                    dict(bytes=sb * T + 8.0 * T))
@@ -862,14 +863,14 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
                 hk, rows2, mvk = hattn, rows, mv
             launch("gemm_fc1", lambda: P.dora_linear_ln(hk, mvk, cfg.ln_eps, *fl["fc1"], u,
                                                    gelu=True, m_dev=rows2, stream=stream),
-                   dict(flops=2.0 * To * d * m,
+                   dict(flops=2.0 * To * d * m, rows=To,
                         bytes=2.0 * (To * d + d * m + To * m) + 8.0 * To + 8.0 * m))
             if l + 1 < cfg.depth:
                 launch("gemm_fc2",
                        lambda: P.dora_linear_residual_stats(u, w["w_fc2"], hk, out, sm,
                                                             bias=w["b_fc2"], m_dev=rows2,
                                                             stream=stream),
-                       dict(flops=2.0 * To * m * d,
+                       dict(flops=2.0 * To * m * d, rows=To,
                             bytes=2.0 * (To * m + m * d + 2 * To * d) + sb * To))
                 launch("merge_moments", lambda: P.dora_merge_moments(sm, mvx[l % 2],
                                                                     rows_dev=rows2,
@@ -879,17 +880,19 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
                 launch("gemm_fc2", lambda: P.dora_linear(u, w["w_fc2"], out, bias=w["b_fc2"],
                                                     residual=hk, epilogue=P.EPI_BIAS_RESIDUAL,
                                                     m_dev=rows2, stream=stream),
-                       dict(flops=2.0 * To * m * d, bytes=2.0 * (To * m + m * d + 2 * To * d)))
+                       dict(flops=2.0 * To * m * d, rows=To,
+                            bytes=2.0 * (To * m + m * d + 2 * To * d)))
             x = out
     torch.cuda.synchronize()
     agg = {}
     for cls, a, b, work in records:
-        e = agg.setdefault(cls, dict(ms=0.0, launches=0, flops=0.0, bytes=0.0))
+        e = agg.setdefault(cls, dict(ms=0.0, launches=0, flops=0.0, bytes=0.0, rows=0.0))
         e["ms"] += a.elapsed_time(b)
         e["launches"] += 1
         e["flops"] += work.get("flops", 0.0)
         e["bytes"] += work.get("bytes", 0.0)
-    gemm = dict(ms=0.0, launches=0, flops=0.0, bytes=0.0)
+        e["rows"] += work.get("rows", 0.0)
+    gemm = dict(ms=0.0, launches=0, flops=0.0, bytes=0.0, rows=0.0)
     for k in [k for k in agg if k.startswith("gemm_")]:
         for f in gemm:
             gemm[f] += agg[k][f]
@@ -901,6 +904,7 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
         e["launches"] //= steps
         e["flops"] /= steps
         e["bytes"] /= steps
+        e["rows"] /= steps
         if e["flops"]:
             e["tflops"] = e["flops"] / (e["ms"] * 1e-3) / 1e12
     return agg
@@ -911,7 +915,10 @@ def roofline_report(kern, peaks, peak_src, workload):
     g = kern["gemm"]
     gemm_tf = g["flops"] / (g["ms"] * 1e-3) / 1e12
     src = os.path.join(ROOT, "paper_2609_34325_gb300", "csrc", "gemm_tcgen05.cu")
-    tr = NCU_TRAFFIC.get((workload, sha256_of(src)))
+    per_row = NCU_GEMM_BYTES_PER_ROW.get(sha256_of(src)) if workload == "cfg3" else None
+    tr = None
+    if per_row is not None:
+        tr = round(sum(per_row[k] * kern[k]["rows"] for k in per_row) / g["launches"])
     # the per-kernel pass times each launch on its own over a fraction of a
     # second: the burst peak is its denominator
     out = {"roofline": {"kernel": "gemm_tcgen05 (QKV/proj/fc1/fc2)", "bound": "tensor",
@@ -920,6 +927,9 @@ def roofline_report(kern, peaks, peak_src, workload):
                         "peak_kind": f"bf16 burst ({tag})",
                         "frac_of_sustained": round(gemm_tf / peaks["bf16_tflops_sustained"], 4),
                         "traffic": tr,
+                        "traffic_case": None if tr is None else (
+                            "ncu DRAM bytes per row of each linear on the micro-benchmark "
+                            "(50432 rows), scaled by this step's row counts"),
                         "algorithmic_bytes_per_launch": round(g["bytes"] / g["launches"]),
                         "share_of_step": round(g["share"], 4)}}
     a = kern["attention"]
