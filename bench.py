@@ -151,7 +151,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", self.gpu_id, "--query-gpu=" + self.FIELDS,
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -215,6 +215,12 @@ def device_tensors(torch, cfg, seed, n_sets, dev):
             "ln2_b": torch.zeros(d, dtype=bf16, device=dev),
             "w_fc1": normal((m, d), 0.02), "b_fc1": torch.zeros(m, dtype=bf16, device=dev),
             "w_fc2": normal((d, m), 0.02), "b_fc2": torch.zeros(d, dtype=bf16, device=dev)})
+        if cfg.layerscale:
+            # per-channel LayerScale on both branches (folded into w_proj and
+            # w_fc2 at load), gamma ~ 0.05 + 0.45 U(0, 1) as the host generator draws it
+            for nm in ("ls1", "ls2"):
+                u = torch.rand(d, generator=g, device=dev, dtype=torch.float32)
+                blocks[-1][nm] = (0.05 + 0.45 * u).to(bf16)
     xs = [normal((cfg.batch * cfg.n_tokens, d), 1.0) for _ in range(n_sets)]
     return blocks, xs
 
@@ -243,8 +249,8 @@ def gpu_uuid_arg(torch, dev_index):
 
 
 # the other forward shapes timed beside the main workload (pruned, dense and
-# the per-kernel pass): ViT-L/16 and ViT-B/16 at 384 pixels
-EXTRA_WORKLOADS = ("cfg4", "cfg5")
+# the per-kernel pass): ViT-L/16, ViT-B/16 at 384 pixels and DINOv2-B/14
+EXTRA_WORKLOADS = ("cfg4", "cfg5", "cfg6")
 
 
 def run_gpu(args, rank, world, local_rank):
