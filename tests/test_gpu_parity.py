@@ -1069,10 +1069,17 @@ def _check_actor(cfg, cu, qkv, rho, e_prev, wa, got, block, images):
     # encoder output within the block tolerance; gate probability in fp32
     assert_close(got["z"][rows], ref["z"], "actor Z", atol=ACTOR_ATOL, rtol=ACTOR_RTOL)
     assert np.all(np.abs(got["p"][images] - ref["p"]) <= 1e-4)
-    # decisions agree wherever the oracle's margin exceeds the arithmetic's error
+    # decisions agree wherever the oracle's margin exceeds the arithmetic's error,
+    # and the filter leaves out only near-ties: all but 5% (at least one) of
+    # the gate decisions are compared, and all but 15% (at least one) of the
+    # budgets equal the oracle's own argmax (the rest are within 0.05 of its
+    # best logit)
     clear = np.abs(ref["p"] - 0.5) > 1e-4
     assert np.array_equal((got["p"][images] >= 0.5)[clear], (ref["p"] >= 0.5)[clear])
+    skipped = int((~clear).sum())
+    assert skipped <= max(1, int(0.05 * clear.size)), f"gate decisions skipped: {skipped}"
     grid = O.budget_grid(cfg.n_vis0)
+    exact = total = 0
     for j, i in enumerate(images):
         bud = int(got["budget"][i])
         feas = grid <= n_vis[j] - 4
@@ -1082,6 +1089,10 @@ def _check_actor(cfg, cu, qkv, rho, e_prev, wa, got, block, images):
         assert bud in grid[feas]
         best = ref["logits"][j][feas].max()
         assert ref["logits"][j][list(grid).index(bud)] >= best - 0.05, (i, bud, ref["budget"][j])
+        total += 1
+        exact += int(bud == int(ref["budget"][j]))
+    assert exact >= total - max(1, int(0.15 * total)), (
+        f"budgets equal to the oracle's: {exact}/{total}")
     # the integer bookkeeping is exact given the GPU's own decisions
     g, bud = got["gate"][images], got["budget"][images]
     assert np.array_equal(g, ((got["p"][images] >= 0.5) & (bud > 0)).astype(np.int32))
