@@ -60,15 +60,21 @@ __device__ __forceinline__ void load_rows(const QkvMaps& mp, uint16_t* dst, uint
   if (r16 & 16) tma_load_2d(dst + off * HD, &mp.m16, bar, x, y + off);
 }
 
-// Rows of image `img`, clamped to the buffer (0 when its start lies outside).
-__device__ __forceinline__ int image_rows(const int32_t* cu, int img, int t_cap, int& lo) {
-  lo = cu[img];
-  const int n = cu[img + 1] - lo;
+// Rows of the image with bounds [b0, b1), clamped to the buffer (0 when its
+// start lies outside); lo receives its first row.
+__device__ __forceinline__ int clamp_rows(int b0, int b1, int t_cap, int& lo) {
+  lo = b0;
+  const int n = b1 - b0;
   if (lo < 0 || lo > t_cap) {
     lo = 0;
     return 0;
   }
   return n < 0 ? 0 : (n > t_cap - lo ? t_cap - lo : n);
+}
+
+// Rows of image `img`, clamped to the buffer (0 when its start lies outside).
+__device__ __forceinline__ int image_rows(const int32_t* cu, int img, int t_cap, int& lo) {
+  return clamp_rows(cu[img], cu[img + 1], t_cap, lo);
 }
 
 // Estimated cost of one image-head with n rows, in steps: every query tile
@@ -121,82 +127,83 @@ struct Walker {
 };
 
 // Whole warp: the CTA's image-head range.  Image-head ih belongs to CTA
-// floor(C(ih) * grid / total), C being the cost of the image-heads before it;
-// CTA 0 also checks every image against the buffer and max_seqlen.
+// floor(C(ih) * grid / total), C being the cost of the image-heads before it
+// (image-major, head-minor order); CTA 0 also checks every image against the
+// buffer and max_seqlen.  Each lane owns a contiguous block of images whose
+// bounds it reads as one batch of independent loads, so the whole search
+// costs about two memory round trips for any batch (a walk over the batch
+// 32 images at a time, each chunk's loads waiting for the previous chunk's
+// shuffles, took 4-9 us at 256 images).
 __device__ inline void find_range(const int32_t* cu, int batch, int heads, int t_cap, int max_seqlen,
-                           int32_t* status, long long& ih_b, long long& ih_e) {
+                                  int32_t* status, long long& ih_b, long long& ih_e) {
   const int lane = threadIdx.x & 31;
-  long long total = 0;
-  for (int i0 = 0; i0 < batch; i0 += 32) {
-    const int i = i0 + lane;
-    long long c = 0;
-    if (i < batch) {
-      int lo;
-      c = ih_cost(image_rows(cu, i, t_cap, lo));
-      if (blockIdx.x == 0) {
-        const int l0 = cu[i], n = cu[i + 1] - l0;
-        if (l0 < 0 || l0 > t_cap || n > t_cap - l0 || n > max_seqlen)
-          record_status(status, DORA_ERR_DEVICE_SEQLEN);
+  const int per = (batch + 31) / 32;
+  const int i0 = min(batch, lane * per), i1 = min(batch, i0 + per);
+  long long mine = 0, c_last = 0;       // this lane's cost sum and its last image's cost
+  for (int k0 = i0; k0 < i1; k0 += 8) {
+    int bnd[9];
+#pragma unroll
+    for (int t = 0; t < 9; ++t) bnd[t] = (k0 + t <= i1) ? __ldg(cu + k0 + t) : 0;
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      if (k0 + t < i1) {
+        int lo;
+        c_last = ih_cost(clamp_rows(bnd[t], bnd[t + 1], t_cap, lo));
+        mine += c_last;
+        if (blockIdx.x == 0) {
+          const int l0 = bnd[t], n = bnd[t + 1] - l0;
+          if (l0 < 0 || l0 > t_cap || n > t_cap - l0 || n > max_seqlen)
+            record_status(status, DORA_ERR_DEVICE_SEQLEN);
+        }
       }
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-    total += c;
   }
+  long long incl = mine;                // one head's cost of the images up to this lane's last
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  const long long one_head = __shfl_sync(0xffffffffu, incl, 31);
   const long long nih = static_cast<long long>(batch) * heads;
-  const long long G = gridDim.x, b = blockIdx.x;
-  ih_b = nih;
-  ih_e = nih;
-  if (total == 0) {
+  if (one_head == 0) {
     ih_b = ih_e = 0;
     return;
   }
-  total *= heads;
-  const long long xb = b * total, xe = (b + 1) * total;
-  bool fb = false, fe = (b == G - 1);
-  long long pre = 0;                 // cost of one head of the images before i0
-  for (int i0 = 0; i0 < batch && !(fb && fe); i0 += 32) {
-    const int i = i0 + lane;
-    long long c = 0;
-    if (i < batch) {
-      int lo;
-      c = ih_cost(image_rows(cu, i, t_cap, lo));
-    }
-    long long incl = c;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const long long t = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += t;
-    }
-    const long long base = static_cast<long long>(heads) * (pre + incl - c) * G;   // C(i, 0) * G
-    // first image-head of image i whose C * G reaches x, or -1
-    auto first_at = [&](long long x) -> long long {
-      if (i >= batch) return -1;
-      if (base >= x) return static_cast<long long>(i) * heads;
-      if (c > 0) {
-        const long long h = (x - base + c * G - 1) / (c * G);
-        if (h < heads) return static_cast<long long>(i) * heads + h;
-      }
-      return -1;
-    };
-    if (!fb) {
-      const long long r = first_at(xb);
-      const unsigned m = __ballot_sync(0xffffffffu, r >= 0);
-      if (m) {
-        ih_b = __shfl_sync(0xffffffffu, r, __ffs(m) - 1);
-        fb = true;
+  const long long total = one_head * heads, G = gridDim.x, bx = blockIdx.x;
+  // first image-head with C * G >= x (nih if none): C grows along the order,
+  // so it lies in the first lane whose last image-head reaches x, found by
+  // that lane walking its own images (their bounds are in L1 by now)
+  auto locate = [&](long long x) -> long long {
+    const bool has = i0 < i1 && (heads * (incl - c_last) + (heads - 1) * c_last) * G >= x;
+    const unsigned m = __ballot_sync(0xffffffffu, has);
+    if (m == 0u) return nih;
+    const int owner = __ffs(m) - 1;
+    long long r = nih;
+    if (lane == owner) {
+      long long pre = incl - mine;      // one head's cost of the images before i0
+      for (int i = i0; i < i1; ++i) {
+        int lo;
+        const long long c = ih_cost(image_rows(cu, i, t_cap, lo));
+        const long long base = heads * pre * G;
+        if (base >= x) {
+          r = static_cast<long long>(i) * heads;
+          break;
+        }
+        if (c > 0) {
+          const long long h = (x - base + c * G - 1) / (c * G);
+          if (h < heads) {
+            r = static_cast<long long>(i) * heads + h;
+            break;
+          }
+        }
+        pre += c;
       }
     }
-    if (!fe) {
-      const long long r = first_at(xe);
-      const unsigned m = __ballot_sync(0xffffffffu, r >= 0);
-      if (m) {
-        ih_e = __shfl_sync(0xffffffffu, r, __ffs(m) - 1);
-        fe = true;
-      }
-    }
-    pre += __shfl_sync(0xffffffffu, incl, 31);
-  }
+    return __shfl_sync(0xffffffffu, r, owner);
+  };
+  ih_b = locate(bx * total);
+  ih_e = (bx == G - 1) ? nih : locate((bx + 1) * total);
 }
 
 __device__ __forceinline__ void mask_tail(uint32_t (&a)[32], int live) {
