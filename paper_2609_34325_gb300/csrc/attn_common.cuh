@@ -190,12 +190,9 @@ __device__ inline void find_range(const int32_t* cu, int batch, int heads, int t
           r = static_cast<long long>(i) * heads;
           break;
         }
-        if (c > 0) {
-          const long long h = (x - base + c * G - 1) / (c * G);
-          if (h < heads) {
-            r = static_cast<long long>(i) * heads + h;
-            break;
-          }
+        if (base + (heads - 1) * c * G >= x) {   // one of this image's heads (c > 0)
+          r = static_cast<long long>(i) * heads + (x - base + c * G - 1) / (c * G);
+          break;
         }
         pre += c;
       }
