@@ -724,6 +724,30 @@ def test_attention_empty_images_and_long_image_flag():
     assert st == 6
 
 
+@pytest.mark.parametrize("mix", ["many_images", "skewed", "few_image_heads"])
+def test_attention_range_split_over_many_images(mix):
+    """The split of image-heads over the persistent CTAs (each lane of the
+    range search reading a block of image bounds): batches above 256 images
+    (several rounds of loads per lane), skewed costs with many empty and
+    one-token images beside a few of 300 tokens (the kernel for images past
+    256 tokens), and fewer image-heads than SMs.  Every row of every
+    image is compared with the oracle, so an image-head given to no CTA (its
+    rows keep the fill value) or to two fails."""
+    rng = np.random.default_rng({"many_images": 21, "skewed": 22, "few_image_heads": 23}[mix])
+    if mix == "many_images":
+        lens = rng.integers(0, 201, 1100)
+        lens[rng.random(1100) < 0.2] = 0
+        heads = 2
+    elif mix == "skewed":
+        lens = rng.integers(0, 4, 700)
+        lens[rng.choice(700, 9, replace=False)] = 300    # the per-key-half kernel
+        heads = 3
+    else:
+        lens = rng.integers(0, 257, 40)
+        heads = 1
+    _check_attn(lens, heads, 24)
+
+
 def test_attention_matches_dense_when_unpruned():
     """k = 0: packed attention equals dense batched attention (torch SDPA on
     the same bf16 values, fp64) on the GPU path too."""
