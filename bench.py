@@ -49,8 +49,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # null once the source changes.
 NCU_GEMM_BYTES_PER_ROW = {
     # profiles/gemm_tcgen05_deit_base_b256.md
-    "34028c7f64f651efea1ca44f9acc035d375b0841fc63cfcd50bdad42358a173f": {
-        "gemm_qkv": 5141.4, "gemm_proj": 4038.9, "gemm_fc1": 6640.8, "gemm_fc2": 9156.8},
+    "5b47db1d6d015aabefc6c8661ff652173f8c4bb2ce27827b8d1c06fab80c04fb": {
+        "gemm_qkv": 5137.0, "gemm_proj": 4040.4, "gemm_fc1": 6634.5, "gemm_fc2": 9164.1},
 }
 
 

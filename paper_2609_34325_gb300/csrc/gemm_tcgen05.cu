@@ -235,8 +235,9 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   // Work is a list of tile pairs: pair p covers M-tiles 2*(p / n_tiles) and
-  // 2*(p / n_tiles) + 1 of N-tile p % n_tiles; CTA `rank` of cluster c takes
-  // the M-tile 2*(p / n_tiles) + rank of pairs c, c + clusters, ...
+  // 2*(p / n_tiles) + 1 of N-tile p % n_tiles (row pairs counted from the
+  // last with ep.m_reverse); CTA `rank` of cluster c takes the M-tile
+  // 2*(p / n_tiles) + rank of pairs c, c + clusters, ...
   // Both CTAs of a cluster walk the same pairs in lockstep.
   const int rank = static_cast<int>(cluster_ctarank());
   const int cid = blockIdx.x / kCluster;
@@ -290,13 +291,20 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
   const int num_pairs = m_pairs * n_tiles;
   const uint32_t tmem = s.tmem_base;
   volatile int* abort = &s.abort_flag;
+  // row pair of work item p; m_reverse walks them from the last, so that a
+  // linear reading the output of one that walked forward starts on the rows
+  // written last, still in L2
+  auto mpair = [&](int p) {
+    const int q0 = p / n_tiles;
+    return ep.m_reverse ? m_pairs - 1 - q0 : q0;
+  };
 
   if (warp == 0) {
     if (lane == 0) {
       int it = 0;
       bool ok = true;
       for (int pr = cid; ok && pr < num_pairs; pr += n_clusters) {
-        const int mt = 2 * (pr / n_tiles) + rank;
+        const int mt = 2 * mpair(pr) + rank;
         const int nt = pr % n_tiles;
         for (int kb = 0; kb < kb_count; ++kb) {
           const int st = it % kStages;
@@ -405,7 +413,7 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
     // load per chunk into the chunk's staging buffer, once the stores of the
     // previous tile have read those buffers.
     auto prefetch_residual = [&](int p) {
-      const int row0 = (2 * (p / n_tiles) + rank) * BM + q * 32;
+      const int row0 = (2 * mpair(p) + rank) * BM + q * 32;
       if (row0 + 32 > M) return;
       const int col0 = (p % n_tiles) * BN + slot * kCols;
       if (lane == 0) bulk_wait_group_read0();
@@ -454,7 +462,7 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
     // (a warp's 32 rows are one 256-byte load).
     float2 mv = make_float2(0.f, 0.f);
     auto load_mv = [&](int p) {
-      const int row_p = (2 * (p / n_tiles) + rank) * BM + q * 32 + lane;
+      const int row_p = (2 * mpair(p) + rank) * BM + q * 32 + lane;
       if (row_p < M) mv = __ldg(reinterpret_cast<const float2*>(ep.stats_in) + row_p);
     };
     if constexpr (C::kLn)
@@ -469,7 +477,7 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
     for (int pr = cid; ok && pr < num_pairs; pr += n_clusters, ++ti) {
       const int acc = ti & 1;
       const uint32_t aph = (ti >> 1) & 1;
-      const int mt = 2 * (pr / n_tiles) + rank;
+      const int mt = 2 * mpair(pr) + rank;
       const int nt = pr % n_tiles;
       const int row0 = mt * BM + q * 32;          // first row of this warp
       const int row = row0 + lane;

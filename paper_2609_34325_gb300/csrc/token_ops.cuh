@@ -108,6 +108,7 @@ struct LinearEpi {
   float* stats_out = nullptr;           // slice moments of y, [n/64][m_cap], nullable
   float eps = 0.f;                      // LayerNorm epsilon (LN epilogues)
   int32_t slices = 0;                   // n / 64 (stats_out)
+  int32_t m_reverse = 0;                // 1: walk the row blocks from the last one
 };
 // lda: row pitch of x in elements (0 = k; a multiple of 8).
 cudaError_t launch_linear(const uint16_t* x, int32_t m_cap, const int32_t* m_dev, int32_t k,
