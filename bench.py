@@ -40,6 +40,9 @@ METRIC = "pruned ViT forward images/sec on 1 GB300; varlen-attn % bf16 peak; com
 UNIT = "images/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
+# buffer sets the end-to-end leg rotates (inputs uploaded, outputs read back)
+E2E_SETS = 3
+
 # DRAM traffic of the GEMM (dram__bytes_read.sum + dram__bytes_write.sum)
 # from an ncu capture of the linear micro-benchmark (50432 rows, D = 768, MLP
 # 3072: one launch of each linear, inputs far above L2), keyed by the sha256 of
@@ -324,17 +327,17 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream, cfg_name, cor
                  ws=P.alloc_workspace(tc, nb, blocks[0], dev),
                  scores=torch.zeros(tc, dtype=torch.float32, device=dev),
                  kept=torch.zeros(tc, dtype=torch.int32, device=dev))
-        # two sets of ping-pong buffers: the e2e pipeline alternates them between
-        # steps so that a step's readback never races the next step's writes
+        # E2E_SETS sets of buffers: the e2e pipeline rotates them between steps
+        # so that a step's readback never races a later step's writes
         L["xbufs"] = [[torch.zeros(tc, cfg.dim, dtype=torch.bfloat16, device=dev)
-                       for _ in range(2)] for _ in range(2)]
+                       for _ in range(2)] for _ in range(E2E_SETS)]
         L["cubufs"] = [[torch.zeros(nb + 1, dtype=torch.int32, device=dev) for _ in range(2)]
-                       for _ in range(2)]
+                       for _ in range(E2E_SETS)]
         L["idbufs"] = [[torch.zeros(tc, dtype=torch.int32, device=dev) for _ in range(2)]
-                       for _ in range(2)]
+                       for _ in range(E2E_SETS)]
         # row moments handed from block to block (x_out_moments -> x_in_moments)
         L["mvbufs"] = [[torch.zeros(tc, 2, dtype=torch.float32, device=dev) for _ in range(2)]
-                       for _ in range(2)]
+                       for _ in range(E2E_SETS)]
         lanes.append(L)
     ws = lanes[0]["ws"]
     prune = list(cfg.prune_blocks)
@@ -664,37 +667,44 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream, cfg_name, cor
 
     # End to end through the C ABI with host buffers: every step copies its
     # inputs from pinned host memory and reads its result (final tokens and
-    # boundaries) back.  Copies run on a second stream, double-buffered, so
-    # step i+1's upload and step i's readback overlap step i's compute.
+    # boundaries) back.  Uploads and readbacks run on two more streams over
+    # E2E_SETS rotating buffer sets, so step i+1's upload and step i's
+    # readback overlap step i's compute.  (One copy stream over two sets, the
+    # readback of step i queued ahead of the upload of step i+2, left some
+    # 20-step runs 10-25% slower than the device-only step on the same box;
+    # two streams over three sets did not.)
     pin = [dict(x=torch.from_numpy(s["x"].view(np.int16)).view(torch.bfloat16).pin_memory(),
                 keeps=[torch.from_numpy(k.astype(np.int32)).pin_memory() for k in s["keeps"]],
                 tables=[torch.from_numpy(t).pin_memory() for t in s["tables"]])
            for s in hw.sets]
     dev_in = [dict(x=torch.empty_like(sets[0]["x"]),
                    keeps=[torch.empty_like(k) for k in sets[0]["keeps"]],
-                   tables=[torch.empty_like(t) for t in sets[0]["tables"]]) for _ in range(2)]
-    host_out = [torch.empty(t_cap, cfg.dim, dtype=torch.bfloat16).pin_memory() for _ in range(2)]
-    host_cu = [torch.empty(cfg.batch + split, dtype=torch.int32).pin_memory() for _ in range(2)]
+                   tables=[torch.empty_like(t) for t in sets[0]["tables"]]) for _ in range(E2E_SETS)]
+    host_out = [torch.empty(t_cap, cfg.dim, dtype=torch.bfloat16).pin_memory()
+                for _ in range(E2E_SETS)]
+    host_cu = [torch.empty(cfg.batch + split, dtype=torch.int32).pin_memory()
+               for _ in range(E2E_SETS)]
     h2d = (pin[0]["x"].numel() * 2 + sum(k.numel() * 4 for k in pin[0]["keeps"])
            + sum(t.numel() * 4 for t in pin[0]["tables"]))
     d2h = host_out[0].numel() * 2 + host_cu[0].numel() * 4
-    cstream = torch.cuda.Stream(device=dev)
+    up_stream = torch.cuda.Stream(device=dev)
+    down_stream = torch.cuda.Stream(device=dev)
 
     def ev():
         return torch.cuda.Event()
 
     def upload(i, after):
-        with torch.cuda.stream(cstream):
+        with torch.cuda.stream(up_stream):
             if after is not None:
-                cstream.wait_event(after)
-            src, dst = pin[i % nsets], dev_in[i & 1]
+                up_stream.wait_event(after)
+            src, dst = pin[i % nsets], dev_in[i % E2E_SETS]
             dst["x"].copy_(src["x"], non_blocking=True)
             for a, b in zip(dst["keeps"], src["keeps"]):
                 a.copy_(b, non_blocking=True)
             for a, b in zip(dst["tables"], src["tables"]):
                 a.copy_(b, non_blocking=True)
             e = ev()
-            e.record(cstream)
+            e.record(up_stream)
         return e
 
     def run_e2e(steps):
@@ -702,22 +712,23 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream, cfg_name, cor
         comp, down = {}, {}
         for i in range(steps):
             if i + 1 < steps:
-                up[i + 1] = upload(i + 1, comp.get(i - 1))    # slot (i+1)&1 free after step i-1
+                # input set (i+1) % E2E_SETS is free once step i+1-E2E_SETS is done
+                up[i + 1] = upload(i + 1, comp.get(i + 1 - E2E_SETS))
             stream.wait_event(up[i])
-            if i - 2 in down:
-                stream.wait_event(down[i - 2])                # output pair i&1 read back
-            outs = forward(dev_in[i & 1], True, pair=i & 1)
+            if i - E2E_SETS in down:
+                stream.wait_event(down[i - E2E_SETS])         # its output set read back
+            outs = forward(dev_in[i % E2E_SETS], True, pair=i % E2E_SETS)
             comp[i] = ev()
             comp[i].record(stream)
-            with torch.cuda.stream(cstream):
-                cstream.wait_event(comp[i])
+            with torch.cuda.stream(down_stream):
+                down_stream.wait_event(comp[i])
                 c0 = 0
                 for L, (x, cu) in zip(lanes, outs):     # each lane's rows and boundaries
-                    host_out[i & 1][L["r0"]:L["r1"]].copy_(x, non_blocking=True)
-                    host_cu[i & 1][c0:c0 + L["nb"] + 1].copy_(cu, non_blocking=True)
+                    host_out[i % E2E_SETS][L["r0"]:L["r1"]].copy_(x, non_blocking=True)
+                    host_cu[i % E2E_SETS][c0:c0 + L["nb"] + 1].copy_(cu, non_blocking=True)
                     c0 += L["nb"] + 1
                 down[i] = ev()
-                down[i].record(cstream)
+                down[i].record(down_stream)
         stream.wait_event(down[steps - 1])
 
     esteps = max(3, min(args.steps, 50))
@@ -726,7 +737,8 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream, cfg_name, cor
     barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    cstream.wait_event(e0)
+    up_stream.wait_event(e0)
+    down_stream.wait_event(e0)
     run_e2e(esteps)
     e1.record(stream)
     torch.cuda.synchronize()
@@ -735,7 +747,8 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream, cfg_name, cor
     result["e2e"] = {"value": round(cfg.batch * esteps * world / esecs, 1), "unit": UNIT,
                      "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                      "ms_per_step": round(1000 * esecs / esteps, 4),
-                     "copies": "pinned host <-> device on a second stream, overlapped with compute"}
+                     "copies": "pinned host <-> device on an upload and a readback stream, "
+                               f"{E2E_SETS} rotating buffer sets, overlapped with compute"}
 
     # per-kernel pass: the same step driven kernel by kernel with events
     kern = profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap,
