@@ -377,9 +377,11 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream, cfg_name, cor
                                              L["idbufs"][pair], L["mvbufs"][pair])
                 out = xbuf[l % 2]
                 mv_out = mvbuf[l % 2] if l + 1 < cfg.depth else None
-                # QKV, attention, projection, merge, fc1, fc2 (+ row moments of the
-                # first input, + merge of the output's moments)
-                n += 6 + (c["mv"] is None) + (mv_out is not None)
+                # QKV, attention, projection, fc1, fc2, the merge of the
+                # projection's moments (the compaction merges them for the kept
+                # rows at a pruning block) (+ row moments of the first input, +
+                # merge of the output's moments)
+                n += 5 + (not (pruned and l in prune)) + (c["mv"] is None) + (mv_out is not None)
                 sl = L["stream"]
                 if pruned and l in prune and with_actor:
                     j = prune.index(l)
@@ -394,9 +396,9 @@ def _run_gpu_on_stream(args, rank, world, local_rank, dev, stream, cfg_name, cor
                     c["cu"], c["ids"] = cubuf[j % 2], idbuf[j % 2]
                     # actor: input projection, gate, LayerNorm statistics, QKV,
                     # attention, output projection, moment merge, two
-                    # feed-forward linears, budget and selector; then the
-                    # selection fused with the compaction
-                    n += 10 + 1
+                    # feed-forward linears, the selector's first linear, budget
+                    # and selector; then the selection fused with the compaction
+                    n += 12 + 1
                 elif pruned and l in prune:
                     j = prune.index(l)
                     P.dora_gather_scores(inp["tables"][j][L["i0"]:L["i1"]], c["ids"], c["cu"],

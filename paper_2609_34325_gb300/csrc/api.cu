@@ -532,7 +532,11 @@ static int pruned_block_impl(const dora_bf16* x_in, const int32_t* cu_in, const 
   if (launch_linear(o, t_cap, rows_in, d, w->w_proj, d, DORA_EPI_BIAS_RESIDUAL, e_proj, hattn,
                     status, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
-  if (launch_merge_moments(sm, t_cap, rows_in, d / kSliceCols, mv, stream) != cudaSuccess)
+  // LayerNorm' reads the row moments of H_attn; with a deletion only the kept
+  // rows', which the compaction merges from the slice moments itself
+  const bool deleting = scores != nullptr || hook != nullptr;
+  if (!deleting &&
+      launch_merge_moments(sm, t_cap, rows_in, d / kSliceCols, mv, stream) != cudaSuccess)
     return DORA_ERR_CUDA;
   // the actor reads this block's keys (Sec. 3.2; deletion follows the
   // attention residual, Eq. 1)
@@ -551,8 +555,8 @@ static int pruned_block_impl(const dora_bf16* x_in, const int32_t* cu_in, const 
   const int32_t* rows_mid = rows_in;
   if (scores) {
     if (launch_select_compact(scores, cu_in, keep_counts, batch, max_seqlen, hattn, d, t_cap,
-                              ids_in, mv, kept, cu_out, hkeep, ids_out, mv2, status,
-                              stream) != cudaSuccess)
+                              ids_in, sm, kept, cu_out, hkeep, ids_out, mv2, status, stream,
+                              d / kSliceCols) != cudaSuccess)
       return DORA_ERR_CUDA;
     hk = hkeep;
     rows_mid = cu_out + batch;

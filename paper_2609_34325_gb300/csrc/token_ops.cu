@@ -116,14 +116,53 @@ __device__ __forceinline__ int clamped_keep(int lo, int n, int m, int max_seqlen
 constexpr int kRadixBins = 256;
 static_assert(kSelectThreads == kRadixBins, "one histogram bin per thread");
 
+// Row moments (mean, var) of one row from its S slice moments (mean_s, M2_s)
+// over 64 columns each, stored slice-major with `stride` rows between slices:
+// mean = (1/S) sum mean_s, M2 = sum (M2_s + 64 (mean_s - mean)^2) (the
+// pairwise update of Chan, Golub & LeVeque with equal counts), var = M2 / (64 S).
+// Every rounding is explicit, so each caller gets the same bits.
+__device__ __forceinline__ float2 merge_slice_moments(const float2* __restrict__ p, size_t stride,
+                                                      int slices) {
+  constexpr int kHeld = 16;     // slices held in registers (dim <= 1024): one round of loads
+  const float inv_s = __frcp_rn(static_cast<float>(slices));
+  float mean, m2 = 0.f;
+  if (slices <= kHeld) {
+    float2 t[kHeld];
+#pragma unroll
+    for (int j = 0; j < kHeld; ++j)
+      if (j < slices) t[j] = __ldg(p + j * stride);
+    float sum = 0.f;
+#pragma unroll
+    for (int j = 0; j < kHeld; ++j)
+      if (j < slices) sum = __fadd_rn(sum, t[j].x);
+    mean = __fmul_rn(sum, inv_s);
+#pragma unroll
+    for (int j = 0; j < kHeld; ++j)
+      if (j < slices) {
+        const float d = __fsub_rn(t[j].x, mean);
+        m2 = __fadd_rn(m2, __fmaf_rn(__fmul_rn(static_cast<float>(kSliceCols), d), d, t[j].y));
+      }
+  } else {
+    float sum = 0.f;
+    for (int j = 0; j < slices; ++j) sum = __fadd_rn(sum, __ldg(p + j * stride).x);
+    mean = __fmul_rn(sum, inv_s);
+    for (int j = 0; j < slices; ++j) {
+      const float2 t = __ldg(p + j * stride);
+      const float d = __fsub_rn(t.x, mean);
+      m2 = __fadd_rn(m2, __fmaf_rn(__fmul_rn(static_cast<float>(kSliceCols), d), d, t.y));
+    }
+  }
+  return make_float2(mean, __fmul_rn(__fmul_rn(m2, inv_s), 1.0f / kSliceCols));
+}
+
 template <int CPL>
 __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
     const float* __restrict__ scores, const int32_t* __restrict__ cu_in,
     const int32_t* __restrict__ keep_counts, int32_t batch, int32_t max_seqlen, int32_t t_cap,
     int32_t splits, int32_t* __restrict__ kept_idx, int32_t* __restrict__ cu_out,
     const uint4* __restrict__ x, int32_t chunks, const int32_t* __restrict__ ids_in,
-    const float2* __restrict__ mv_in, uint4* __restrict__ packed, int32_t* __restrict__ ids_out,
-    float2* __restrict__ mv_out, int32_t* status) {
+    const float2* __restrict__ mv_in, int32_t mv_slices, uint4* __restrict__ packed,
+    int32_t* __restrict__ ids_out, float2* __restrict__ mv_out, int32_t* status) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ uint32_t keys[];            // [max_seqlen] keys, then [max_seqlen] kept rows
@@ -281,12 +320,18 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
           if (two) dst2[c] = v2[q];
         }
       }
+      // row moments of the kept rows: copied, or merged from the slice
+      // moments the producing linear wrote (mv_slices > 0)
       if (lane == 0) {
         if (ids_out != nullptr) ids_out[off + r] = ids_in[s1];
-        if (mv_out != nullptr) mv_out[off + r] = mv_in[s1];
+        if (mv_out != nullptr)
+          mv_out[off + r] = mv_slices > 0 ? merge_slice_moments(mv_in + s1, cap, mv_slices)
+                                          : mv_in[s1];
       } else if (lane == 1 && two) {
         if (ids_out != nullptr) ids_out[off + r2] = ids_in[s2];
-        if (mv_out != nullptr) mv_out[off + r2] = mv_in[s2];
+        if (mv_out != nullptr)
+          mv_out[off + r2] = mv_slices > 0 ? merge_slice_moments(mv_in + s2, cap, mv_slices)
+                                           : mv_in[s2];
       }
     }
   }
@@ -541,9 +586,7 @@ __global__ void __launch_bounds__(kRowThreads) row_stats_kernel(
   }
 }
 
-// One thread per row: mean = (1/S) sum mean_s, M2 = sum (M2_s + 64 (mean_s -
-// mean)^2) over the row's S slices of 64 (the pairwise update of Chan, Golub
-// & LeVeque with equal counts), var = M2 / (64 S).
+// One thread per row: the row's slice moments merged (merge_slice_moments).
 __global__ void __launch_bounds__(256) merge_moments_kernel(const float2* __restrict__ sm,
                                                             int32_t rows_cap,
                                                             const int32_t* __restrict__ rows_dev,
@@ -554,39 +597,8 @@ __global__ void __launch_bounds__(256) merge_moments_kernel(const float2* __rest
   int rows = rows_cap;
   if (rows_dev != nullptr) rows = min(rows_cap, max(0, *rows_dev));
   const size_t stride = static_cast<size_t>(rows_cap);
-  const float inv_s = 1.0f / static_cast<float>(slices);
-  constexpr int kHeld = 16;     // slices held in registers (dim <= 1024): one round of loads
-  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += gridDim.x * blockDim.x) {
-    const float2* p = sm + r;
-    float mean, m2 = 0.f;
-    if (slices <= kHeld) {
-      float2 t[kHeld];
-#pragma unroll
-      for (int j = 0; j < kHeld; ++j)
-        if (j < slices) t[j] = __ldg(p + j * stride);
-      float sum = 0.f;
-#pragma unroll
-      for (int j = 0; j < kHeld; ++j)
-        if (j < slices) sum += t[j].x;
-      mean = sum * inv_s;
-#pragma unroll
-      for (int j = 0; j < kHeld; ++j)
-        if (j < slices) {
-          const float d = t[j].x - mean;
-          m2 += t[j].y + static_cast<float>(kSliceCols) * d * d;
-        }
-    } else {
-      float sum = 0.f;
-      for (int j = 0; j < slices; ++j) sum += __ldg(p + j * stride).x;
-      mean = sum * inv_s;
-      for (int j = 0; j < slices; ++j) {
-        const float2 t = __ldg(p + j * stride);
-        const float d = t.x - mean;
-        m2 += t.y + static_cast<float>(kSliceCols) * d * d;
-      }
-    }
-    mv[r] = make_float2(mean, m2 * inv_s * (1.0f / kSliceCols));
-  }
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += gridDim.x * blockDim.x)
+    mv[r] = merge_slice_moments(sm + r, stride, slices);
 }
 
 // ---------------------------------------------------------------------------
@@ -690,7 +702,7 @@ cudaError_t launch_select_keep(const float* scores, const int32_t* cu_in,
   return launch_pdl(select_keep_kernel<0>, dim3(batch), dim3(kSelectThreads), smem, stream,
                     scores, cu_in, keep_counts, batch, max_seqlen, -1, 1, kept_idx,
                     cu_out, static_cast<const uint4*>(nullptr), 0,
-                    static_cast<const int32_t*>(nullptr), static_cast<const float2*>(nullptr),
+                    static_cast<const int32_t*>(nullptr), static_cast<const float2*>(nullptr), 0,
                     static_cast<uint4*>(nullptr), static_cast<int32_t*>(nullptr),
                     static_cast<float2*>(nullptr), status);
 }
@@ -712,9 +724,9 @@ static cudaError_t select_compact_cpl(const float* scores, const int32_t* cu_in,
                                       const int32_t* keep_counts, int32_t batch,
                                       int32_t max_seqlen, const uint16_t* x, int32_t chunks,
                                       int32_t t_in_cap, const int32_t* ids_in,
-                                      const float* mv_in, int32_t* kept_idx, int32_t* cu_out,
-                                      uint16_t* packed, int32_t* ids_out, float* mv_out,
-                                      int32_t* status, cudaStream_t stream) {
+                                      const float* mv_in, int32_t mv_slices, int32_t* kept_idx,
+                                      int32_t* cu_out, uint16_t* packed, int32_t* ids_out,
+                                      float* mv_out, int32_t* status, cudaStream_t stream) {
   size_t smem = 0;
   cudaError_t e = select_smem(reinterpret_cast<const void*>(select_keep_kernel<CPL>),
                               max_seqlen, &smem);
@@ -726,8 +738,9 @@ static cudaError_t select_compact_cpl(const float* scores, const int32_t* cu_in,
                     dim3(kSelectThreads), smem, stream, scores, cu_in, keep_counts, batch,
                     max_seqlen, t_in_cap, splits, kept_idx, cu_out,
                     reinterpret_cast<const uint4*>(x), chunks, ids_in,
-                    reinterpret_cast<const float2*>(mv_in), reinterpret_cast<uint4*>(packed),
-                    ids_out, reinterpret_cast<float2*>(mv_out), status);
+                    reinterpret_cast<const float2*>(mv_in), mv_slices,
+                    reinterpret_cast<uint4*>(packed), ids_out, reinterpret_cast<float2*>(mv_out),
+                    status);
 }
 
 cudaError_t launch_select_compact(const float* scores, const int32_t* cu_in,
@@ -735,25 +748,26 @@ cudaError_t launch_select_compact(const float* scores, const int32_t* cu_in,
                                   const uint16_t* x, int32_t dim, int32_t t_in_cap,
                                   const int32_t* ids_in, const float* mv_in, int32_t* kept_idx,
                                   int32_t* cu_out, uint16_t* packed, int32_t* ids_out,
-                                  float* mv_out, int32_t* status, cudaStream_t stream) {
+                                  float* mv_out, int32_t* status, cudaStream_t stream,
+                                  int32_t mv_slices) {
   if (batch == 0) return cudaSuccess;
   const int chunks = dim / 8;
   switch ((chunks + 31) / 32) {
     case 1: return select_compact_cpl<1>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
-                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         t_in_cap, ids_in, mv_in, mv_slices, kept_idx, cu_out, packed, ids_out,
                                          mv_out, status, stream);
     case 2: return select_compact_cpl<2>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
-                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         t_in_cap, ids_in, mv_in, mv_slices, kept_idx, cu_out, packed, ids_out,
                                          mv_out, status, stream);
     case 3: return select_compact_cpl<3>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
-                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         t_in_cap, ids_in, mv_in, mv_slices, kept_idx, cu_out, packed, ids_out,
                                          mv_out, status, stream);
     case 4: return select_compact_cpl<4>(scores, cu_in, keep_counts, batch, max_seqlen, x, chunks,
-                                         t_in_cap, ids_in, mv_in, kept_idx, cu_out, packed, ids_out,
+                                         t_in_cap, ids_in, mv_in, mv_slices, kept_idx, cu_out, packed, ids_out,
                                          mv_out, status, stream);
     default: return select_compact_cpl<kMaxChunksPerLane>(
         scores, cu_in, keep_counts, batch, max_seqlen, x, chunks, t_in_cap, ids_in, mv_in,
-        kept_idx, cu_out, packed, ids_out, mv_out, status, stream);
+        mv_slices, kept_idx, cu_out, packed, ids_out, mv_out, status, stream);
   }
 }
 

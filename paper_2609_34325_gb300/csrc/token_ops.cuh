@@ -47,13 +47,17 @@ cudaError_t launch_select_keep(const float* scores, const int32_t* cu_in,
 // Selection fused with the compaction of the kept rows (ids_in/ids_out and
 // mv_in/mv_out nullable in pairs): the same kept_idx and cu_out as
 // launch_select_keep, then packed[r] = x[kept_idx[r]], ids and row moments.
+// mv_slices = 0: mv_in holds row moments [t_in_cap][2], copied; mv_slices =
+// S > 0: mv_in holds the rows' slice moments [S][t_in_cap][2], merged per
+// kept row (the same bits as launch_merge_moments).
 int select_compact_splits(int32_t batch, int32_t max_seqlen);
 cudaError_t launch_select_compact(const float* scores, const int32_t* cu_in,
                                   const int32_t* keep_counts, int32_t batch, int32_t max_seqlen,
                                   const uint16_t* x, int32_t dim, int32_t t_in_cap,
                                   const int32_t* ids_in, const float* mv_in, int32_t* kept_idx,
                                   int32_t* cu_out, uint16_t* packed, int32_t* ids_out,
-                                  float* mv_out, int32_t* status, cudaStream_t stream);
+                                  float* mv_out, int32_t* status, cudaStream_t stream,
+                                  int32_t mv_slices = 0);
 
 // ln_out (LayerNorm' of the kept rows) is nullable; so is mv_out, which
 // receives mv_in[kept_idx[r]] (row moments, below) for every packed row r.
