@@ -123,28 +123,29 @@ static_assert(kSelectThreads == kRadixBins, "one histogram bin per thread");
 // Every rounding is explicit, so each caller gets the same bits.
 __device__ __forceinline__ float2 merge_slice_moments(const float2* __restrict__ p, size_t stride,
                                                       int slices) {
-  constexpr int kHeld = 16;     // slices held in registers (dim <= 1024): one round of loads
+  constexpr int kHeld = 16;     // slice means held in registers (dim <= 1024)
   const float inv_s = __frcp_rn(static_cast<float>(slices));
   float mean, m2 = 0.f;
   if (slices <= kHeld) {
-    float2 t[kHeld];
+    float mu[kHeld];
 #pragma unroll
     for (int j = 0; j < kHeld; ++j)
-      if (j < slices) t[j] = __ldg(p + j * stride);
+      if (j < slices) mu[j] = __ldg(&p[j * stride].x);
     float sum = 0.f;
 #pragma unroll
     for (int j = 0; j < kHeld; ++j)
-      if (j < slices) sum = __fadd_rn(sum, t[j].x);
+      if (j < slices) sum = __fadd_rn(sum, mu[j]);
     mean = __fmul_rn(sum, inv_s);
 #pragma unroll
     for (int j = 0; j < kHeld; ++j)
-      if (j < slices) {
-        const float d = __fsub_rn(t[j].x, mean);
-        m2 = __fadd_rn(m2, __fmaf_rn(__fmul_rn(static_cast<float>(kSliceCols), d), d, t[j].y));
+      if (j < slices) {             // the M2 halves are read again (L1)
+        const float d = __fsub_rn(mu[j], mean);
+        m2 = __fadd_rn(m2, __fmaf_rn(__fmul_rn(static_cast<float>(kSliceCols), d), d,
+                                     __ldg(&p[j * stride].y)));
       }
   } else {
     float sum = 0.f;
-    for (int j = 0; j < slices; ++j) sum = __fadd_rn(sum, __ldg(p + j * stride).x);
+    for (int j = 0; j < slices; ++j) sum = __fadd_rn(sum, __ldg(&p[j * stride].x));
     mean = __fmul_rn(sum, inv_s);
     for (int j = 0; j < slices; ++j) {
       const float2 t = __ldg(p + j * stride);
@@ -320,20 +321,20 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
           if (two) dst2[c] = v2[q];
         }
       }
-      // row moments of the kept rows: copied, or merged from the slice
-      // moments the producing linear wrote (mv_slices > 0)
       if (lane == 0) {
         if (ids_out != nullptr) ids_out[off + r] = ids_in[s1];
-        if (mv_out != nullptr)
-          mv_out[off + r] = mv_slices > 0 ? merge_slice_moments(mv_in + s1, cap, mv_slices)
-                                          : mv_in[s1];
+        if (mv_out != nullptr && mv_slices == 0) mv_out[off + r] = mv_in[s1];
       } else if (lane == 1 && two) {
         if (ids_out != nullptr) ids_out[off + r2] = ids_in[s2];
-        if (mv_out != nullptr)
-          mv_out[off + r2] = mv_slices > 0 ? merge_slice_moments(mv_in + s2, cap, mv_slices)
-                                           : mv_in[s2];
+        if (mv_out != nullptr && mv_slices == 0) mv_out[off + r2] = mv_in[s2];
       }
     }
+    // row moments merged from the slice moments the producing linear wrote
+    // (mv_slices > 0): one thread per kept row, apart from the row copies so
+    // that the merge's registers do not weigh on them
+    if (mv_out != nullptr && mv_slices > 0)
+      for (int q = part * blockDim.x + tid; q < rows; q += splits * blockDim.x)
+        mv_out[off + q] = merge_slice_moments(mv_in + kept_rows[q], cap, mv_slices);
   }
 }
 
