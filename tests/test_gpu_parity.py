@@ -496,6 +496,27 @@ def _ln_rows(rng, rows, dim):
     return S.f32_to_bf16_bits(off + sd * rng.standard_normal((rows, dim)))
 
 
+@pytest.mark.parametrize("slices", [1, 3, 12, 16, 17, 32])
+def test_merge_moments_slice_counts(slices):
+    """Row moments merged from 64-column slice moments: the held path (up to
+    16 slices in registers) and the streaming one past it, rows past the live
+    count untouched."""
+    rng = np.random.default_rng(40 + slices)
+    rows, live = 300, 257
+    xb = _ln_rows(rng, rows, 64 * slices)
+    v = O.bf16_to_f64(xb).reshape(rows, slices, 64)
+    s_mean = v.mean(axis=2)
+    s_m2 = ((v - s_mean[..., None]) ** 2).sum(axis=2)
+    sm = np.stack([s_mean, s_m2], axis=2).transpose(1, 0, 2).astype(np.float32)   # [S, rows, 2]
+    sm_d = torch.from_numpy(np.ascontiguousarray(sm)).to(dev())
+    mv = torch.full((rows, 2), -3.0, dtype=torch.float32, device=dev())
+    P.dora_merge_moments(sm_d, mv, rows_dev=i32([live]))
+    torch.cuda.synchronize()
+    got = mv.cpu().numpy().astype(np.float64)
+    assert np.all(got[live:] == -3.0)
+    _check_row_moments(got[:live], xb[:live], f"merged moments, {slices} slices")
+
+
 @pytest.mark.parametrize("dim", [64, 192, 768, 1024, 2048])
 def test_row_stats(dim):
     rng = np.random.default_rng(dim + 1)
