@@ -849,6 +849,34 @@ def test_block_full_oracle(name):
     assert np.array_equal(bits(r["x_out"][:t_out]), bits(r0["x_out"])[ref["kept_idx"]])
 
 
+@pytest.mark.parametrize("name", ["cfg1", "cfg3"])
+def test_block_tiny_batch(name):
+    """Fewer rows than one 256-row tile pair, before and after the deletion
+    (the linears' row walks, forward and from the last row block, meet a
+    single partial row block), with a one-token image; the one-CTA-pair path
+    (D = 768) and the one-CTA path (D = 192)."""
+    cfg = S.get_config(name, batch=3)
+    lens = np.array([5, 1, 40])
+    cu = O.cu_from_counts(lens)
+    ids = np.concatenate([np.arange(n) for n in lens]).astype(np.int32)
+    rng = np.random.default_rng(61)
+    x = S.f32_to_bf16_bits(rng.standard_normal((int(cu[-1]), cfg.dim)))
+    wb = S.block_weights(cfg, 0, 61, random_affine=True)
+    w = _device_weights(cfg, wb)
+    scores = rng.random(int(cu[-1])).astype(np.float32)
+    keeps = np.array([2, 1, 7], dtype=np.int32)
+    wf = O.decode_weights(wb)
+    for sc, kp in ((scores, keeps), (None, None)):
+        r = _run_block(cfg, x, cu, ids, w, sc, kp)
+        assert r["status"] == 0
+        ref = O.pruned_block(O.bf16_to_f64(x), cu, ids, wf, cfg.heads, cfg.ln_eps, sc, kp)
+        t_out = int(ref["cu_out"][-1]) if sc is not None else int(cu[-1])
+        if sc is not None:
+            assert np.array_equal(r["cu_out"], ref["cu_out"])
+            assert np.array_equal(r["kept"][:t_out], ref["kept_idx"])
+        assert_close(f64(r["x_out"][:t_out]), ref["x_out"], f"tiny block {name}")
+
+
 def test_block_prefolded_weights_give_the_same_bits():
     """Weights folded once (dora_fold_block_weights) and weights folded inside
     every call produce the same block output bit for bit."""
