@@ -1,6 +1,7 @@
 """Micro-benchmark of one block's kernels through the C ABI.
 
     python -m paper_2609_34325_gb300.microbench [--images 256] [--iters 20]
+    python -m paper_2609_34325_gb300.microbench --mixes cfg6 [--iters 20]
 
 Times, with CUDA events on the launching stream, the QKV linear with
 LayerNorm folded in, the projection and fc2 with their residuals (and the
@@ -11,6 +12,14 @@ attention over `images` images of `tokens` tokens.  Prints one line per
 kernel: microseconds per launch and TFLOP/s.  It is also the small case for
 profiling one launch of a kernel: the linears run in that order, each
 warmup + iters launches, then the attention.
+
+With ``--mixes CFG`` it times only the varlen attention, on the length mixes
+of that configuration's seeded deletion schedule (the full-length batch, then
+the batch after each pruning block), each twice: with max_seqlen set to the
+mix's own longest image and to the configuration's token count N.  The
+attention picks its kernel from max_seqlen (the short-image kernel up to 256,
+the per-key-half kernel beyond), so the two lines show what a caller that
+knows the kept maximum would gain over one that passes N.
 """
 from __future__ import annotations
 
@@ -31,7 +40,46 @@ def _args(argv):
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--mixes", default=None,
+                    help="time the attention on this configuration's length mixes instead")
     return ap.parse_args(argv)
+
+
+def _time(fn, warmup, iters, stream):
+    for _ in range(warmup):
+        fn()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(iters):
+        fn()
+    e1.record(stream)
+    e1.synchronize()
+    return 1000.0 * e0.elapsed_time(e1) / iters
+
+
+def attention_mixes(a, dev):
+    """Varlen attention on each length mix of a configuration's seeded schedule."""
+    import numpy as np
+
+    import dora_synth as S
+
+    cfg = S.get_config(a.mixes)
+    keeps, _ = S.keep_schedule(cfg, a.seed)
+    mixes = [np.full(cfg.batch, cfg.n_tokens, dtype=np.int64)] + [k.astype(np.int64) for k in keeps]
+    heads, d = cfg.heads, cfg.dim
+    t_cap = cfg.batch * cfg.n_tokens
+    g = torch.Generator(device=dev).manual_seed(a.seed)
+    qkv = torch.randn(t_cap, 3 * d, generator=g, device=dev).to(torch.bfloat16)
+    o = torch.empty(t_cap, d, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream()
+    for j, lens in enumerate(mixes):
+        cu = torch.from_numpy(np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)).to(dev)
+        flops = 4.0 * float((lens * lens).sum()) * cfg.head_dim * heads
+        label = "full length" if j == 0 else f"after pruning {j}"
+        for msl in sorted({int(lens.max()), cfg.n_tokens}):
+            us = _time(lambda: dora_varlen_attn(qkv, cu, msl, heads, o), a.warmup, a.iters, stream)
+            print(f"{a.mixes} {label:18s} mean {lens.mean():6.1f} max {lens.max():4d} "
+                  f"max_seqlen {msl:4d}: {us:8.1f} us  {flops / (us * 1e-6) / 1e12:7.1f} TFLOP/s")
 
 
 def main(argv=None):
@@ -39,6 +87,9 @@ def main(argv=None):
     load_library()
     dev = torch.device("cuda:0")
     torch.cuda.set_device(dev)
+    if a.mixes is not None:
+        attention_mixes(a, dev)
+        return
     g = torch.Generator(device=dev).manual_seed(a.seed)
     bf16, f32 = torch.bfloat16, torch.float32
     T, D, F = a.images * a.tokens, a.dim, a.mlp
@@ -84,15 +135,7 @@ def main(argv=None):
     stream = torch.cuda.current_stream()
     torch.cuda.synchronize()
     for name, n, k, fn in runs:
-        for _ in range(a.warmup):
-            fn()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(a.iters):
-            fn()
-        e1.record(stream)
-        e1.synchronize()
-        us = 1000.0 * e0.elapsed_time(e1) / a.iters
+        us = _time(fn, a.warmup, a.iters, stream)
         if n is None:         # attention: k holds its FLOPs
             shape, flops = f"{a.images} x {a.tokens} tokens x {heads} heads", k
         else:
