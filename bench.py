@@ -779,7 +779,13 @@ def profile_kernels(torch, P, cfg, hw, sets, blocks, dev, stream, t_cap, steps):
     """Run the pruned step launch by launch through the fine-grained entry
     points (the same kernels dora_pruned_block launches), bracketing each
     launch with CUDA events on the launching stream.  Returns per-class times
-    and algorithmic work."""
+    and algorithmic work.
+
+    One difference: at a pruning block dora_pruned_block merges the kept
+    rows' slice moments inside the fused selection and skips the
+    projection's merge launch; the public dora_select_compact takes row
+    moments, so this pass runs that merge launch (23 merges a DeiT-B step
+    against the block's 20) and its selection copies merged moments."""
     d, m = cfg.dim, cfg.mlp_dim
     bf16, f32 = torch.bfloat16, torch.float32
     sm = torch.zeros(d // 64, t_cap, 2, dtype=f32, device=dev)      # slice moments
