@@ -29,8 +29,10 @@
 //              memory (64-byte swizzle) and write it with a TMA tensor store.
 //              The residual epilogue gives each chunk its own buffer, into
 //              which a TMA load brings the residual chunk while the tile's
-//              MMAs still run; the result is written over it in place.  The
-//              tile that straddles the live row count stores row by row.
+//              MMAs still run; the result is written over it in place (a
+//              long-K linear keeps two buffers a warp and reloads them within
+//              the tile, for one more stage).  The tile that straddles the
+//              live row count stores row by row.
 // The live row count M may come from device memory (rows left after a
 // deletion); tiles past it are never scheduled.  Every wait is bounded.
 #include <cuda.h>
@@ -49,6 +51,14 @@ constexpr int BK = 64;
 constexpr int kCluster = 2;
 constexpr int kStageChunk = 32 * 32;   // one warp's 32 rows x 32 columns, bf16
 constexpr int kSmemLimit = 227 * 1024;
+// The residual epilogue of a long-K linear (K >= kLongK, fc2): two staging
+// buffers per epilogue warp instead of one per chunk, so the stage ring gets
+// one more stage.  The residual of a tile's first two chunks is loaded a tile
+// ahead as in the plain residual epilogue; that of the other two is loaded
+// into the first two's buffers once their stores have read them, inside an
+// epilogue that a long main loop leaves mostly idle.
+constexpr int kEpiResidualLongK = 5;
+constexpr int kLongK = 2048;
 
 // Per-instantiation layout.
 // Pair mode: one MMA of M = 256 spans both CTAs of the cluster, each holding
@@ -70,10 +80,13 @@ struct Cfg {
   static constexpr int kChunks = kCols / 32;
   // chunks per TMEM load: two (64 registers) unless 16 warps cap registers at 96
   static constexpr int kBatch = kEpiWarps == 16 ? 1 : (kChunks < 2 ? kChunks : 2);
-  static constexpr bool kResTma = EPI == DORA_EPI_BIAS_RESIDUAL;
+  static constexpr bool kResTma = EPI == DORA_EPI_BIAS_RESIDUAL || EPI == kEpiResidualLongK;
   // staging buffers per epilogue warp: one per chunk for the residual (its
-  // TMA load lands there), one with 16 warps or the folded LayerNorm, else two
-  static constexpr int kBufs = kResTma ? kChunks : ((kEpiWarps == 16 || kLn) ? 1 : 2);
+  // TMA load lands there; two for a long K), one with 16 warps or the folded
+  // LayerNorm, else two
+  static constexpr int kBufs =
+      kResTma ? (EPI == kEpiResidualLongK && kChunks > 2 ? 2 : kChunks)
+              : ((kEpiWarps == 16 || kLn) ? 1 : 2);
   // folded LayerNorm: each epilogue warp's c and d columns, staged per tile
   static constexpr int kCdCols = kLn ? kCols : 1;
   static constexpr int kThreads = 64 + 32 * kEpiWarps;
@@ -94,7 +107,7 @@ struct Smem {
   float cd[C::kEpiWarps][2][C::kCdCols];            // colsum, colbias of the warp's columns
   uint64_t full[C::kStages];
   uint64_t empty[C::kStages];
-  uint64_t res_full[C::kEpiWarps][C::kResTma ? C::kChunks : 1];
+  uint64_t res_full[C::kEpiWarps][C::kResTma ? C::kBufs : 1];
   uint64_t cd_full[C::kEpiWarps];
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
@@ -260,7 +273,7 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
       mbar_init(&s.acc_empty[i], kPair ? 2 * kEpiWarps : kEpiWarps);
     }
     for (int w = 0; w < kEpiWarps; ++w) {
-      for (int c = 0; c < (C::kResTma ? C::kChunks : 1); ++c) mbar_init(&s.res_full[w][c], 1);
+      for (int c = 0; c < (C::kResTma ? C::kBufs : 1); ++c) mbar_init(&s.res_full[w][c], 1);
       mbar_init(&s.cd_full[w], 1);
     }
     mbar_init(&s.drain, 1);
@@ -407,11 +420,20 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
     const int slot = ew >> 2;                     // which column slice
     const uint32_t lane_sel = static_cast<uint32_t>(q * 32) << 16;
     int buf = 0;                                  // staging buffer to write next
-    uint32_t res_pend = 0;                        // residual chunks in flight
+    uint32_t res_pend = 0;                        // staging buffers with a residual load in flight
     uint32_t res_par = 0;                         // their next completion parity
-    // Residual of the warp's whole 32-row chunks of tile pair `p`: one TMA
-    // load per chunk into the chunk's staging buffer, once the stores of the
-    // previous tile have read those buffers.
+    // Residual chunk `c` of the warp's 32 rows from row0, column col0 on, into
+    // staging buffer c % kBufs (whose previous store must have read it).
+    auto load_residual = [&](int c, int row0, int col0) {
+      const int b = c % kBufs;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&s.res_full[ew][b], kStageChunk * 2);
+        tma_load_2d(s.out[ew][b], &tmR, &s.res_full[ew][b], col0 + c * 32, row0);
+      }
+      res_pend |= 1u << b;
+    };
+    // Residual of the warp's whole 32-row chunks of tile pair `p` (the first
+    // kBufs chunks), once the stores of the previous tile have read the buffers.
     auto prefetch_residual = [&](int p) {
       const int row0 = (2 * mpair(p) + rank) * BM + q * 32;
       if (row0 + 32 > M) return;
@@ -419,13 +441,9 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
       if (lane == 0) bulk_wait_group_read0();
       __syncwarp();
 #pragma unroll
-      for (int c = 0; c < kChunks; ++c) {
+      for (int c = 0; c < kBufs; ++c) {
         if (col0 + c * 32 >= N) break;
-        if (lane == 0) {
-          mbar_arrive_expect_tx(&s.res_full[ew][c], kStageChunk * 2);
-          tma_load_2d(s.out[ew][c], &tmR, &s.res_full[ew][c], col0 + c * 32, row0);
-        }
-        res_pend |= 1u << c;
+        load_residual(c, row0, col0);
       }
     };
     // Slice moments of the rounded output row: the first chunk of a 64-column
@@ -529,14 +547,14 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
             // of row l sits at piece j ^ ((l >> 1) & 3).
             uint16_t* stage;
             if constexpr (C::kResTma) {
-              const int ch = cb + c;
-              stage = s.out[ew][ch];
-              if (!mbar_wait_warp(&s.res_full[ew][ch], (res_par >> ch) & 1u, abort)) {
+              const int rb = (cb + c) % kBufs;
+              stage = s.out[ew][rb];
+              if (!mbar_wait_warp(&s.res_full[ew][rb], (res_par >> rb) & 1u, abort)) {
                 ok = false;
                 break;
               }
-              res_par ^= 1u << ch;
-              res_pend &= ~(1u << ch);
+              res_par ^= 1u << rb;
+              res_pend &= ~(1u << rb);
             } else {
               // the store issued kBufs chunks ago from this buffer must have read it
               stage = s.out[ew][buf];
@@ -567,8 +585,18 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
               tma_store_2d(&tmY, stage, gcol, row0);
               bulk_commit_group();
             }
+            if constexpr (C::kResTma && kBufs < kChunks) {
+              // the chunk kBufs on goes into this buffer once the store has read it
+              const int nc = cb + c + kBufs;
+              const int col0 = nt * BN + slot * kCols;
+              if (nc < kChunks && col0 + nc * 32 < N) {
+                if (lane == 0) bulk_wait_group_read0();
+                __syncwarp();
+                load_residual(nc, row0, col0);
+              }
+            }
           } else if (row < M) {
-            if constexpr (EPI == DORA_EPI_BIAS_RESIDUAL) {
+            if constexpr (C::kResTma) {
               const uint4* rp =
                   reinterpret_cast<const uint4*>(ep.residual + static_cast<size_t>(row) * N + gcol);
 #pragma unroll
@@ -593,7 +621,7 @@ __global__ void __launch_bounds__(Cfg<BN, EPI, PAIR>::kThreads, 1)
     if (lane == 0) {
       bulk_wait_group0();                         // stores done before the CTA exits
       // after an abort: residual loads issued but never consumed land first
-      for (int c = 0; c < kChunks; ++c)
+      for (int c = 0; c < kBufs; ++c)
         if (res_pend & (1u << c))
           mbar_wait_limited(&s.res_full[ew][c], (res_par >> c) & 1u, 100ull * 1000 * 1000);
       if (cd_pend) mbar_wait_limited(&s.cd_full[ew], cd_par, 100ull * 1000 * 1000);
@@ -627,6 +655,7 @@ static cudaError_t launch_bn_epi(const CUtensorMap& ta, const CUtensorMap& tb,
                                  const CUtensorMap& ty, const CUtensorMap& tr, uint16_t* y,
                                  const LinearEpi& ep, int m_cap, const int32_t* m_dev, int n,
                                  int k, int32_t* status, cudaStream_t stream) {
+  static_assert(sizeof(Smem<BN, EPI, PAIR>) <= kSmemLimit, "shared memory");
   const size_t smem = sizeof(Smem<BN, EPI, PAIR>);
   auto kern = gemm_kernel<BN, EPI, PAIR>;
   cudaError_t e =
@@ -679,6 +708,9 @@ static cudaError_t launch_bn(const CUtensorMap& ta, const CUtensorMap& tb, const
     case DORA_EPI_BIAS_RESIDUAL:
       return launch_bn_epi<BN, DORA_EPI_BIAS_RESIDUAL, kPair>(ta, tb, ty, tr, y, ep, m_cap, m_dev,
                                                               n, k, status, stream);
+    case kEpiResidualLongK:
+      return launch_bn_epi<BN, kEpiResidualLongK, kPair>(ta, tb, ty, tr, y, ep, m_cap, m_dev, n,
+                                                         k, status, stream);
     case kEpiLn:
       return launch_bn_epi<BN, kEpiLn, kPair>(ta, tb, ty, tr, y, ep, m_cap, m_dev, n, k, status,
                                               stream);
@@ -715,9 +747,12 @@ cudaError_t launch_linear(const uint16_t* x, int32_t m_cap, const int32_t* m_dev
       encode_tmap_2d_bf16(&tr, ep.residual, static_cast<uint64_t>(n), static_cast<uint64_t>(m_cap),
                           static_cast<uint64_t>(n) * 2, 32, 32, 64) != 0)
     return cudaErrorInvalidValue;
-  if (bn == 256)
-    return gemm::launch_bn<256>(ta, tb, ty, tr, y, ep, epilogue, m_cap, m_dev, n, k, status,
-                                stream);
+  if (bn == 256) {
+    const int epi = (epilogue == DORA_EPI_BIAS_RESIDUAL && k >= gemm::kLongK)
+                        ? gemm::kEpiResidualLongK
+                        : epilogue;
+    return gemm::launch_bn<256>(ta, tb, ty, tr, y, ep, epi, m_cap, m_dev, n, k, status, stream);
+  }
   return gemm::launch_bn<128>(ta, tb, ty, tr, y, ep, epilogue, m_cap, m_dev, n, k, status, stream);
 }
 
