@@ -663,6 +663,43 @@ def test_linear_residual_stats(m_cap, m_live, k, n):
     _check_row_moments(mv.cpu().numpy().astype(np.float64)[:m_live], yb, "merged moments")
 
 
+@pytest.mark.parametrize("m_cap,m_live", [(20000, 19999), (20224, 20224)])
+def test_linear_residual_long_k_many_tiles(m_cap, m_live):
+    """A long-K residual linear (K = 3072, the fc2 shape) over enough rows
+    that every CTA pair runs several tiles, so each warp's two staging
+    buffers are reloaded within a tile and reused across tiles: sampled rows
+    against the fp64 oracle, every row and slice moment against the plain
+    residual entry point bit for bit, and the rows past the live count
+    untouched."""
+    k, n = 3072, 768
+    rng = np.random.default_rng(m_cap + 31)
+    x = S.f32_to_bf16_bits(rng.standard_normal((m_cap, k)))
+    w = S.f32_to_bf16_bits(0.02 * rng.standard_normal((n, k)))
+    b = S.f32_to_bf16_bits(0.1 * rng.standard_normal(n))
+    r = _ln_rows(rng, m_cap, n)
+    m_dev = i32([m_live])
+    y = torch.full((m_cap, n), 7.0, dtype=torch.bfloat16, device=dev())
+    y2 = torch.full((m_cap, n), 7.0, dtype=torch.bfloat16, device=dev())
+    sm = torch.full((n // 64, m_cap, 2), -3.0, dtype=torch.float32, device=dev())
+    st = _status()
+    P.dora_linear_residual_stats(bf(x), bf(w), bf(r), y, sm, bias=bf(b), m_dev=m_dev, status=st)
+    P.dora_linear(bf(x), bf(w), y2, bias=bf(b), residual=bf(r), epilogue=P.EPI_BIAS_RESIDUAL,
+                  m_dev=m_dev)
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert torch.equal(y, y2)
+    assert torch.all(y[m_live:] == 7.0)
+    assert torch.all(sm[:, m_live:] == -3.0)
+    rows = np.unique(np.concatenate([rng.integers(0, m_live, 250), [0, m_live - 1]]))
+    ref = O.linear(O.bf16_to_f64(x[rows]), O.bf16_to_f64(w), O.bf16_to_f64(b)) + O.bf16_to_f64(r[rows])
+    assert_close(f64(y[torch.from_numpy(rows).to(dev())]), ref, f"long-K residual {m_cap}")
+    v = O.bf16_to_f64(bits(y[torch.from_numpy(rows).to(dev())])).reshape(len(rows), n // 64, 64)
+    got = sm.cpu().numpy().astype(np.float64).transpose(1, 0, 2)[rows]
+    s_mean = v.mean(axis=2)
+    s_scale = np.abs(v).max(axis=2)
+    assert np.all(np.abs(got[:, :, 0] - s_mean) <= 4e-6 * s_scale + 1e-30)
+
+
 # ---------------------------------------------------------------------------
 # varlen attention (tcgen05)
 # ---------------------------------------------------------------------------
