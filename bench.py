@@ -64,8 +64,8 @@ NCU_GEMM_BYTES_PER_ROW = {
 NCU_TRAFFIC_SELECT_COMPACT = {
     # profiles/select_compact_tokens.md: mean of 3 launches, 256 x 197 tokens,
     # D = 768, 34,284 rows kept (106.5 MB algorithmic)
-    "aff5318b6fb178805ad3ba9d1e7c68ff4d149d4aa8e548d1f9665121d11a0748": {
-        "traffic": 59440043, "case": "micro-benchmark: 256 x 197 tokens, D = 768, 34284 kept "
+    "649eef5b074bfadcdf5bd8b3ba07099ee9032bd7c2c64f8680288f9c33f8e844": {
+        "traffic": 59518976, "case": "micro-benchmark: 256 x 197 tokens, D = 768, 34284 kept "
                                      "rows, inputs cycled beyond 2 x L2"},
 }
 

@@ -95,12 +95,13 @@ __device__ __forceinline__ int clamped_keep(int lo, int n, int m, int max_seqlen
 // compaction of the kept rows
 // ---------------------------------------------------------------------------
 // Work of one CTA (kSelectThreads threads) for image i = blockIdx.x / splits:
-//  1. its output offset, the sum of the clamped keep counts of images < i;
-//  2. the image's candidate keys (ordered uint32 of the deletion scores) in
-//     shared memory;
+//  1. its output offset, the sum of the clamped keep counts of images < i,
+//  2. and, in the same round of loads, the image's candidate keys (ordered
+//     uint32 of the deletion scores) in shared memory;
 //  3. radix select, 8 bits a pass from the top: the key T of the
 //     (m-1)-th smallest candidate and how many candidates equal to T are
-//     kept (the lowest-indexed ones: ties are broken by index);
+//     kept (the lowest-indexed ones: ties are broken by index); once a
+//     single candidate has T's prefix, its key is T and the passes stop;
 //  4. one block-wide scan over contiguous index segments of the packed
 //     counts (candidates below T, candidates equal to T), which gives every
 //     kept token its output position in index order;
@@ -172,6 +173,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
   __shared__ int hist[kRadixBins];
   __shared__ uint32_t sel_prefix;
   __shared__ int sel_rank;
+  __shared__ int sel_count;
+  __shared__ uint32_t sel_key;
   const int i = blockIdx.x / splits;
   const int part = blockIdx.x - i * splits;
   const int tid = threadIdx.x;
@@ -180,25 +183,22 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
   // when the caller gives none
   const int cap = t_cap >= 0 ? t_cap : cu_in[batch];
 
-  // 1. output offset of this image; the image's own bounds and keep count
-  // come in the same round of loads (the thread that reads entry i shares them)
-  __shared__ int own[3];
-  int acc = 0;
-  for (int t = tid; t <= i; t += blockDim.x) {
-    const int l0 = cu_in[t], l1 = cu_in[t + 1], kt = keep_counts[t];
-    if (t < i) {
-      acc += clamped_keep(l0, l1 - l0, kt, max_seqlen, cap);
-    } else {
-      own[0] = l0;
-      own[1] = l1 - l0;
-      own[2] = kt;
-    }
-  }
-  const int off = block_sum(acc, scratch);   // its barriers publish own[]
-  const int lo = own[0];
-  const int n = own[1];
-  const int m = own[2];
+  // 1-2. the image's own bounds and keep count (every thread reads the same
+  // three words), its candidate keys into shared memory, and its output
+  // offset, the sum of the clamped keep counts of the images before it: the
+  // loads of the keys and of the offset's terms go out in one round
+  const int lo = cu_in[i];
+  const int n = cu_in[i + 1] - lo;
+  const int m = keep_counts[i];
   const int me = clamped_keep(lo, n, m, max_seqlen, cap);
+  if (me > 0)                                   // the rows lie inside the input
+    for (int j = tid; j < n; j += blockDim.x) keys[j] = score_key(scores[lo + j]);
+  int acc = 0;
+  for (int t = tid; t < i; t += blockDim.x) {
+    const int l0 = cu_in[t];
+    acc += clamped_keep(l0, cu_in[t + 1] - l0, keep_counts[t], max_seqlen, cap);
+  }
+  const int off = block_sum(acc, scratch);   // its barriers also publish the keys
   if (part == 0 && tid == 0) {
     // rows outside the input, or (boundaries not increasing) outputs past it
     if (n > max_seqlen || (n > 0 && (lo < 0 || lo > cap - n)) || off > cap - me)
@@ -209,10 +209,6 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
     if (i == 0) cu_out[0] = 0;
   }
   if (me == 0) return;
-
-  // 2. candidate keys
-  for (int j = tid; j < n; j += blockDim.x) keys[j] = score_key(scores[lo + j]);
-  __syncthreads();
 
   // 3. threshold key T and the number of candidates equal to T that are kept
   const int need = me - 1;                       // visual tokens kept
@@ -246,11 +242,21 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
       if (below < rank && rank <= below + c) {
         sel_prefix = prefix | (static_cast<uint32_t>(tid) << shift);
         sel_rank = rank - below;
+        sel_count = c;
       }
       __syncthreads();
       prefix = sel_prefix;
       rank = sel_rank;
       hi_mask |= 0xFFu << shift;
+      if (shift > 0 && sel_count == 1) {
+        // one candidate has this prefix: its key is the threshold (no other
+        // key equals it, so rank is 1) and the lower bytes need no pass
+        for (int j = tid; j < n; j += blockDim.x)
+          if (j >= 1 && ((keys[j] ^ prefix) & hi_mask) == 0u) sel_key = keys[j];
+        __syncthreads();
+        prefix = sel_key;
+        break;
+      }
     }
     thr = prefix;
     ties_keep = rank;
