@@ -79,22 +79,39 @@ def _edge_lengths():
     return np.array([1, 2, 15, 16, 17, 31, 32, 33, 64, 127, 128, 129, 197, 255, 256, 257, 577])
 
 
-@pytest.mark.parametrize("kind", ["uniform", "ties", "special", "allequal"])
+def _edge_scores(rng, t, kind):
+    """Scores of one edge-case kind for t tokens."""
+    if kind == "uniform":
+        return rng.random(t).astype(np.float32)
+    if kind == "ties":
+        return rng.choice(np.array([0.0, 0.25, 0.5], np.float32), size=t)
+    if kind == "allequal":
+        return np.full(t, 0.125, np.float32)
+    if kind == "prefixes":
+        # positive floats whose bit patterns share their top one, two or
+        # three bytes, with exact duplicates: the threshold's prefix is
+        # unique after the first, second or third 8-bit pass, or never
+        b3 = rng.choice(np.array([0x3E, 0x3F], np.uint32), size=t)
+        b2 = rng.choice(np.array([0x00, 0x80], np.uint32), size=t)
+        b1 = rng.choice(np.array([0x10, 0x20, 0x30], np.uint32), size=t)
+        b0 = rng.integers(0, 256, size=t).astype(np.uint32)
+        s = ((b3 << 24) | (b2 << 16) | (b1 << 8) | b0).view(np.float32)
+        dup = rng.random(t) < 0.1
+        s[dup] = np.roll(s, 1)[dup]
+        return s
+    pal = np.array([0.0, -0.0, np.nan, -np.nan, np.inf, -np.inf, 1.0, -1.0, 1e-38, -1e-38],
+                   dtype=np.float32)
+    return rng.choice(pal, size=t)
+
+
+@pytest.mark.parametrize("kind", ["uniform", "ties", "special", "allequal", "prefixes"])
 def test_select_keep_edges(kind):
     rng = np.random.default_rng(42)
     lens = _edge_lengths()
     cu = O.cu_from_counts(lens)
     t = int(cu[-1])
-    if kind == "uniform":
-        s = rng.random(t).astype(np.float32)
-    elif kind == "ties":
-        s = rng.choice(np.array([0.0, 0.25, 0.5], np.float32), size=t)
-    elif kind == "allequal":
-        s = np.full(t, 0.125, np.float32)
-    else:
-        pal = np.array([0.0, -0.0, np.nan, -np.nan, np.inf, -np.inf, 1.0, -1.0, 1e-38, -1e-38],
-                       dtype=np.float32)
-        s = rng.choice(pal, size=t)
+    s = _edge_scores(rng, t, kind)
+    if kind == "special":
         s[rng.random(t) < 0.02] = np.float32(np.nan)
     for mode in ("one", "all", "random"):
         if mode == "one":
@@ -275,7 +292,7 @@ def test_select_compact_configs(name):
 
 
 @pytest.mark.parametrize("dim", [64, 192, 384, 768, 1024, 2048])
-@pytest.mark.parametrize("kind", ["uniform", "ties", "special", "allequal"])
+@pytest.mark.parametrize("kind", ["uniform", "ties", "special", "allequal", "prefixes"])
 def test_select_compact_edges(kind, dim):
     """Lengths 1..577 around the 16/32/128/256 boundaries, ties, signed
     zeros, NaN and infinities, keep one / all / random, every row width class
@@ -284,16 +301,7 @@ def test_select_compact_edges(kind, dim):
     lens = _edge_lengths()
     cu = O.cu_from_counts(lens)
     t = int(cu[-1])
-    if kind == "uniform":
-        s = rng.random(t).astype(np.float32)
-    elif kind == "ties":
-        s = rng.choice(np.array([0.0, 0.25, 0.5], np.float32), size=t)
-    elif kind == "allequal":
-        s = np.full(t, 0.125, np.float32)
-    else:
-        pal = np.array([0.0, -0.0, np.nan, -np.nan, np.inf, -np.inf, 1.0, -1.0, 1e-38, -1e-38],
-                       dtype=np.float32)
-        s = rng.choice(pal, size=t)
+    s = _edge_scores(rng, t, kind)
     x, ids, mv = _row_inputs(rng, t, dim)
     for n, mode in enumerate(("one", "all", "random")):
         if mode == "one":
