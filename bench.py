@@ -972,7 +972,8 @@ def roofline_report(kern, peaks, peak_src, workload):
     c = kern["select_compact"]
     c_gbs = c["bytes"] / (c["ms"] * 1e-3) / 1e9
     tok_src = os.path.join(ROOT, "paper_2609_34325_gb300", "csrc", "token_ops.cu")
-    ctr = NCU_TRAFFIC_SELECT_COMPACT.get(sha256_of(tok_src))
+    # the captured traffic is the DeiT-B case's; other shapes report none
+    ctr = NCU_TRAFFIC_SELECT_COMPACT.get(sha256_of(tok_src)) if workload == "cfg3" else None
     out["roofline_compact"] = {
         "kernel": "select_keep_kernel (selection fused with the compaction of the kept rows, "
                   "their ids and row moments)", "bound": "hbm",
