@@ -174,24 +174,32 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
         self.thread.join(timeout=2)
-        sm, mx, reasons = [], None, set()
-        for ts, ln in self.lines:
-            f = [x.strip() for x in ln.split(",")]
-            if len(f) < 9 or not (t0 - 0.05 <= ts <= t1 + 0.15):
-                continue
-            try:
-                sm.append(float(f[1]))
-                mx = float(f[2])
-            except ValueError:
-                continue
-            names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-            for name, v in zip(names, f[5:9]):
-                if v.lower().startswith("active"):
-                    reasons.add(name)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": [], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
-                "samples": len(sm)}
+        return clock_summary(self.lines, t0, t1)
+
+
+def clock_summary(lines, t0, t1):
+    """Median SM clock, the maximum clock and the throttle reasons seen in the
+    (arrival time, nvidia-smi CSV line) samples that fall in [t0, t1] (with a
+    little slack for the sampler's latency); lines that do not parse are
+    skipped."""
+    sm, mx, reasons = [], None, set()
+    for ts, ln in lines:
+        f = [x.strip() for x in ln.split(",")]
+        if len(f) < 9 or not (t0 - 0.05 <= ts <= t1 + 0.15):
+            continue
+        try:
+            sm.append(float(f[1]))
+            mx = float(f[2])
+        except ValueError:
+            continue
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for name, v in zip(names, f[5:9]):
+            if v.lower().startswith("active"):
+                reasons.add(name)
+    if not sm:
+        return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": [], "samples": 0}
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+            "samples": len(sm)}
 
 
 def device_tensors(torch, cfg, seed, n_sets, dev):
