@@ -96,7 +96,7 @@ __device__ __forceinline__ int clamped_keep(int lo, int n, int m, int max_seqlen
 // ---------------------------------------------------------------------------
 // Work of one CTA (kSelectThreads threads) for image i = blockIdx.x / splits:
 //  1. its output offset, the sum of the clamped keep counts of images < i,
-//  2. and, in the same round of loads, the image's candidate keys (ordered
+//  2. and, with those loads in flight, the image's candidate keys (ordered
 //     uint32 of the deletion scores) in shared memory;
 //  3. radix select, 8 bits a pass from the top: the key T of the
 //     (m-1)-th smallest candidate and how many candidates equal to T are
@@ -186,7 +186,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_keep_kernel(
   // 1-2. the image's own bounds and keep count (every thread reads the same
   // three words), its candidate keys into shared memory, and its output
   // offset, the sum of the clamped keep counts of the images before it: the
-  // loads of the keys and of the offset's terms go out in one round
+  // keys' loads and the offset's are in flight together, and the offset's
+  // block reduction is also the barrier that publishes the keys
   const int lo = cu_in[i];
   const int n = cu_in[i + 1] - lo;
   const int m = keep_counts[i];
